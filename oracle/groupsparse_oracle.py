@@ -1,0 +1,221 @@
+"""CPU oracle for the group-sparse linear layer  y = x (W (.) M)^T.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import or call
+this module: only the test-suite, the package smoke check and the benchmark's
+CPU-baseline / reference leg use it.  It shares no code with the CUDA library
+and imports nothing from it.
+
+Everything is plain numpy in float64 on the exact bf16 values (bf16 widens to
+float64 without rounding).  Each function follows one definition:
+
+* group partition and mask expansion, Sec. 2.1 and Eq. 1:
+  M = B (x) 1_{g_out x g_in},  W_hat = W (.) M
+* sparsity accounting, Eq. 2: s^l = 1 - sum(B^l) / (G_out G_in),
+  s = sum_l s^l d_out d_in / sum_l d_out d_in
+* the layer output: y = x W_hat^T (the linear projection the masked weight
+  replaces; no bias), computed as one float64 matrix product
+* the packed layout (chunk-major kept-row lists, weight tiles, offsets), which
+  the paper leaves unspecified; the layout is defined by the sequential loop in
+  `pack` below.
+
+Readings where the paper is silent (all listed in the design notes):
+* groups are 1 x 256 along the input dimension, aligned at multiples of 256;
+* M acts as a select, so a pruned weight is +0.0 (bit pattern 0x0000) even
+  where W is negative;
+* a nonzero mask byte means "keep".
+
+Parity pins: every function here is pinned by the `-m "not gpu"` tests in
+tests/test_oracle_pins.py (exact integer cases, complement and disjoint-union
+identities, one-hot masks, permutation equivariance, hand-derived golden
+layouts, closed-form sparsities).
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, Iterable, List, Sequence, Tuple
+
+import numpy as np
+
+G_IN = 256
+WIN16 = 16   # row-window height of the per-(chunk, window) metadata in the packed layout
+
+
+def _bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    bits = np.ascontiguousarray(bits, dtype=np.uint16)
+    return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 1: mask expansion and masked weight
+# ---------------------------------------------------------------------------
+
+def expand_mask(B: np.ndarray, g_out: int = 1, g_in: int = G_IN) -> np.ndarray:
+    """M = B (x) 1_{g_out x g_in} (Kronecker product, Eq. 1) as a boolean matrix."""
+    B = (np.asarray(B) != 0).astype(np.uint8)
+    return np.kron(B, np.ones((g_out, g_in), dtype=np.uint8)).astype(bool)
+
+
+def masked_weight(W_bits: np.ndarray, B: np.ndarray, g_out: int = 1, g_in: int = G_IN) -> np.ndarray:
+    """W_hat = W (.) M in float64 (Eq. 1); pruned entries are +0.0."""
+    W = _bf16_to_f64(W_bits)
+    M = expand_mask(B, g_out, g_in)
+    if M.shape != W.shape:
+        raise ValueError(f"mask expands to {M.shape}, weight is {W.shape}")
+    return np.where(M, W, 0.0)
+
+
+def masked_weight_bits(W_bits: np.ndarray, B: np.ndarray, g_out: int = 1, g_in: int = G_IN) -> np.ndarray:
+    """W_hat as bf16 bits: W's bits where kept, 0x0000 (+0.0) where pruned."""
+    W_bits = np.asarray(W_bits, dtype=np.uint16)
+    M = expand_mask(B, g_out, g_in)
+    return np.where(M, W_bits, np.uint16(0)).astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# the layer: y = x W_hat^T
+# ---------------------------------------------------------------------------
+
+def linear(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray) -> Tuple[np.ndarray, np.ndarray]:
+    """y[t, r] = sum_k x[t, k] W_hat[r, k] in float64, and the magnitude sum
+    A[t, r] = sum_k |x[t, k] W_hat[r, k]| that scales the acceptance bound.
+
+    x_bits: uint16 [T, in] bf16 bits; W_bits: uint16 [out, in]; B: [out, in/256].
+    """
+    x = _bf16_to_f64(x_bits)
+    What = masked_weight(W_bits, B)
+    if x.ndim != 2 or x.shape[1] != What.shape[1]:
+        raise ValueError("x must be [T, in]")
+    y = x @ What.T
+    A = np.abs(x) @ np.abs(What).T
+    return y, A
+
+
+def linear_tokens(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray,
+                  tokens: Sequence[int]) -> Tuple[np.ndarray, np.ndarray]:
+    """`linear` restricted to the listed token rows of x."""
+    idx = np.asarray(list(tokens), dtype=np.int64)
+    return linear(np.asarray(x_bits)[idx], W_bits, B)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 2: sparsity accounting
+# ---------------------------------------------------------------------------
+
+def layer_sparsity(B: np.ndarray) -> float:
+    """s^l = 1 - sum_uv B_uv / (G_out G_in)."""
+    B = (np.asarray(B) != 0)
+    return 1.0 - float(B.sum()) / float(B.size)
+
+
+def global_sparsity(Bs: Iterable[np.ndarray], shapes: Iterable[Tuple[int, int]]) -> float:
+    """s = sum_l s^l d_out d_in / sum_l d_out d_in (parameter-weighted mean)."""
+    num = 0.0
+    den = 0.0
+    for B, (d_out, d_in) in zip(Bs, shapes):
+        num += layer_sparsity(B) * d_out * d_in
+        den += d_out * d_in
+    return num / den
+
+
+def preserved_rate(B: np.ndarray, g_out: int = 1, g_in: int = G_IN) -> float:
+    """Active weights / total weights after applying the binary mask (App. F)."""
+    M = expand_mask(B, g_out, g_in)
+    return float(M.sum()) / float(M.size)
+
+
+# ---------------------------------------------------------------------------
+# packed layout (chunk-major kept-row lists)
+# ---------------------------------------------------------------------------
+
+@dataclasses.dataclass
+class Packed:
+    out: int
+    inp: int
+    offsets: np.ndarray     # int64 [G+1]; chunk c owns packed rows [offsets[c], offsets[c+1])
+    row_idx: np.ndarray     # int32 [K]; ascending kept rows of each chunk
+    tiles: np.ndarray       # uint16 [K, 256]; tiles[j] = W[row_idx[j], 256c : 256c+256]
+    win_off16: np.ndarray   # int32 [G, nw16+1]; first packed row of window w (rows 16w..) in chunk c
+    kmask16: np.ndarray     # uint16 [G, nw16]; bit i = row 16w+i kept in chunk c
+
+    @property
+    def G(self) -> int:
+        return self.inp // G_IN
+
+    @property
+    def kept(self) -> int:
+        return int(self.offsets[-1])
+
+
+def pack(W_bits: np.ndarray, B: np.ndarray) -> Packed:
+    """Chunk-major packing: for chunk c = 0..G-1, for row r = 0..out-1 in ascending
+    order, if B[r, c] keeps the group, append r to the row list and the 256
+    weights W[r, 256c : 256c+256] (bit copy) to the tiles."""
+    W_bits = np.asarray(W_bits, dtype=np.uint16)
+    keep = np.asarray(B) != 0
+    out, inp = W_bits.shape
+    if inp % G_IN != 0:
+        raise ValueError("in must be a multiple of 256")
+    G = inp // G_IN
+    if keep.shape != (out, G):
+        raise ValueError("mask must be [out, in/256]")
+    rows: List[int] = []
+    tiles: List[np.ndarray] = []
+    offsets = [0]
+    for c in range(G):
+        for r in range(out):
+            if keep[r, c]:
+                rows.append(r)
+                tiles.append(W_bits[r, G_IN * c: G_IN * (c + 1)])
+        offsets.append(len(rows))
+    nw16 = (out + WIN16 - 1) // WIN16
+    win_off16 = np.zeros((G, nw16 + 1), dtype=np.int32)
+    kmask16 = np.zeros((G, nw16), dtype=np.uint16)
+    for c in range(G):
+        pos = offsets[c]
+        for w in range(nw16):
+            win_off16[c, w] = pos
+            bits = 0
+            for i in range(WIN16):
+                r = WIN16 * w + i
+                if r < out and keep[r, c]:
+                    bits |= 1 << i
+                    pos += 1
+            kmask16[c, w] = bits
+        win_off16[c, nw16] = pos
+        assert pos == offsets[c + 1]
+    return Packed(out=out, inp=inp,
+                  offsets=np.asarray(offsets, dtype=np.int64),
+                  row_idx=np.asarray(rows, dtype=np.int32),
+                  tiles=(np.stack(tiles) if tiles else np.zeros((0, G_IN), np.uint16)).astype(np.uint16),
+                  win_off16=win_off16, kmask16=kmask16)
+
+
+def unpack(p: Packed) -> np.ndarray:
+    """Scatter the packed tiles back to a dense [out, in] bf16 matrix; groups that are
+    not in the row lists stay +0.0 (0x0000)."""
+    W = np.zeros((p.out, p.inp), dtype=np.uint16)
+    for c in range(p.G):
+        for j in range(int(p.offsets[c]), int(p.offsets[c + 1])):
+            r = int(p.row_idx[j])
+            W[r, G_IN * c: G_IN * (c + 1)] = p.tiles[j]
+    return W
+
+
+def linear_packed(x_bits: np.ndarray, p: Packed) -> np.ndarray:
+    """y from the packed layout: for every kept group (c, row_idx[j]), add the float64
+    dot product of its 256 weights with x[:, 256c : 256c+256]; groups are visited in
+    packed order, the 256 products of one group are summed left to right."""
+    x = _bf16_to_f64(x_bits)
+    T = x.shape[0]
+    y = np.zeros((T, p.out), dtype=np.float64)
+    tiles = _bf16_to_f64(p.tiles)
+    for c in range(p.G):
+        xc = x[:, G_IN * c: G_IN * (c + 1)]
+        for j in range(int(p.offsets[c]), int(p.offsets[c + 1])):
+            r = int(p.row_idx[j])
+            for t in range(T):
+                acc = 0.0
+                for k in range(G_IN):
+                    acc += xc[t, k] * tiles[j, k]
+                y[t, r] += acc
+    return y

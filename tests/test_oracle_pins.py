@@ -1,0 +1,275 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Each test targets a plausible mistake: a dropped or extra group, a wrong sign,
+a transposed operand or mask, a wrong group orientation, a wrong packing order.
+Sources of truth: hand-derived golden fixtures (tests/golden), exact integer
+arithmetic (Python / numpy int64), correctly rounded sums (math.fsum), brute
+force over every mask of tiny layers, and identities that Eq. 1 implies
+(complement, disjoint union, permutation equivariance, scaling).
+"""
+import itertools
+import json
+import math
+from pathlib import Path
+
+import numpy as np
+import pytest
+
+from oracle import groupsparse_oracle as orc
+from paper_2609_33977_gb300 import workload as wl
+
+GOLDEN = Path(__file__).resolve().parent / "golden"
+
+
+def bits_of(a):
+    return wl.f32_to_bf16_bits(np.asarray(a, dtype=np.float32))
+
+
+def const_groups(vals, width=256):
+    """Expand a [rows, G] table of constants into a [rows, G*width] bf16 bit matrix."""
+    v = np.repeat(np.asarray(vals, dtype=np.float32), width, axis=1)
+    return bits_of(v)
+
+
+def int_bits(rng, shape, lo=-4, hi=4):
+    """bf16 bits of small integers (exact in bf16), and the integers."""
+    ints = rng.integers(lo, hi + 1, size=shape)
+    return bits_of(ints.astype(np.float32)), ints.astype(np.int64)
+
+
+def int_reference(x_int, W_int, B):
+    """Exact y via int64 arithmetic, summing kept groups chunk by chunk."""
+    T = x_int.shape[0]
+    out, G = B.shape
+    y = np.zeros((T, out), dtype=np.int64)
+    for r in range(out):
+        for c in range(G):
+            if B[r, c]:
+                y[:, r] += x_int[:, 256 * c:256 * (c + 1)] @ W_int[r, 256 * c:256 * (c + 1)]
+    return y
+
+
+# --------------------------------------------------------------------- golden
+
+def test_golden_tiny_layer():
+    g = json.loads((GOLDEN / "tiny_layer.json").read_text())
+    B = np.asarray(g["mask"], dtype=np.uint8)
+    W = const_groups(g["W_const"])
+    x = const_groups(g["x_const"])
+    assert W.shape == (g["out"], g["in"])
+    y, A = orc.linear(x, W, B)
+    e = g["expected"]
+    assert np.array_equal(y, np.asarray(e["y"]))
+    assert np.array_equal(A, np.asarray(e["A"]))
+    p = orc.pack(W, B)
+    assert p.offsets.tolist() == e["offsets"]
+    assert p.row_idx.tolist() == e["row_idx"]
+    assert np.array_equal(p.tiles, const_groups(np.asarray(e["tile_const"])[:, None]))
+    assert p.kmask16.tolist() == e["kmask16"]
+    assert p.win_off16.tolist() == e["win_off16"]
+    assert orc.layer_sparsity(B) == pytest.approx(e["layer_sparsity"], abs=0, rel=1e-15)
+
+
+def test_golden_global_sparsity():
+    g = json.loads((GOLDEN / "global_sparsity.json").read_text())
+    Bs = [np.asarray(l["mask"]) for l in g["layers"]]
+    shapes = [(l["d_out"], l["d_in"]) for l in g["layers"]]
+    for B, l in zip(Bs, g["layers"]):
+        assert orc.layer_sparsity(B) == l["s"]
+    assert orc.global_sparsity(Bs, shapes) == g["s_global"]
+
+
+# --------------------------------------------------------------------- exact integer cases
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_exact_integer_layer(seed):
+    rng = np.random.default_rng(seed)
+    out, inp, T = 5, 768, 3
+    xb, xi = int_bits(rng, (T, inp))
+    Wb, Wi = int_bits(rng, (out, inp))
+    B = (rng.random((out, inp // 256)) < 0.5).astype(np.uint8)
+    y, A = orc.linear(xb, Wb, B)
+    yi = int_reference(xi, Wi, B)
+    assert np.array_equal(y, yi.astype(np.float64))
+    Ai = int_reference(np.abs(xi), np.abs(Wi), B)
+    assert np.array_equal(A, Ai.astype(np.float64))
+
+
+def test_brute_force_every_mask_tiny():
+    rng = np.random.default_rng(7)
+    out, inp, T = 2, 512, 2
+    xb, xi = int_bits(rng, (T, inp), -8, 8)
+    Wb, Wi = int_bits(rng, (out, inp), -8, 8)
+    G = inp // 256
+    for bits in itertools.product([0, 1], repeat=out * G):
+        B = np.asarray(bits, dtype=np.uint8).reshape(out, G)
+        y, _ = orc.linear(xb, Wb, B)
+        assert np.array_equal(y, int_reference(xi, Wi, B).astype(np.float64)), bits
+
+
+def test_all_kept_is_dense_product_and_all_pruned_is_zero():
+    rng = np.random.default_rng(3)
+    out, inp, T = 4, 1024, 3
+    xb, xi = int_bits(rng, (T, inp))
+    Wb, Wi = int_bits(rng, (out, inp))
+    ones = np.ones((out, inp // 256), np.uint8)
+    y, _ = orc.linear(xb, Wb, ones)
+    assert np.array_equal(y, (xi @ Wi.T).astype(np.float64))      # B = 1: the dense teacher
+    y0, A0 = orc.linear(xb, Wb, np.zeros_like(ones))
+    assert not np.any(y0) and not np.any(A0)
+
+
+def test_complement_and_disjoint_union():
+    rng = np.random.default_rng(4)
+    out, inp, T = 6, 1280, 2
+    xb, _ = int_bits(rng, (T, inp))
+    Wb, _ = int_bits(rng, (out, inp))
+    G = inp // 256
+    B1 = (rng.random((out, G)) < 0.3).astype(np.uint8)
+    B2 = ((rng.random((out, G)) < 0.5) & (B1 == 0)).astype(np.uint8)
+    y1, _ = orc.linear(xb, Wb, B1)
+    y2, _ = orc.linear(xb, Wb, B2)
+    y12, _ = orc.linear(xb, Wb, B1 | B2)
+    yc, _ = orc.linear(xb, Wb, 1 - B1)
+    yd, _ = orc.linear(xb, Wb, np.ones_like(B1))
+    assert np.array_equal(y1 + y2, y12)
+    assert np.array_equal(y1 + yc, yd)
+
+
+def test_one_hot_group_orientation():
+    """Keeping a single group (r0, c0) must touch only output r0 and only input
+    columns 256*c0 .. 256*c0+255 (groups run along the input dimension)."""
+    rng = np.random.default_rng(5)
+    out, inp, T = 3, 768, 2
+    xb = wl.random_activation_bits(T, inp, seed=11)
+    Wb = wl.random_weight_bits(out, inp, seed=12)
+    x = wl.bf16_bits_to_f64(xb)
+    W = wl.bf16_bits_to_f64(Wb)
+    for r0 in range(out):
+        for c0 in range(inp // 256):
+            B = np.zeros((out, inp // 256), np.uint8)
+            B[r0, c0] = 1
+            y, _ = orc.linear(xb, Wb, B)
+            for t in range(T):
+                for r in range(out):
+                    if r != r0:
+                        assert y[t, r] == 0.0
+                ref = math.fsum(x[t, 256 * c0 + k] * W[r0, 256 * c0 + k] for k in range(256))
+                assert y[t, r0] == pytest.approx(ref, rel=1e-13, abs=1e-300)
+
+
+def test_against_correctly_rounded_sums():
+    out, inp, T = 4, 768, 3
+    xb = wl.random_activation_bits(T, inp, seed=21)
+    Wb = wl.random_weight_bits(out, inp, seed=22)
+    B = wl.random_mask(out, inp // 256, 0.6, seed=23)
+    x = wl.bf16_bits_to_f64(xb)
+    W = wl.bf16_bits_to_f64(Wb)
+    y, A = orc.linear(xb, Wb, B)
+    for t in range(T):
+        for r in range(out):
+            terms = [x[t, 256 * c + k] * W[r, 256 * c + k]
+                     for c in range(inp // 256) if B[r, c] for k in range(256)]
+            ref = math.fsum(terms)
+            aref = math.fsum(abs(v) for v in terms)
+            assert abs(y[t, r] - ref) <= 1e-14 * aref + 1e-300
+            assert A[t, r] == pytest.approx(aref, rel=1e-14, abs=0)
+            assert abs(y[t, r]) <= A[t, r]
+
+
+def test_permutation_equivariance_and_scaling():
+    rng = np.random.default_rng(6)
+    out, inp, T = 5, 1024, 3
+    xb, _ = int_bits(rng, (T, inp))
+    Wb, _ = int_bits(rng, (out, inp))
+    G = inp // 256
+    B = (rng.random((out, G)) < 0.5).astype(np.uint8)
+    y, _ = orc.linear(xb, Wb, B)
+    # permuting output rows (W rows and mask rows) permutes y's columns
+    pr = rng.permutation(out)
+    yp, _ = orc.linear(xb, Wb[pr], B[pr])
+    assert np.array_equal(yp, y[:, pr])
+    # permuting whole 256-wide chunks of x, W and the mask columns leaves y unchanged
+    pc = rng.permutation(G)
+    cols = np.concatenate([np.arange(256 * c, 256 * (c + 1)) for c in pc])
+    yc, _ = orc.linear(xb[:, cols], Wb[:, cols], B[:, pc])
+    assert np.array_equal(yc, y)
+    # permuting tokens permutes y's rows; scaling x by 2 scales y by 2 (exact in binary)
+    pt = rng.permutation(T)
+    yt, _ = orc.linear(xb[pt], Wb, B)
+    assert np.array_equal(yt, y[pt])
+    x2 = bits_of(wl.bf16_bits_to_f32(xb) * np.float32(2.0))
+    y2, _ = orc.linear(x2, Wb, B)
+    assert np.array_equal(y2, 2.0 * y)
+
+
+# --------------------------------------------------------------------- packing
+
+@pytest.mark.parametrize("out,inp,d,seed", [(1, 256, 1.0, 0), (17, 512, 0.5, 1), (40, 1280, 0.3, 2),
+                                             (33, 768, 0.0, 3), (64, 256, 1.0, 4)])
+def test_pack_invariants_and_roundtrip(out, inp, d, seed):
+    Wb = wl.random_weight_bits(out, inp, seed=seed)
+    B = wl.random_mask(out, inp // 256, d, seed=seed + 100)
+    p = orc.pack(Wb, B)
+    G = inp // 256
+    assert p.offsets[0] == 0 and p.kept == int(B.sum())
+    assert np.all(np.diff(p.offsets) == B.sum(axis=0))               # n_c = #kept rows of chunk c
+    for c in range(G):
+        rows = p.row_idx[p.offsets[c]:p.offsets[c + 1]]
+        assert np.all(np.diff(rows) > 0)                              # ascending, distinct
+        assert all(B[r, c] for r in rows)
+        for j, r in zip(range(p.offsets[c], p.offsets[c + 1]), rows):
+            assert np.array_equal(p.tiles[j], Wb[r, 256 * c:256 * (c + 1)])
+    # window metadata: brute force from the mask
+    nw16 = (out + 15) // 16
+    for c in range(G):
+        for w in range(nw16):
+            rows = [r for r in range(16 * w, min(16 * w + 16, out)) if B[r, c]]
+            assert p.kmask16[c, w] == sum(1 << (r - 16 * w) for r in rows)
+            assert p.win_off16[c, w] == p.offsets[c] + int(B[:16 * w, c].sum())
+        assert p.win_off16[c, nw16] == p.offsets[c + 1]
+    # unpack reproduces W (.) M bit-exactly, pruned = +0.0
+    assert np.array_equal(orc.unpack(p), orc.masked_weight_bits(Wb, B))
+
+
+def test_masked_weight_uses_positive_zero():
+    Wb = bits_of(-np.ones((2, 512), np.float32))
+    B = np.array([[1, 0], [0, 1]], np.uint8)
+    Wh = orc.masked_weight_bits(Wb, B)
+    assert np.all(Wh[0, 256:] == 0) and np.all(Wh[1, :256] == 0)
+    assert np.all(Wh[0, :256] == 0xBF80) and np.all(Wh[1, 256:] == 0xBF80)
+    assert np.all(np.signbit(orc.masked_weight(Wb, B)) == (Wh == 0xBF80))
+
+
+def test_packed_route_equals_definition():
+    out, inp, T = 6, 768, 2
+    xb = wl.random_activation_bits(T, inp, seed=31)
+    Wb = wl.random_weight_bits(out, inp, seed=32)
+    B = wl.random_mask(out, inp // 256, 0.5, seed=33)
+    y, A = orc.linear(xb, Wb, B)
+    yp = orc.linear_packed(xb, orc.pack(Wb, B))
+    assert np.all(np.abs(yp - y) <= 1e-14 * A + 1e-300)
+
+
+# --------------------------------------------------------------------- Eq. 2 / App. F
+
+def test_sparsity_closed_forms():
+    assert orc.layer_sparsity(np.ones((4, 3))) == 0.0
+    assert orc.layer_sparsity(np.zeros((4, 3))) == 1.0
+    B = np.zeros((8, 4), np.uint8)
+    B[:, :2] = 1
+    assert orc.layer_sparsity(B) == 0.5
+    # with 1x256 groups every group holds 256 weights: preserved rate = 1 - s^l
+    rng = np.random.default_rng(0)
+    B = (rng.random((10, 6)) < 0.37).astype(np.uint8)
+    assert orc.preserved_rate(B) == pytest.approx(1.0 - orc.layer_sparsity(B), abs=1e-15)
+    # square groups (g_out = g_in = 2): each selector covers 4 weights
+    Bs = np.array([[1, 0], [0, 0]])
+    assert orc.expand_mask(Bs, 2, 2).sum() == 4 and orc.expand_mask(Bs, 2, 2)[:2, :2].all()
+
+
+def test_bf16_rounding_helper():
+    # round-to-nearest-even on hand-picked values
+    v = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, 1.0 + 2 ** -7, -2.5, 0.0], np.float32)
+    assert wl.f32_to_bf16_bits(v).tolist() == [0x3F80, 0x3F80, 0x3F82, 0x3F81, 0xC020, 0x0000]
+    assert np.array_equal(wl.bf16_bits_to_f32(np.array([0x3F80, 0xC020], np.uint16)), np.array([1.0, -2.5], np.float32))

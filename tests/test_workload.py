@@ -1,0 +1,78 @@
+"""Seeded workload generator: budgets, determinism, shapes (no method arithmetic here)."""
+import numpy as np
+import pytest
+
+from oracle import groupsparse_oracle as orc
+from paper_2609_33977_gb300 import workload as wl
+
+
+def test_config_group_counts_and_budgets():
+    assert wl.workload(1).total_groups == 4096 and wl.workload(1).budget == 2048
+    assert wl.workload(2).total_groups == 790528 and wl.workload(2).budget == 395264
+    assert wl.workload(3).total_groups == 25296896 and wl.workload(3).budget == 12648448
+    assert wl.workload(4).total_groups == 49561600 and wl.workload(4).budget == 24780800
+    w5 = wl.workload(5, 0.5)
+    assert w5.total_groups == 25489408
+    for d in (0.3, 0.5, 0.7):
+        assert wl.workload(5, d).budget == int(np.floor(d * 25489408 + 0.5))
+    assert {l.G for l in wl.workload(5).layers[:7]} == {14, 74}
+
+
+@pytest.mark.parametrize("cfg,d", [(1, 0.5), (2, 0.5), (3, 0.5), (4, 0.5), (5, 0.3), (5, 0.5), (5, 0.7)])
+def test_keep_counts_hit_budget_exactly(cfg, d):
+    w = wl.workload(cfg, d)
+    k = wl.keep_counts(w)
+    N = np.array([l.groups for l in w.layers])
+    assert int(k.sum()) == w.budget
+    assert np.all(k >= 0) and np.all(k <= N)
+    if w.ratio_range is not None:
+        # layer-adaptive: per-layer densities spread out around the global one
+        dens = k / N
+        assert dens.std() > 0.05
+    assert np.array_equal(k, wl.keep_counts(w))     # deterministic
+
+
+def test_allocation_edge_cases():
+    assert wl.allocate_keep_counts([10, 10], [1.0, 1.0], 20).tolist() == [10, 10]
+    assert wl.allocate_keep_counts([10, 10], [0.5, 0.5], 0).tolist() == [0, 0]
+    k = wl.allocate_keep_counts([100, 10], [0.9, 0.9], 105)       # second layer saturates
+    assert k.tolist() == [95, 10]
+    with pytest.raises(ValueError):
+        wl.allocate_keep_counts([10], [0.5], 11)
+
+
+def test_block_masks_meet_budget_and_eq2():
+    """Masks of the one-block workload keep exactly the allocated groups; the
+    parameter-weighted sparsity of Eq. 2 then equals 1 - K*/N because every
+    1x256 group holds the same number of weights."""
+    w = wl.workload(2)
+    k = wl.keep_counts(w)
+    masks = [wl.group_mask(w, i, int(k[i])) for i in range(len(w.layers))]
+    for m, ki, L in zip(masks, k, w.layers):
+        assert m.shape == (L.out, L.G) and int(m.sum()) == ki
+    s = orc.global_sparsity(masks, [(L.out, L.inp) for L in w.layers])
+    assert s == pytest.approx(1.0 - w.budget / w.total_groups, abs=1e-12)
+    assert np.array_equal(masks[0], wl.group_mask(w, 0, int(k[0])))
+
+
+def test_weights_and_activations_distribution():
+    w = wl.workload(1)
+    Wb = wl.weight_bits(w, 0)
+    W = wl.bf16_bits_to_f64(Wb)
+    assert W.shape == (1024, 1024)
+    assert abs(W.std() - 0.02) < 5e-4 and abs(W.mean()) < 1e-3
+    xb = wl.activation_bits(w, 0, 8)
+    assert xb.shape == (8, 1024)
+    assert np.array_equal(Wb, wl.weight_bits(w, 0))
+
+
+def test_outlier_channels():
+    w = wl.workload(3, blocks=1)
+    L = w.layers[0]
+    ch = wl.outlier_channels(w, 0)
+    assert ch.size == 41                    # 1 % of 4096 channels
+    x = wl.bf16_bits_to_f64(wl.activation_bits(w, 0, 64))
+    big = np.abs(x[:, ch]).mean()
+    rest = np.abs(np.delete(x, ch, axis=1)).mean()
+    assert 15 < big / rest < 25
+    assert wl.outlier_channels(w, 6).size == 110   # down_proj: 1 % of 11008
