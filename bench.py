@@ -1,0 +1,536 @@
+#!/usr/bin/env python
+"""Throughput benchmark of the group-sparse linear layer y = x (W (.) M)^T.
+
+Workload: one LLaMA-2-7B-shaped decoder block (q/k/v/o 4096x4096, gate/up
+11008x4096, down 4096x11008), bf16 weights ~ N(0, 0.02^2), 1x256 groups along
+the input dimension, per-module keep ratios U[0.3, 0.7] rescaled so the block
+keeps exactly 50 % of its 790,528 groups, decode batches of 1, 4 and 16 tokens.
+
+One step = the seven projections at T = 1, 4 and 16 (three batched launches of
+the decode kernel, 21 tokens through the block), on one of R rotated packed
+copies so that the weights streamed per step never sit in L2.  Packing is a
+one-time transform of frozen weights and is timed separately ("pack").  The
+tensor-core prefill kernel is measured on the first block of the 7B stack at
+T = 2048 with activation outliers ("prefill").
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+N > 1 runs under torch.distributed.run: each rank holds an independent replica
+(the layer shards into independent problems, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+from pathlib import Path
+
+import numpy as np
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+from paper_2609_33977_gb300 import workload as wl  # noqa: E402
+
+METRIC = "group-sparse linear tokens/s; decode HBM GB/s and prefill TFLOP/s vs GB300 peak"
+DECODE_T = (1, 4, 16)
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def load_peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, interval_ms: int = 50):
+        self.gpu = gpu_index
+        self.interval = interval_ms
+        self.proc = None
+        self.path = Path(os.environ.get("TMPDIR", "/tmp")) / f"gs_clocks_{os.getpid()}.csv"
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 f"-lms={self.interval}"], stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        for line in self.path.read_text().splitlines():
+            parts = [s.strip() for s in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        try:
+            self.path.unlink()
+        except OSError:
+            pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max((float(r[3]) for r in rows if r[3].replace(".", "").isdigit()), default=None)}
+
+
+# ----------------------------------------------------------------------------- traffic record
+def kernel_source_hash(name: str) -> str:
+    return hashlib.sha256((ROOT / "paper_2609_33977_gb300" / "csrc" / name).read_bytes()).hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, source: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel source is unchanged since."""
+    p = ROOT / "profiles" / "traffic.json"
+    if not p.exists():
+        return None
+    try:
+        d = json.loads(p.read_text())
+        e = d.get(kernel, {}).get(workload)
+        if e and e.get("source_sha256_16") == kernel_source_hash(source):
+            return e["dram_bytes_per_launch"]
+    except Exception:
+        return None
+    return None
+
+
+# ----------------------------------------------------------------------------- workload
+def block_inputs():
+    w = wl.workload(2)
+    k = wl.keep_counts(w)
+    layers = []
+    for i, L in enumerate(w.layers):
+        layers.append({"L": L, "k": int(k[i]), "W": wl.weight_bits(w, i), "B": wl.group_mask(w, i, int(k[i])),
+                       "x": {T: wl.activation_bits(w, i, T) for T in DECODE_T}})
+    return w, layers
+
+
+def decode_bytes(layers, T):
+    """Algorithmic bytes of one decode launch over the block: kept weights + the index
+    metadata the kernel reads (16-bit window mask + 32-bit offset per chunk x 16-row
+    window) + x + y."""
+    b = 0
+    for d in layers:
+        L = d["L"]
+        nw16 = (L.out + 15) // 16
+        b += 512 * d["k"] + 6 * L.G * nw16 + 2 * T * L.inp + 2 * T * L.out
+    return b
+
+
+# ----------------------------------------------------------------------------- CPU oracle timing
+def oracle_sample_rate(layers, seconds: float, rows_per_call: int = 256):
+    """Times the fp64 oracle on bounded samples: one token through `rows_per_call`
+    output rows of one projection per call, rotating over the projections, for
+    about `seconds`.  Returns block tokens/s extrapolated by weight count."""
+    from oracle import groupsparse_oracle as orc
+    total_weights = sum(d["L"].out * d["L"].inp for d in layers)
+    done_weights = 0
+    t_used = 0.0
+    calls = 0
+    i = 0
+    t_end = time.perf_counter() + seconds
+    while time.perf_counter() < t_end or calls < len(layers):
+        d = layers[i % len(layers)]
+        L = d["L"]
+        r0 = (calls * 977) % max(1, L.out - rows_per_call)
+        rows = slice(r0, r0 + rows_per_call)
+        x1 = d["x"][1]
+        t0 = time.perf_counter()
+        orc.linear(x1, d["W"][rows], d["B"][rows])
+        t_used += time.perf_counter() - t0
+        done_weights += rows_per_call * L.inp
+        calls += 1
+        i += 1
+    sec_per_weight = t_used / done_weights
+    tokens_per_s = 1.0 / (sec_per_weight * total_weights)
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max((p.get("num_threads", 1) for p in threadpool_info()), default=1)
+    except Exception:
+        cores = os.cpu_count() or 1
+    return {"value": tokens_per_s, "unit": "tokens/s", "cores": int(cores), "kind": "oracle",
+            "sample": f"{calls} oracle calls, each 1 token x {rows_per_call} output rows of one projection "
+                      f"(rotating over the 7), {t_used:.1f} s of CPU work; block tokens/s extrapolated by "
+                      f"weight count ({total_weights} weights per block)"}
+
+
+# ----------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    _, layers = block_inputs()
+    from oracle import groupsparse_oracle as orc
+    total_weights = sum(d["L"].out * d["L"].inp for d in layers)
+    rows_per_step = 64
+
+    def one(i):
+        d = layers[i % len(layers)]
+        L = d["L"]
+        r0 = (i * 977) % max(1, L.out - rows_per_step)
+        orc.linear(d["x"][1], d["W"][r0:r0 + rows_per_step], d["B"][r0:r0 + rows_per_step])
+        return rows_per_step * L.inp
+
+    for i in range(args.warmup):
+        one(i)
+    t0 = time.perf_counter()
+    weights = 0
+    for i in range(args.steps):
+        weights += one(i)
+    dt = time.perf_counter() - t0
+    tokens_per_s = weights / total_weights / dt
+    sample = (f"each step: the fp64 oracle on 1 token x {rows_per_step} output rows of one projection "
+              f"(rotating over the 7); block tokens/s extrapolated by weight count")
+    line = {"impl": "reference", "metric": METRIC, "value": tokens_per_s, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / max(1, args.steps),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "llama2-7b-block decode T=1 (sampled rows)", "layers": 7},
+            "cpu_baseline": {"value": tokens_per_s, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": tokens_per_s, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+
+    peaks, peaks_src = load_peaks()
+    t_gen = time.perf_counter()
+    w, layers = block_inputs()
+    log(f"[bench] inputs generated in {time.perf_counter() - t_gen:.1f}s")
+
+    def dev_bits(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    Wd = [dev_bits(d["W"]) for d in layers]
+    Md = [torch.from_numpy(d["B"]).to(dev) for d in layers]
+
+    # ---- pack (one-time transform), timed on its own
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    packs0 = [gs.pack(Wd[i], Md[i]) for i in range(len(layers))]
+    torch.cuda.synchronize()
+    pack_s = time.perf_counter() - t0
+    kept = sum(p.kept for p in packs0)
+    assert kept == w.budget, (kept, w.budget)
+    pack_bytes = sum(512 * d["k"] * 2 + d["L"].groups + 6 * d["L"].G * ((d["L"].out + 15) // 16) + 4 * d["k"]
+                     for d in layers)
+
+    # ---- rotated copies so each step streams weights that are not L2-resident
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    kept_bytes = 512 * kept
+    R = max(2, int(math.ceil(3 * l2 / kept_bytes)) + 1) if args.rotate <= 0 else args.rotate
+    packs = [packs0] + [[gs.pack(Wd[i], Md[i]) for i in range(len(layers))] for _ in range(R - 1)]
+    xs = {T: [dev_bits(d["x"][T]) for d in layers] for T in DECODE_T}
+    ys = {T: [torch.empty((T, d["L"].out), dtype=torch.bfloat16, device=dev) for d in layers] for T in DECODE_T}
+
+    stream = torch.cuda.Stream(device=dev)
+    graphs = []
+    with torch.cuda.stream(stream):
+        for c in range(R):                       # warm-up launches outside capture
+            for T in DECODE_T:
+                gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
+        stream.synchronize()
+        for c in range(R):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for T in DECODE_T:
+                    gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
+            graphs.append(g)
+    stream.synchronize()
+    launches_per_step = len(DECODE_T)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    # ---- warm-up, then exactly K timed steps
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            graphs[i % R].replay()
+    stream.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize(dev)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    n0 = gs.launch_count()
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        for i in range(args.steps):
+            graphs[i % R].replay()
+        ev1.record(stream)
+    ev1.synchronize()
+    torch.cuda.synchronize(dev)
+    barrier()
+    clock_rec = clocks.stop()
+    # graph replays do not go through the library's launch counter: count the
+    # kernels they contain (one decode launch per token batch per step)
+    launches = args.steps * launches_per_step + (gs.launch_count() - n0)
+    elapsed = ev0.elapsed_time(ev1) / 1e3
+    if dist is not None:
+        t = torch.tensor([elapsed], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    tokens_per_step = sum(DECODE_T)
+    value = world * tokens_per_step * args.steps / elapsed
+    bytes_per_step = sum(decode_bytes(layers, T) for T in DECODE_T)
+    achieved_gbs = bytes_per_step * args.steps / elapsed / 1e9
+
+    # ---- per-T kernel timing (decode alone, one graph per T) for the breakdown
+    per_T = {}
+    with torch.cuda.stream(stream):
+        for T in DECODE_T:
+            gT = []
+            for c in range(R):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
+                gT.append(g)
+            n = max(50, min(2000, args.steps))
+            for i in range(10):
+                gT[i % R].replay()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for i in range(n):
+                gT[i % R].replay()
+            b.record(stream)
+            b.synchronize()
+            us = a.elapsed_time(b) * 1e3 / n
+            per_T[str(T)] = {"us_per_launch": us, "GB/s": decode_bytes(layers, T) / us / 1e3,
+                             "tokens/s": T / us * 1e6}
+
+    # ---- end to end through the public API with host buffers
+    xh = {T: torch.cat([xx.reshape(-1) for xx in xs[T]]).cpu().pin_memory() for T in DECODE_T}
+    xd_flat = {T: torch.empty_like(xh[T], device=dev) for T in DECODE_T}
+    xd_views = {}
+    for T in DECODE_T:
+        off = 0
+        views = []
+        for d in layers:
+            n = T * d["L"].inp
+            views.append(xd_flat[T][off:off + n].view(T, d["L"].inp))
+            off += n
+        xd_views[T] = views
+    yd_flat = {T: torch.empty(sum(T * d["L"].out for d in layers), dtype=torch.bfloat16, device=dev)
+               for T in DECODE_T}
+    yd_views = {}
+    for T in DECODE_T:
+        off = 0
+        views = []
+        for d in layers:
+            n = T * d["L"].out
+            views.append(yd_flat[T][off:off + n].view(T, d["L"].out))
+            off += n
+        yd_views[T] = views
+    yh = {T: torch.empty(yd_flat[T].shape, dtype=torch.bfloat16).pin_memory() for T in DECODE_T}
+    h2d = sum(xh[T].numel() * 2 for T in DECODE_T)
+    d2h = sum(yh[T].numel() * 2 for T in DECODE_T)
+    e2e_steps = max(20, min(args.steps, 2000))
+    with torch.cuda.stream(stream):
+        def e2e_step(i):
+            c = i % R
+            for T in DECODE_T:
+                xd_flat[T].copy_(xh[T], non_blocking=True)
+                gs.linear_batched_into(xd_views[T], packs[c], yd_views[T], stream=stream)
+                yh[T].copy_(yd_flat[T], non_blocking=True)
+        for i in range(5):
+            e2e_step(i)
+        stream.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(e2e_steps):
+            e2e_step(i)
+        b.record(stream)
+        b.synchronize()
+    e2e_s = a.elapsed_time(b) / 1e3
+    e2e_value = world * tokens_per_step * e2e_steps / e2e_s
+    # results of the e2e path equal the device-resident path
+    for T in DECODE_T:
+        assert torch.equal(yh[T].to(dev), torch.cat([yy.reshape(-1) for yy in ys[T]])), "e2e result mismatch"
+
+    # ---- dense bf16 torch matmul on the unpruned weights (reference point)
+    dense = {}
+    with torch.cuda.stream(stream):
+        for T in DECODE_T:
+            Wd_rot = [Wd] + [[wt.clone() for wt in Wd] for _ in range(1)]
+            for i in range(5):
+                for j, d in enumerate(layers):
+                    torch.matmul(xs[T][j], Wd_rot[i % 2][j].t())
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            n = 50
+            a.record(stream)
+            for i in range(n):
+                for j, d in enumerate(layers):
+                    torch.matmul(xs[T][j], Wd_rot[i % 2][j].t())
+            b.record(stream)
+            b.synchronize()
+            us = a.elapsed_time(b) * 1e3 / n
+            dense[str(T)] = {"us_per_block": us, "tokens/s": T / us * 1e6}
+            del Wd_rot
+    torch.cuda.empty_cache()
+
+    # ---- tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
+    prefill = None
+    if not args.no_prefill:
+        prefill = measure_prefill(gs, torch, dev, stream, peaks)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = oracle_sample_rate(layers, args.cpu_seconds)
+
+    hbm_peak = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    traffic = recorded_traffic("k_decode", "gs_decode.cu", "llama2-7b-block")
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "llama2-7b-block decode: 7 projections x T=1,4,16 (21 tokens per step)",
+                   "layers": 7, "kept_groups": kept, "total_groups": w.total_groups, "density": kept / w.total_groups,
+                   "kept_weight_bytes": kept_bytes,
+                   "l2": f"inputs larger than L2: {R} rotated packed copies ({R * kept_bytes / 1e6:.0f} MB) vs "
+                         f"L2 {l2 / 1e6:.0f} MB", "parallelism": f"replicas x{world}", "graph": "one CUDA graph per step"},
+        "roofline": {"kernel": "k_decode", "bound": "hbm", "achieved": achieved_gbs, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved_gbs / hbm_peak, "peak_source": f"{peaks_src} hbm_gbs",
+                     "bytes_per_step": bytes_per_step, "traffic": traffic,
+                     "frac_of_8TBs_nominal": achieved_gbs / 8000.0},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "steps": e2e_steps, "how": "pinned host x -> device, gs_linear_batched, device y -> pinned host; "
+                                         "per token batch, through the Python binding (no graph)"},
+        "gpu_launches": launches,
+        "clocks": clock_rec,
+        "per_T": per_T,
+        "dense_torch_bf16": dense,
+        "pack": {"seconds": pack_s, "layers": 7, "GB/s_incl_alloc_and_sync": pack_bytes / pack_s / 1e9},
+        "prefill": prefill,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def measure_prefill(gs, torch, dev, stream, peaks):
+    w = wl.workload(3, blocks=1)
+    k = wl.keep_counts(w)
+    T = 2048
+    # device-side draws of the same distributions (numpy draws of 7 full layers are slow)
+    Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
+    Bd = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in range(7)]
+    xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
+    ps = [gs.pack(Wd[i], Bd[i]) for i in range(7)]
+    ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
+    kept = sum(p.kept for p in ps)
+    flops = 2.0 * T * 256 * kept
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            for i in range(7):
+                gs.linear_into(xd[i], ps[i], ys[i], algo=gs.ALGO_PREFILL, stream=stream)
+        n = 10
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n):
+            for i in range(7):
+                gs.linear_into(xd[i], ps[i], ys[i], algo=gs.ALGO_PREFILL, stream=stream)
+        b.record(stream)
+        b.synchronize()
+        s_block = a.elapsed_time(b) / 1e3 / n
+        # dense bf16 reference point on the unpruned weights
+        for i in range(7):
+            torch.matmul(xd[i], Wd[i].t())
+        a.record(stream)
+        for _ in range(n):
+            for i in range(7):
+                torch.matmul(xd[i], Wd[i].t())
+        b.record(stream)
+        b.synchronize()
+        s_dense = a.elapsed_time(b) / 1e3 / n
+    tflops = flops / s_block / 1e12
+    peak = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
+    dense_flops = 2.0 * T * sum(L.out * L.inp for L in w.layers)
+    assert gs.device_status() == gs.GS_OK
+    out = {"workload": "llama2-7b block 0 (7 projections), T=2048, 1% outlier channels x20, layer-adaptive 50%",
+           "kept_groups": kept, "kept_tflop_per_block": flops / 1e12, "ms_per_block": s_block * 1e3,
+           "tokens/s": T / s_block, "TFLOP/s": tflops, "peak_TFLOP/s": peak, "frac": tflops / peak,
+           "peak_source": "measured bf16_tflops (burst)",
+           "dense_torch_ms_per_block": s_dense * 1e3,
+           "dense_torch_TFLOP/s": dense_flops / s_dense / 1e12, "speedup_vs_dense": s_dense / s_block}
+    del Wd, Bd, xd, ps, ys
+    torch.cuda.empty_cache()
+    return out
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--rotate", type=int, default=0, help="rotated packed copies (0 = enough to exceed 3x L2)")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

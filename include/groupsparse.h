@@ -1,0 +1,154 @@
+/*
+ * groupsparse.h - C ABI of the GB300 group-sparse linear layer.
+ *
+ * The layer is the pruned projection of GroupMask (Sec. 2.1, Eq. 1):
+ *     M = B (x) 1_{1 x 256},   W_hat = W (.) M,   y = x W_hat^T
+ * W[out][in] is a frozen bf16 weight, B[out][in/256] keeps (nonzero) or prunes
+ * (zero) each 1x256 group of W, and x[T][in] holds T tokens.  Pruned groups are
+ * never read: the weight is first packed into a chunk-major compressed layout
+ * (gs_pack), then every gs_linear call streams only the kept groups.
+ *
+ * Conventions shared by every call:
+ *   - Pointers named *_dev are device pointers (cudaMalloc'd or equivalent) on
+ *     the current CUDA device; pointers named *_host are host pointers.
+ *   - bf16 tensors are passed as raw 16-bit storage (void*), row-major, densely
+ *     strided.  Device tensor pointers must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls are
+ *     asynchronous on that stream unless stated otherwise.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     failed validation returns GS_ERR_INVALID_ARG or GS_ERR_UNSUPPORTED and
+ *     touches no device memory.
+ *   - The caller owns W, mask, x, y and W_hat.  The library owns the handle's
+ *     device buffers until gs_free.
+ *   - Kernels bound every wait they perform.  A wait that runs out records
+ *     GS_ERR_DEVICE_TIMEOUT in a library-owned device flag and the kernel
+ *     returns; gs_device_status reads (and clears) that flag.
+ */
+#ifndef GROUPSPARSE_H
+#define GROUPSPARSE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum gs_status {
+  GS_OK = 0,
+  GS_ERR_INVALID_ARG = 1,     /* null pointer, bad size, misaligned pointer    */
+  GS_ERR_UNSUPPORTED = 2,     /* valid request outside what is implemented     */
+  GS_ERR_OOM = 3,             /* device allocation failed                      */
+  GS_ERR_CUDA = 4,            /* a CUDA runtime/driver call or launch failed   */
+  GS_ERR_DEVICE_TIMEOUT = 5   /* a kernel's bounded wait ran out               */
+} gs_status;
+
+/* Kernel family for gs_linear_ex. */
+typedef enum gs_algo {
+  GS_ALGO_AUTO = 0,     /* pick by token count (decode for small T, else prefill)   */
+  GS_ALGO_DECODE = 1,   /* CUDA-core/mma.sync streaming kernel (memory-bound)        */
+  GS_ALGO_PREFILL = 2   /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
+} gs_algo;
+
+typedef struct gs_packed gs_packed;   /* opaque, library-owned */
+
+/*
+ * gs_pack - compress W with the group mask B into the chunk-major layout.
+ *
+ * Follows Eq. 1 (Sec. 2.1): the mask selects whole 1 x group_in groups of W;
+ * only kept groups are stored.  Packed layout (bit-exact, deterministic):
+ *   chunk c (input columns [256c, 256c+256)) owns packed rows
+ *   [offsets[c], offsets[c+1]); within a chunk the kept rows appear in
+ *   ascending row order; row_idx[j] is the output row of packed row j and
+ *   tiles[j][0:256] is a bit copy of W[row_idx[j]][256c : 256c+256].
+ *   win_off16[c][w] is the first packed row of chunk c whose output row is
+ *   >= 16w (w = 0..ceil(out/16); entry ceil(out/16) is offsets[c+1]) and
+ *   kmask16[c][w] has bit i set when row 16w+i is kept in chunk c.
+ *
+ * W_dev     bf16 [out][in] row-major, caller-owned, read only.
+ * mask_dev  uint8 [out][in/256] row-major; nonzero = keep.  Read only.
+ * out, in   out >= 1; in >= 256 and a multiple of 256; out*(in/256) < 2^31.
+ * group_in  must be 256 (other group shapes: GS_ERR_UNSUPPORTED).
+ * stream    work is queued on it; gs_pack synchronizes it once to learn the
+ *           kept-group count before allocating the packed buffers.
+ * handle    receives the new handle (set to NULL on failure).
+ * Errors: INVALID_ARG (nulls, sizes, alignment), UNSUPPORTED (group_in),
+ *         OOM, CUDA.
+ */
+gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in,
+                  int32_t group_in, void* stream, gs_packed** handle);
+
+/*
+ * gs_linear - y = x W_hat^T for the packed weight (Eq. 1 applied as a linear
+ * projection, no bias), fp32 accumulation, bf16 output rounded to nearest even.
+ *
+ * x_dev  bf16 [T][in] row-major, caller-owned, read only.
+ * p      packed handle from gs_pack (read only; may be used concurrently from
+ *        several streams).
+ * T      number of tokens; T == 0 is a no-op, T < 0 is INVALID_ARG.
+ * y_dev  bf16 [T][out] row-major, caller-owned; fully overwritten (rows of
+ *        outputs with no kept group are written as +0.0).
+ * Errors: INVALID_ARG, CUDA.  Asynchronous on `stream`.
+ */
+gs_status gs_linear(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream);
+
+/* gs_linear with an explicit kernel family (same arguments and result). */
+gs_status gs_linear_ex(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream,
+                       gs_algo algo);
+
+/*
+ * gs_linear_batched - n independent layers in one launch per kernel family:
+ * ys[i] = xs[i] W_hat_i^T for the i-th handle, all with the same token count T.
+ * Same per-layer semantics and errors as gs_linear.  n <= 64.
+ */
+gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packed* const* ps,
+                            int64_t T, void* const* ys_dev, void* stream);
+
+/*
+ * gs_unpack - the check path: W_hat_dev[r][k] = W[r][k] where the group of
+ * (r, k) is kept, +0.0 (0x0000) where it is pruned (M of Eq. 1 as a select).
+ * W_hat_dev  bf16 [out][in], caller-owned, fully overwritten.
+ * Errors: INVALID_ARG, CUDA.  Asynchronous on `stream`.
+ */
+gs_status gs_unpack(const gs_packed* p, void* W_hat_dev, void* stream);
+
+/*
+ * gs_packed_info - sizes of a handle (any output pointer may be NULL).
+ * kept_groups = offsets[G] = the number of kept groups (sum of B, Eq. 2);
+ * device_bytes = bytes of device memory the handle owns.
+ */
+gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t* kept_groups,
+                         size_t* device_bytes);
+
+/*
+ * gs_packed_export - synchronous copy of the packed layout to host buffers
+ * (for bit-exact checks).  Sizes: offsets int64[G+1], row_idx int32[K],
+ * tiles uint16[K*256], win_off16 int32[G*(ceil(out/16)+1)],
+ * kmask16 uint16[G*ceil(out/16)], with K = kept_groups.  Any pointer may be NULL.
+ */
+gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* row_idx_host,
+                           uint16_t* tiles_host, int32_t* win_off16_host, uint16_t* kmask16_host);
+
+/* Releases the handle and its device buffers (NULL is a no-op). */
+void gs_free(gs_packed* p);
+
+/* Static description of a status code. */
+const char* gs_status_string(gs_status s);
+
+/*
+ * gs_device_status - synchronizes `stream`, then reads and clears the device
+ * error flag of the current device: GS_OK or GS_ERR_DEVICE_TIMEOUT (a bounded
+ * wait in some earlier kernel ran out).  GS_ERR_CUDA if the stream itself
+ * reports an error.
+ */
+gs_status gs_device_status(void* stream);
+
+/* Number of kernel launches the library issued since the process started (all
+ * families; used to report launch counts). */
+int64_t gs_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GROUPSPARSE_H */

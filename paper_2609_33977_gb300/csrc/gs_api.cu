@@ -1,0 +1,301 @@
+// C ABI of the group-sparse linear layer: host-side validation, ownership of
+// the packed buffers, and dispatch to the pack / decode / prefill kernels.
+#include "gs_common.cuh"
+
+#include <atomic>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+namespace gs {
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_flag_mu;
+int* g_flags[kMaxDevices] = {nullptr};
+std::atomic<int64_t> g_launches{0};
+
+// Token count at and above which gs_linear uses the tensor-core kernel.
+constexpr int64_t kPrefillMinTokens = 33;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+void free_buffers(gs_packed* p) {
+  if (!p) return;
+  int cur = -1;
+  cudaGetDevice(&cur);
+  if (cur != p->device) cudaSetDevice(p->device);
+  if (p->offsets) cudaFree(p->offsets);
+  if (p->row_idx) cudaFree(p->row_idx);
+  if (p->tiles) cudaFree(p->tiles);
+  if (p->win_off16) cudaFree(p->win_off16);
+  if (p->kmask16) cudaFree(p->kmask16);
+  if (cur >= 0 && cur != p->device) cudaSetDevice(cur);
+  p->offsets = nullptr;
+  p->row_idx = nullptr;
+  p->tiles = nullptr;
+  p->win_off16 = nullptr;
+  p->kmask16 = nullptr;
+}
+
+gs_status dev_alloc(void** ptr, size_t bytes, size_t* total) {
+  *ptr = nullptr;
+  if (bytes == 0) return GS_OK;
+  const cudaError_t e = cudaMalloc(ptr, bytes);
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return GS_ERR_OOM;
+  }
+  if (e != cudaSuccess) return GS_ERR_CUDA;
+  *total += bytes;
+  return GS_OK;
+}
+
+gs_status check_handle(const gs_packed* p) {
+  if (!p) return GS_ERR_INVALID_ARG;
+  if (p->out <= 0 || p->in <= 0 || p->G <= 0 || !p->offsets || !p->win_off16 || !p->kmask16)
+    return GS_ERR_INVALID_ARG;
+  return GS_OK;
+}
+
+}  // namespace
+
+int* device_error_flag() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(g_flag_mu);
+  if (!g_flags[dev]) {
+    int* f = nullptr;
+    if (cudaMalloc(&f, sizeof(int)) != cudaSuccess) return nullptr;
+    if (cudaMemset(f, 0, sizeof(int)) != cudaSuccess) {
+      cudaFree(f);
+      return nullptr;
+    }
+    g_flags[dev] = f;
+  }
+  return g_flags[dev];
+}
+
+void note_launch(int64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+}  // namespace gs
+
+using namespace gs;
+
+extern "C" {
+
+gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t group_in,
+                  void* stream, gs_packed** handle) {
+  if (handle) *handle = nullptr;
+  if (!W_dev || !mask_dev || !handle) return GS_ERR_INVALID_ARG;
+  if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX) return GS_ERR_INVALID_ARG;
+  if (group_in != kGroupIn) return GS_ERR_UNSUPPORTED;
+  if (in % kGroupIn != 0) return GS_ERR_INVALID_ARG;
+  if (!aligned16(W_dev)) return GS_ERR_INVALID_ARG;
+  const int64_t G = in / kGroupIn;
+  if (out * G >= (int64_t)INT32_MAX) return GS_ERR_UNSUPPORTED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  gs_packed* p = new (std::nothrow) gs_packed;
+  if (!p) return GS_ERR_OOM;
+  std::memset(p, 0, sizeof(*p));
+  if (cudaGetDevice(&p->device) != cudaSuccess) {
+    delete p;
+    return GS_ERR_CUDA;
+  }
+  if (!device_error_flag()) {  // allocated here so later calls never allocate (graph capture)
+    delete p;
+    return GS_ERR_CUDA;
+  }
+  p->out = out;
+  p->in = in;
+  p->G = (int32_t)G;
+  p->nw16 = (int32_t)((out + kWin16 - 1) / kWin16);
+
+  size_t total = 0;
+  int32_t* cnt = nullptr;
+  gs_status st = GS_OK;
+  const size_t E = (size_t)p->G * (size_t)p->nw16;
+  if ((st = dev_alloc((void**)&p->offsets, sizeof(int64_t) * (size_t)(G + 1), &total)) != GS_OK) goto fail;
+  if ((st = dev_alloc((void**)&p->win_off16, sizeof(int32_t) * (size_t)p->G * (size_t)(p->nw16 + 1), &total)) !=
+      GS_OK)
+    goto fail;
+  if ((st = dev_alloc((void**)&p->kmask16, sizeof(uint16_t) * E, &total)) != GS_OK) goto fail;
+  {
+    size_t scratch = 0;
+    if ((st = dev_alloc((void**)&cnt, sizeof(int32_t) * E, &scratch)) != GS_OK) goto fail;
+  }
+  if ((st = launch_pack_count_scan(mask_dev, p, s, cnt)) != GS_OK) goto fail;
+  {
+    int64_t kept = 0;
+    if (cudaMemcpyAsync(&kept, p->offsets + G, sizeof(int64_t), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+      st = GS_ERR_CUDA;
+      goto fail;
+    }
+    p->kept = kept;
+  }
+  cudaFree(cnt);
+  cnt = nullptr;
+  if ((st = dev_alloc((void**)&p->row_idx, sizeof(int32_t) * (size_t)p->kept, &total)) != GS_OK) goto fail;
+  if ((st = dev_alloc((void**)&p->tiles, (size_t)kTileBytes * (size_t)p->kept, &total)) != GS_OK) goto fail;
+  p->device_bytes = total;
+  if ((st = launch_pack_compact(W_dev, p, s)) != GS_OK) goto fail;
+  if ((st = prefill_prepare_weight_maps(p)) != GS_OK) goto fail;
+  *handle = p;
+  return GS_OK;
+
+fail:
+  if (cnt) cudaFree(cnt);
+  free_buffers(p);
+  delete p;
+  return st;
+}
+
+static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream,
+                             gs_algo algo) {
+  if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
+  if (T < 0 || T > INT32_MAX) return GS_ERR_INVALID_ARG;
+  if (algo != GS_ALGO_AUTO && algo != GS_ALGO_DECODE && algo != GS_ALGO_PREFILL) return GS_ERR_INVALID_ARG;
+  if (T == 0) return GS_OK;
+  if (!x_dev || !y_dev) return GS_ERR_INVALID_ARG;
+  if (!aligned16(x_dev) || !aligned16(y_dev)) return GS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (algo == GS_ALGO_AUTO) algo = T >= kPrefillMinTokens ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
+  if (algo == GS_ALGO_PREFILL) return launch_prefill(x_dev, p, T, y_dev, s);
+  // decode family: token blocks of at most decode_max_tokens()
+  const int64_t blk = decode_max_tokens();
+  for (int64_t t0 = 0; t0 < T; t0 += blk) {
+    const int64_t tb = T - t0 < blk ? T - t0 : blk;
+    DecodeLayer L;
+    std::memset(&L, 0, sizeof(L));
+    L.x = static_cast<const uint16_t*>(x_dev) + t0 * p->in;
+    L.tiles = p->tiles;
+    L.win_off16 = p->win_off16;
+    L.kmask16 = p->kmask16;
+    L.y = static_cast<uint16_t*>(y_dev) + t0 * p->out;
+    L.out = (int32_t)p->out;
+    L.in = (int32_t)p->in;
+    L.G = p->G;
+    L.nw16 = p->nw16;
+    const gs_status st = launch_decode(&L, 1, (int)tb, s);
+    if (st != GS_OK) return st;
+  }
+  return GS_OK;
+}
+
+gs_status gs_linear(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream) {
+  return linear_impl(x_dev, p, T, y_dev, stream, GS_ALGO_AUTO);
+}
+
+gs_status gs_linear_ex(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream,
+                       gs_algo algo) {
+  return linear_impl(x_dev, p, T, y_dev, stream, algo);
+}
+
+gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packed* const* ps, int64_t T,
+                            void* const* ys_dev, void* stream) {
+  if (n < 0 || n > 32) return GS_ERR_INVALID_ARG;
+  if (n == 0) return GS_OK;
+  if (!xs_dev || !ps || !ys_dev) return GS_ERR_INVALID_ARG;
+  if (T < 0 || T > INT32_MAX) return GS_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    if (check_handle(ps[i]) != GS_OK) return GS_ERR_INVALID_ARG;
+    if (T > 0 && (!xs_dev[i] || !ys_dev[i] || !aligned16(xs_dev[i]) || !aligned16(ys_dev[i])))
+      return GS_ERR_INVALID_ARG;
+  }
+  if (T == 0) return GS_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (T >= kPrefillMinTokens) {
+    for (int i = 0; i < n; ++i) {
+      const gs_status st = launch_prefill(xs_dev[i], ps[i], T, ys_dev[i], s);
+      if (st != GS_OK) return st;
+    }
+    return GS_OK;
+  }
+  std::vector<DecodeLayer> L(n);
+  for (int i = 0; i < n; ++i) {
+    std::memset(&L[i], 0, sizeof(DecodeLayer));
+    L[i].x = static_cast<const uint16_t*>(xs_dev[i]);
+    L[i].tiles = ps[i]->tiles;
+    L[i].win_off16 = ps[i]->win_off16;
+    L[i].kmask16 = ps[i]->kmask16;
+    L[i].y = static_cast<uint16_t*>(ys_dev[i]);
+    L[i].out = (int32_t)ps[i]->out;
+    L[i].in = (int32_t)ps[i]->in;
+    L[i].G = ps[i]->G;
+    L[i].nw16 = ps[i]->nw16;
+  }
+  return launch_decode(L.data(), n, (int)T, s);
+}
+
+gs_status gs_unpack(const gs_packed* p, void* W_hat_dev, void* stream) {
+  if (check_handle(p) != GS_OK || !W_hat_dev || !aligned16(W_hat_dev)) return GS_ERR_INVALID_ARG;
+  return launch_unpack(p, W_hat_dev, static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t* kept_groups,
+                         size_t* device_bytes) {
+  if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
+  if (out) *out = p->out;
+  if (in) *in = p->in;
+  if (kept_groups) *kept_groups = p->kept;
+  if (device_bytes) *device_bytes = p->device_bytes;
+  return GS_OK;
+}
+
+gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* row_idx_host, uint16_t* tiles_host,
+                           int32_t* win_off16_host, uint16_t* kmask16_host) {
+  if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
+  const size_t G = (size_t)p->G, nw = (size_t)p->nw16, K = (size_t)p->kept;
+  if (offsets_host && cudaMemcpy(offsets_host, p->offsets, sizeof(int64_t) * (G + 1), cudaMemcpyDeviceToHost))
+    return GS_ERR_CUDA;
+  if (row_idx_host && K && cudaMemcpy(row_idx_host, p->row_idx, sizeof(int32_t) * K, cudaMemcpyDeviceToHost))
+    return GS_ERR_CUDA;
+  if (tiles_host && K && cudaMemcpy(tiles_host, p->tiles, (size_t)kTileBytes * K, cudaMemcpyDeviceToHost))
+    return GS_ERR_CUDA;
+  if (win_off16_host &&
+      cudaMemcpy(win_off16_host, p->win_off16, sizeof(int32_t) * G * (nw + 1), cudaMemcpyDeviceToHost))
+    return GS_ERR_CUDA;
+  if (kmask16_host && cudaMemcpy(kmask16_host, p->kmask16, sizeof(uint16_t) * G * nw, cudaMemcpyDeviceToHost))
+    return GS_ERR_CUDA;
+  return GS_OK;
+}
+
+void gs_free(gs_packed* p) {
+  if (!p) return;
+  free_buffers(p);
+  delete p;
+}
+
+const char* gs_status_string(gs_status s) {
+  switch (s) {
+    case GS_OK: return "ok";
+    case GS_ERR_INVALID_ARG: return "invalid argument";
+    case GS_ERR_UNSUPPORTED: return "unsupported";
+    case GS_ERR_OOM: return "out of device memory";
+    case GS_ERR_CUDA: return "CUDA error";
+    case GS_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+gs_status gs_device_status(void* stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return GS_ERR_CUDA;
+  int* f = device_error_flag();
+  if (!f) return GS_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, f, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return GS_ERR_CUDA;
+  if (v != 0) {
+    cudaMemset(f, 0, sizeof(int));
+    return GS_ERR_DEVICE_TIMEOUT;
+  }
+  return GS_OK;
+}
+
+int64_t gs_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+}  // extern "C"

@@ -1,0 +1,69 @@
+// Shared definitions of the CUDA path (library side only).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+#include <cstddef>
+
+#include "../../include/groupsparse.h"
+
+namespace gs {
+
+constexpr int kGroupIn = 256;     // g_in of the 1x256 groups (Sec. 2.1)
+constexpr int kWin16 = 16;        // row-window height of the per-(chunk, window) metadata
+constexpr int kTileBytes = kGroupIn * 2;   // one packed group: 256 bf16 = 512 B
+
+// Device-error codes written into the library's device flag.
+constexpr int kDevErrTimeout = 1;
+
+}  // namespace gs
+
+// Library-owned packed weight.  All arrays live on `device`.
+struct gs_packed {
+  int device;
+  int64_t out, in;
+  int32_t G;          // in / 256
+  int32_t nw16;       // ceil(out / 16)
+  int64_t kept;       // offsets[G]
+  int64_t* offsets;   // [G+1]
+  int32_t* row_idx;   // [kept]
+  uint16_t* tiles;    // [kept][256]
+  int32_t* win_off16; // [G][nw16+1]
+  uint16_t* kmask16;  // [G][nw16]
+  size_t device_bytes;
+  // tcgen05 prefill: TMA descriptors over the tiles (box heights 128/64/32/16 rows)
+  alignas(64) unsigned char wmaps[4][128];
+  bool wmaps_valid;
+};
+
+namespace gs {
+
+// library-owned per-device error flag (allocated on first use)
+int* device_error_flag();
+void note_launch(int64_t n = 1);
+
+// pack.cu
+gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t s, int32_t* cnt_tmp);
+gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s);
+gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
+
+// decode.cu
+struct DecodeLayer {
+  const uint16_t* x;        // [T][in]
+  const uint16_t* tiles;    // [kept][256]
+  const int32_t* win_off16; // [G][nw16+1]
+  const uint16_t* kmask16;  // [G][nw16]
+  uint16_t* y;              // [T][out]
+  int32_t out, in, G, nw16;
+  int32_t cta_begin;        // first CTA of this layer in the launch
+  int32_t nblk;             // ceil(out / 128)
+};
+gs_status launch_decode(const DecodeLayer* layers, int n, int T, cudaStream_t s);
+int decode_max_tokens();
+
+// prefill.cu
+gs_status prefill_prepare_weight_maps(gs_packed* p);
+gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, cudaStream_t s);
+
+}  // namespace gs

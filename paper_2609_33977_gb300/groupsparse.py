@@ -1,0 +1,201 @@
+"""Python binding of libgroupsparse.so (argument marshalling only).
+
+Every call goes straight to the C ABI declared in include/groupsparse.h; torch
+is used for device memory and the current CUDA stream.  There is no fallback:
+if the compiled library is missing or fails to load, importing this module
+raises.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+_PKG = Path(__file__).resolve().parent
+LIB_PATH = _PKG / "libgroupsparse.so"
+
+GS_OK, GS_ERR_INVALID_ARG, GS_ERR_UNSUPPORTED, GS_ERR_OOM, GS_ERR_CUDA, GS_ERR_DEVICE_TIMEOUT = range(6)
+ALGO_AUTO, ALGO_DECODE, ALGO_PREFILL = 0, 1, 2
+
+_c_i64p = ctypes.POINTER(ctypes.c_int64)
+_c_i32p = ctypes.POINTER(ctypes.c_int32)
+_c_u16p = ctypes.POINTER(ctypes.c_uint16)
+
+
+def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
+    if not path.exists():
+        raise ImportError(f"{path} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(str(path))
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    lib.gs_pack.argtypes = [vp, vp, i64, i64, i32, vp, ctypes.POINTER(vp)]
+    lib.gs_linear.argtypes = [vp, vp, i64, vp, vp]
+    lib.gs_linear_ex.argtypes = [vp, vp, i64, vp, vp, ctypes.c_int]
+    lib.gs_linear_batched.argtypes = [i32, ctypes.POINTER(vp), ctypes.POINTER(vp), i64, ctypes.POINTER(vp), vp]
+    lib.gs_unpack.argtypes = [vp, vp, vp]
+    lib.gs_packed_info.argtypes = [vp, _c_i64p, _c_i64p, _c_i64p, ctypes.POINTER(ctypes.c_size_t)]
+    lib.gs_packed_export.argtypes = [vp, _c_i64p, _c_i32p, _c_u16p, _c_i32p, _c_u16p]
+    lib.gs_free.argtypes = [vp]
+    lib.gs_free.restype = None
+    lib.gs_status_string.argtypes = [ctypes.c_int]
+    lib.gs_status_string.restype = ctypes.c_char_p
+    lib.gs_device_status.argtypes = [vp]
+    lib.gs_launch_count.argtypes = []
+    lib.gs_launch_count.restype = ctypes.c_int64
+    for fn in (lib.gs_pack, lib.gs_linear, lib.gs_linear_ex, lib.gs_linear_batched, lib.gs_unpack,
+               lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status):
+        fn.restype = ctypes.c_int
+    return lib
+
+
+lib = _load()
+
+
+class GroupSparseError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {lib.gs_status_string(status).decode()} (status {status})")
+        self.status = status
+
+
+def _check(status: int, what: str) -> None:
+    if status != GS_OK:
+        raise GroupSparseError(status, what)
+
+
+def _stream_ptr(stream: Optional[torch.cuda.Stream] = None) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _require_cuda(t: torch.Tensor, dtype: torch.dtype, name: str) -> None:
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+class Packed:
+    """A packed group-sparse weight (owns the library handle)."""
+
+    def __init__(self, handle: int, out: int, inp: int):
+        self._h = ctypes.c_void_p(handle)
+        self.out = out
+        self.inp = inp
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if not self._h:
+            raise ValueError("packed weight already freed")
+        return self._h
+
+    @property
+    def G(self) -> int:
+        return self.inp // 256
+
+    def info(self):
+        out, inp, kept = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+        nbytes = ctypes.c_size_t()
+        _check(lib.gs_packed_info(self.handle, ctypes.byref(out), ctypes.byref(inp), ctypes.byref(kept),
+                                  ctypes.byref(nbytes)), "gs_packed_info")
+        return {"out": out.value, "in": inp.value, "kept": kept.value, "device_bytes": nbytes.value}
+
+    @property
+    def kept(self) -> int:
+        return self.info()["kept"]
+
+    def export(self):
+        """Host copies of the packed layout: offsets, row_idx, tiles, win_off16, kmask16."""
+        K = self.kept
+        G = self.G
+        nw16 = (self.out + 15) // 16
+        offsets = np.zeros(G + 1, np.int64)
+        row_idx = np.zeros(max(K, 1), np.int32)
+        tiles = np.zeros((max(K, 1), 256), np.uint16)
+        win = np.zeros((G, nw16 + 1), np.int32)
+        km = np.zeros((G, nw16), np.uint16)
+        _check(lib.gs_packed_export(self.handle, offsets.ctypes.data_as(_c_i64p), row_idx.ctypes.data_as(_c_i32p),
+                                    tiles.ctypes.data_as(_c_u16p), win.ctypes.data_as(_c_i32p),
+                                    km.ctypes.data_as(_c_u16p)), "gs_packed_export")
+        return {"offsets": offsets, "row_idx": row_idx[:K], "tiles": tiles[:K], "win_off16": win, "kmask16": km}
+
+    def free(self) -> None:
+        if self._h:
+            lib.gs_free(self._h)
+            self._h = ctypes.c_void_p(None)
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def pack(W: torch.Tensor, mask: torch.Tensor, stream: Optional[torch.cuda.Stream] = None) -> Packed:
+    """Pack a bf16 weight [out, in] with a uint8/bool group mask [out, in/256] (nonzero = keep)."""
+    _require_cuda(W, torch.bfloat16, "W")
+    if mask.dtype == torch.bool:
+        mask = mask.to(torch.uint8)
+    _require_cuda(mask, torch.uint8, "mask")
+    out, inp = W.shape
+    if tuple(mask.shape) != (out, inp // 256):
+        raise ValueError("mask must be [out, in/256]")
+    h = ctypes.c_void_p()
+    _check(lib.gs_pack(W.data_ptr(), mask.data_ptr(), out, inp, 256, _stream_ptr(stream), ctypes.byref(h)),
+           "gs_pack")
+    return Packed(h.value, out, inp)
+
+
+def linear_into(x: torch.Tensor, p: Packed, y: torch.Tensor, algo: int = ALGO_AUTO,
+                stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    _require_cuda(x, torch.bfloat16, "x")
+    _require_cuda(y, torch.bfloat16, "y")
+    T = x.shape[0]
+    if x.dim() != 2 or x.shape[1] != p.inp or tuple(y.shape) != (T, p.out):
+        raise ValueError("x must be [T, in] and y [T, out]")
+    _check(lib.gs_linear_ex(x.data_ptr(), p.handle, T, y.data_ptr(), _stream_ptr(stream), algo), "gs_linear")
+    return y
+
+
+def linear(x: torch.Tensor, p: Packed, algo: int = ALGO_AUTO, stream: Optional[torch.cuda.Stream] = None):
+    """y = x (W (.) M)^T as bf16 [T, out]."""
+    y = torch.empty((x.shape[0], p.out), dtype=torch.bfloat16, device=x.device)
+    return linear_into(x, p, y, algo, stream)
+
+
+def linear_batched_into(xs: Sequence[torch.Tensor], ps: Sequence[Packed], ys: Sequence[torch.Tensor],
+                        stream: Optional[torch.cuda.Stream] = None) -> None:
+    n = len(ps)
+    if not (len(xs) == len(ys) == n):
+        raise ValueError("xs, ps, ys must have the same length")
+    if n == 0:
+        return
+    T = xs[0].shape[0]
+    for x, p, y in zip(xs, ps, ys):
+        _require_cuda(x, torch.bfloat16, "x")
+        _require_cuda(y, torch.bfloat16, "y")
+        if x.shape[0] != T or x.shape[1] != p.inp or tuple(y.shape) != (T, p.out):
+            raise ValueError("every x must be [T, in_i] and y [T, out_i] with one T")
+    arr = ctypes.c_void_p * n
+    xa = arr(*[x.data_ptr() for x in xs])
+    pa = arr(*[p.handle.value for p in ps])
+    ya = arr(*[y.data_ptr() for y in ys])
+    _check(lib.gs_linear_batched(n, xa, pa, T, ya, _stream_ptr(stream)), "gs_linear_batched")
+
+
+def unpack(p: Packed, stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """W_hat = W (.) M as bf16 [out, in]; pruned groups are +0.0."""
+    W = torch.empty((p.out, p.inp), dtype=torch.bfloat16, device="cuda")
+    _check(lib.gs_unpack(p.handle, W.data_ptr(), _stream_ptr(stream)), "gs_unpack")
+    return W
+
+
+def device_status(stream: Optional[torch.cuda.Stream] = None) -> int:
+    return int(lib.gs_device_status(_stream_ptr(stream)))
+
+
+def launch_count() -> int:
+    return int(lib.gs_launch_count())

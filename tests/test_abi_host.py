@@ -1,0 +1,74 @@
+"""The C-ABI library loads, exports every symbol include/*.h declares, and rejects
+bad arguments on the host before touching any device (no GPU needed)."""
+import ctypes
+import re
+from pathlib import Path
+
+import pytest
+
+ROOT = Path(__file__).resolve().parent.parent
+
+
+def declared_functions():
+    names = set()
+    for h in (ROOT / "include").glob("*.h"):
+        text = re.sub(r"/\*.*?\*/", "", h.read_text(), flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w\s\*]*?\b(gs_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib(built_lib):
+    return ctypes.CDLL(str(built_lib))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("gs_pack", "gs_linear", "gs_unpack", "gs_free", "gs_packed_info", "gs_status_string"):
+        assert required in names
+    assert len(names) >= 10
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_binding_loads(built_lib):
+    from paper_2609_33977_gb300 import groupsparse as gs
+    assert gs.lib.gs_status_string(0) == b"ok"
+    assert gs.lib.gs_status_string(5) == b"device wait timed out"
+
+
+def test_host_side_validation(lib):
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    lib.gs_pack.argtypes = [vp, vp, i64, i64, i32, vp, ctypes.POINTER(vp)]
+    lib.gs_linear.argtypes = [vp, vp, i64, vp, vp]
+    lib.gs_linear_ex.argtypes = [vp, vp, i64, vp, vp, ctypes.c_int]
+    lib.gs_unpack.argtypes = [vp, vp, vp]
+    lib.gs_linear_batched.argtypes = [i32, vp, vp, i64, vp, vp]
+    lib.gs_packed_info.argtypes = [vp, vp, vp, vp, vp]
+    lib.gs_packed_export.argtypes = [vp, vp, vp, vp, vp, vp]
+    lib.gs_free.argtypes = [vp]
+    lib.gs_free.restype = None
+    h = vp(12345)
+    fake = 0x10000  # never dereferenced: each call below fails validation first
+    INVALID, UNSUPPORTED = 1, 2
+    assert lib.gs_pack(None, fake, 4, 256, 256, None, ctypes.byref(h)) == INVALID
+    assert h.value is None                                            # handle cleared on failure
+    assert lib.gs_pack(fake, None, 4, 256, 256, None, ctypes.byref(h)) == INVALID
+    assert lib.gs_pack(fake, fake, 4, 256, 256, None, None) == INVALID
+    assert lib.gs_pack(fake, fake, 0, 256, 256, None, ctypes.byref(h)) == INVALID
+    assert lib.gs_pack(fake, fake, 4, 300, 256, None, ctypes.byref(h)) == INVALID   # in % 256 != 0
+    assert lib.gs_pack(fake, fake, 4, 256, 128, None, ctypes.byref(h)) == UNSUPPORTED
+    assert lib.gs_pack(fake + 2, fake, 4, 256, 256, None, ctypes.byref(h)) == INVALID  # misaligned W
+    assert lib.gs_linear(fake, None, 4, fake, None) == INVALID
+    assert lib.gs_linear_ex(fake, None, 4, fake, None, 7) == INVALID
+    assert lib.gs_unpack(None, fake, None) == INVALID
+    assert lib.gs_linear_batched(-1, None, None, 1, None, None) == INVALID
+    assert lib.gs_linear_batched(33, fake, fake, 1, fake, None) == INVALID
+    assert lib.gs_linear_batched(0, None, None, 1, None, None) == 0
+    assert lib.gs_packed_info(None, None, None, None, None) == INVALID
+    assert lib.gs_packed_export(None, None, None, None, None, None) == INVALID
+    lib.gs_free(None)

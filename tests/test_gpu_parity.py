@@ -1,0 +1,202 @@
+"""CUDA path vs the CPU oracle, through the C ABI (pack / linear / unpack).
+
+Packing and unpacking must match bit for bit; y must satisfy
+|y - y_oracle| <= 2^-7 * sum_kept |x w| + 1e-6 element-wise.
+"""
+import numpy as np
+import pytest
+
+from oracle import groupsparse_oracle as orc
+from paper_2609_33977_gb300 import workload as wl
+from tests._gpu_util import assert_within_bound, sample_tokens, to_bits, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def gs(built_lib):
+    import torch
+    assert torch.cuda.is_available(), "the -m gpu tests need a CUDA device"
+    from paper_2609_33977_gb300 import groupsparse
+    return groupsparse
+
+
+_cache = {}
+
+
+def layer(out, inp, d, seed):
+    key = (out, inp, d, seed)
+    if key not in _cache:
+        Wb = wl.random_weight_bits(out, inp, seed=seed)
+        B = wl.random_mask(out, inp // 256, d, seed=seed + 1000)
+        _cache[key] = (Wb, B)
+    return _cache[key]
+
+
+def packed(gs, Wb, B):
+    import torch
+    return gs.pack(to_dev(Wb), torch.from_numpy(np.ascontiguousarray(B, dtype=np.uint8)).cuda())
+
+
+PACK_SHAPES = [(1, 256, 1.0, 1), (17, 512, 0.5, 2), (300, 768, 0.5, 3), (1024, 1024, 0.5, 4),
+               (512, 3584, 0.3, 5), (4096, 4096, 0.5, 6), (11008, 4096, 0.45, 7), (4096, 11008, 0.5, 8),
+               (129, 256, 0.0, 9), (200, 2048, 1.0, 10)]
+
+
+@pytest.mark.parametrize("out,inp,d,seed", PACK_SHAPES)
+def test_pack_and_unpack_bit_exact(gs, out, inp, d, seed):
+    Wb, B = layer(out, inp, d, seed)
+    p = packed(gs, Wb, B)
+    ref = orc.pack(Wb, B)
+    got = p.export()
+    assert p.kept == ref.kept == int(B.sum())
+    assert np.array_equal(got["offsets"], ref.offsets)
+    assert np.array_equal(got["row_idx"], ref.row_idx)
+    assert np.array_equal(got["tiles"], ref.tiles)
+    assert np.array_equal(got["win_off16"], ref.win_off16)
+    assert np.array_equal(got["kmask16"], ref.kmask16)
+    assert np.array_equal(to_bits(gs.unpack(p)), orc.masked_weight_bits(Wb, B))
+
+
+def test_pack_is_deterministic(gs):
+    Wb, B = layer(4096, 4096, 0.5, 6)
+    a = packed(gs, Wb, B).export()
+    b = packed(gs, Wb, B).export()
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+DECODE_SHAPES = [(300, 768, 0.5, 3), (1024, 1024, 0.5, 4), (512, 3584, 0.3, 5), (4096, 4096, 0.5, 6),
+                 (4096, 11008, 0.5, 8), (17, 512, 0.5, 2), (129, 256, 0.0, 9), (200, 2048, 1.0, 10)]
+DECODE_T = list(range(1, 18)) + [24, 31, 32, 33, 64, 65, 100]
+
+
+@pytest.mark.parametrize("out,inp,d,seed", DECODE_SHAPES)
+def test_decode_parity(gs, out, inp, d, seed):
+    Wb, B = layer(out, inp, d, seed)
+    p = packed(gs, Wb, B)
+    for T in DECODE_T:
+        xb = wl.random_activation_bits(T, inp, seed=seed * 100 + T)
+        y = gs.linear(to_dev(xb), p, algo=gs.ALGO_DECODE)
+        assert_within_bound(to_bits(y), xb, Wb, B, what=f"decode {out}x{inp} d={d} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
+PREFILL_SHAPES = [(300, 768, 0.5, 3), (1024, 1024, 0.5, 4), (640, 2560, 0.9, 11), (520, 512, 0.05, 12),
+                  (256, 4096, 1.0, 13), (1000, 1280, 0.0, 14), (4096, 4096, 0.5, 6), (17, 512, 0.5, 2)]
+PREFILL_T = [1, 7, 64, 127, 128, 129, 255, 256, 300, 513]
+
+
+@pytest.mark.parametrize("out,inp,d,seed", PREFILL_SHAPES)
+def test_prefill_parity(gs, out, inp, d, seed):
+    Wb, B = layer(out, inp, d, seed)
+    p = packed(gs, Wb, B)
+    for T in PREFILL_T:
+        xb = wl.random_activation_bits(T, inp, seed=seed * 100 + T + 7)
+        y = gs.linear(to_dev(xb), p, algo=gs.ALGO_PREFILL)
+        assert_within_bound(to_bits(y), xb, Wb, B, what=f"prefill {out}x{inp} d={d} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
+def test_auto_dispatch_and_empty_batch(gs):
+    import torch
+    Wb, B = layer(1024, 1024, 0.5, 4)
+    p = packed(gs, Wb, B)
+    for T in (1, 16, 32, 33, 200):
+        xb = wl.random_activation_bits(T, 1024, seed=T)
+        assert_within_bound(to_bits(gs.linear(to_dev(xb), p)), xb, Wb, B, what=f"auto T={T}")
+    x0 = torch.empty((0, 1024), dtype=torch.bfloat16, device="cuda")
+    assert gs.linear(x0, p).shape == (0, 1024)
+
+
+def test_deterministic_outputs(gs):
+    Wb, B = layer(4096, 4096, 0.5, 6)
+    p = packed(gs, Wb, B)
+    for T, algo in ((16, gs.ALGO_DECODE), (1, gs.ALGO_DECODE), (300, gs.ALGO_PREFILL)):
+        x = to_dev(wl.random_activation_bits(T, 4096, seed=5))
+        a = to_bits(gs.linear(x, p, algo=algo))
+        b = to_bits(gs.linear(x, p, algo=algo))
+        assert np.array_equal(a, b)
+
+
+def test_single_layer_workload(gs):
+    """1024x1024 layer, exactly half of its 4096 groups kept, 8 tokens."""
+    w = wl.workload(1)
+    k = wl.keep_counts(w)
+    Wb = wl.weight_bits(w, 0)
+    B = wl.group_mask(w, 0, int(k[0]))
+    xb = wl.activation_bits(w, 0, 8)
+    p = packed(gs, Wb, B)
+    assert p.kept == 2048
+    for algo in (gs.ALGO_AUTO, gs.ALGO_DECODE, gs.ALGO_PREFILL):
+        assert_within_bound(to_bits(gs.linear(to_dev(xb), p, algo=algo)), xb, Wb, B, what=f"cfg1 algo={algo}")
+
+
+def test_block_workload_decode_batched(gs):
+    """One LLaMA-2-7B-shaped block (7 projections, exactly 50 % of groups kept),
+    decode with 1, 4 and 16 tokens, all layers in one batched launch."""
+    import torch
+    w = wl.workload(2)
+    k = wl.keep_counts(w)
+    Ws, Bs, ps = [], [], []
+    for i in range(len(w.layers)):
+        Wb = wl.weight_bits(w, i)
+        B = wl.group_mask(w, i, int(k[i]))
+        Ws.append(Wb)
+        Bs.append(B)
+        ps.append(packed(gs, Wb, B))
+    assert sum(p.kept for p in ps) == w.budget
+    for T in w.tokens:
+        xs = [wl.activation_bits(w, i, T) for i in range(len(w.layers))]
+        xd = [to_dev(x) for x in xs]
+        ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device="cuda") for L in w.layers]
+        gs.linear_batched_into(xd, ps, ys)
+        ys2 = [torch.empty_like(y) for y in ys]
+        gs.linear_batched_into(xd, ps, ys2)
+        for i in range(len(w.layers)):
+            assert torch.equal(ys[i], ys2[i])          # deterministic for a fixed launch configuration
+            assert_within_bound(to_bits(ys[i]), xs[i], Ws[i], Bs[i], what=f"cfg2 {w.layers[i].name} T={T}")
+            # the single-layer call may split chunks differently (another fp32 order)
+            y1 = gs.linear(xd[i], ps[i])
+            assert_within_bound(to_bits(y1), xs[i], Ws[i], Bs[i], what=f"cfg2 single {w.layers[i].name} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
+@pytest.mark.parametrize("cfg,T", [(3, 2048), (4, 512), (5, 1024)])
+def test_stack_shapes_prefill_sampled(gs, cfg, T):
+    """First block of the 7B (with activation outliers), 13B and Qwen stacks at
+    prefill token counts; every layer checked on a deterministic token sample."""
+    w = wl.workload(cfg, 0.5)
+    k = wl.keep_counts(w)
+    for i in range(7):
+        Wb = wl.weight_bits(w, i)
+        B = wl.group_mask(w, i, int(k[i]))
+        xb = wl.activation_bits(w, i, T)
+        p = packed(gs, Wb, B)
+        y = to_bits(gs.linear(to_dev(xb), p))
+        assert_within_bound(y, xb, Wb, B, tokens=sample_tokens(T, seed=i),
+                            what=f"cfg{cfg} {w.layers[i].name} T={T}")
+        del p
+    assert gs.device_status() == gs.GS_OK
+
+
+def test_graph_capture_replay(gs):
+    import torch
+    Wb, B = layer(4096, 4096, 0.5, 6)
+    p = packed(gs, Wb, B)
+    for T, algo in ((16, gs.ALGO_DECODE), (256, gs.ALGO_PREFILL)):
+        x = to_dev(wl.random_activation_bits(T, 4096, seed=T))
+        y = torch.empty((T, 4096), dtype=torch.bfloat16, device="cuda")
+        ref = to_bits(gs.linear(x, p, algo=algo))
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            gs.linear_into(x, p, y, algo=algo)   # warm-up outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        g = torch.cuda.CUDAGraph()
+        y.zero_()
+        with torch.cuda.graph(g):
+            gs.linear_into(x, p, y, algo=algo)
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(to_bits(y), ref)
