@@ -514,6 +514,85 @@ def measure_prefill(gs, torch, dev, stream, peaks):
     return out
 
 
+def run_layer(args):
+    """One synthetic layer (random mask of the given density), one kernel family,
+    timed with CUDA events; prints one JSON line.  Used for sweeps and for the
+    small cases that ncu captures."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+    T = args.tokens
+    dev = torch.device("cuda", 0)
+    if args.layer == "llama2-7b-block":
+        return run_block_layers(args, gs, torch, dev)
+    out, inp = (int(v) for v in args.layer.lower().split("x"))
+    g = torch.Generator(device=dev)
+    g.manual_seed(1234)
+    W = (torch.randn((out, inp), generator=g, device=dev) * 0.02).to(torch.bfloat16)
+    B = (torch.rand((out, inp // 256), generator=g, device=dev) < args.density).to(torch.uint8)
+    x = torch.randn((T, inp), generator=g, device=dev).to(torch.bfloat16)
+    p = gs.pack(W, B)
+    y = torch.empty((T, out), dtype=torch.bfloat16, device=dev)
+    algo = {"auto": gs.ALGO_AUTO, "decode": gs.ALGO_DECODE, "prefill": gs.ALGO_PREFILL}[args.algo]
+    for _ in range(args.warmup):
+        gs.linear_into(x, p, y, algo=algo)
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        gs.linear_into(x, p, y, algo=algo)
+    b.record()
+    b.synchronize()
+    s = a.elapsed_time(b) / 1e3 / args.steps
+    kept = p.kept
+    G, nw16 = inp // 256, (out + 15) // 16
+    nbytes = 512 * kept + 6 * G * nw16 + 2 * T * inp + 2 * T * out
+    flops = 2.0 * T * 256 * kept
+    assert gs.device_status() == gs.GS_OK
+    print(json.dumps({"layer": f"{out}x{inp}", "T": T, "density": args.density, "algo": args.algo, "kept": kept,
+                      "us": s * 1e6, "GB/s": nbytes / s / 1e9, "TFLOP/s": flops / s / 1e12}), flush=True)
+    return 0
+
+
+def run_block_layers(args, gs, torch, dev):
+    """The seven LLaMA-2-7B block projections (random masks of --density) in one
+    batched call per step, timed with CUDA events over R rotated packed copies."""
+    shapes = [(o, i) for (_, o, i) in wl.LLAMA2_7B_BLOCK]
+    T = args.tokens
+    g = torch.Generator(device=dev)
+    g.manual_seed(1234)
+    R = 4
+    packs = []
+    for _ in range(R):
+        hs = []
+        for (o, i) in shapes:
+            W = (torch.randn((o, i), generator=g, device=dev) * 0.02).to(torch.bfloat16)
+            B = (torch.rand((o, i // 256), generator=g, device=dev) < args.density).to(torch.uint8)
+            hs.append(gs.pack(W, B))
+        packs.append(hs)
+    xs = [torch.randn((T, i), generator=g, device=dev).to(torch.bfloat16) for (o, i) in shapes]
+    ys = [torch.empty((T, o), dtype=torch.bfloat16, device=dev) for (o, i) in shapes]
+    for r in range(args.warmup):
+        gs.linear_batched_into(xs, packs[r % R], ys)
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for r in range(args.steps):
+        gs.linear_batched_into(xs, packs[r % R], ys)
+    b.record()
+    b.synchronize()
+    s = a.elapsed_time(b) / 1e3 / args.steps
+    kept = sum(p.kept for p in packs[0])
+    nbytes = 512 * kept + sum(16 * (i // 256) * ((o + 63) // 64) + 2 * T * (i + o) for (o, i) in shapes)
+    assert gs.device_status() == gs.GS_OK
+    print(json.dumps({"layer": "llama2-7b-block x7 batched", "T": T, "density": args.density, "kept": kept,
+                      "us": s * 1e6, "GB/s": nbytes / s / 1e9}), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -524,11 +603,17 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--layer", default=None, help="single-layer mode: OUTxIN (random mask of --density)")
+    ap.add_argument("--tokens", type=int, default=16)
+    ap.add_argument("--density", type=float, default=0.5)
+    ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.layer:
+        return run_layer(args)
     return run_ours(args)
 
 

@@ -70,7 +70,8 @@ typedef struct gs_packed gs_packed;   /* opaque, library-owned */
  * out, in   out >= 1; in >= 256 and a multiple of 256; out*(in/256) < 2^31.
  * group_in  must be 256 (other group shapes: GS_ERR_UNSUPPORTED).
  * stream    work is queued on it; gs_pack synchronizes it once to learn the
- *           kept-group count before allocating the packed buffers.
+ *           kept-group count before allocating the packed buffers; the
+ *           remaining packing kernels complete in stream order on `stream`.
  * handle    receives the new handle (set to NULL on failure).
  * Errors: INVALID_ARG (nulls, sizes, alignment), UNSUPPORTED (group_in),
  *         OOM, CUDA.
@@ -83,8 +84,10 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
  * projection, no bias), fp32 accumulation, bf16 output rounded to nearest even.
  *
  * x_dev  bf16 [T][in] row-major, caller-owned, read only.
- * p      packed handle from gs_pack (read only; may be used concurrently from
- *        several streams).
+ * p      packed handle from gs_pack.  The handle also owns the decode kernel's
+ *        split-reduction scratch, so gs_linear / gs_linear_ex /
+ *        gs_linear_batched calls that share a handle must be ordered with
+ *        respect to each other (same stream, or synchronized streams).
  * T      number of tokens; T == 0 is a no-op, T < 0 is INVALID_ARG.
  * y_dev  bf16 [T][out] row-major, caller-owned; fully overwritten (rows of
  *        outputs with no kept group are written as +0.0).
@@ -97,9 +100,12 @@ gs_status gs_linear_ex(const void* x_dev, const gs_packed* p, int64_t T, void* y
                        gs_algo algo);
 
 /*
- * gs_linear_batched - n independent layers in one launch per kernel family:
- * ys[i] = xs[i] W_hat_i^T for the i-th handle, all with the same token count T.
- * Same per-layer semantics and errors as gs_linear.  n <= 64.
+ * gs_linear_batched - n independent layers, ys[i] = xs[i] W_hat_i^T for the
+ * i-th handle, all with the same token count T.  In the decode regime all n
+ * layers share one launch per 16 tokens (one grid streams every layer's kept
+ * groups); in the prefill regime the layers run back to back.  Same per-layer
+ * semantics and errors as gs_linear.  1 <= n <= 32 (n == 0 is a no-op); the
+ * handles must be distinct.
  */
 gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packed* const* ps,
                             int64_t T, void* const* ys_dev, void* stream);

@@ -32,6 +32,7 @@ void free_buffers(gs_packed* p) {
   if (p->tiles) cudaFree(p->tiles);
   if (p->win_off16) cudaFree(p->win_off16);
   if (p->kmask16) cudaFree(p->kmask16);
+  decode_release(p);
   if (cur >= 0 && cur != p->device) cudaSetDevice(cur);
   p->offsets = nullptr;
   p->row_idx = nullptr;
@@ -143,6 +144,7 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
   if ((st = dev_alloc((void**)&p->tiles, (size_t)kTileBytes * (size_t)p->kept, &total)) != GS_OK) goto fail;
   p->device_bytes = total;
   if ((st = launch_pack_compact(W_dev, p, s)) != GS_OK) goto fail;
+  if ((st = decode_prepare(p, s)) != GS_OK) goto fail;
   if ((st = prefill_prepare_weight_maps(p)) != GS_OK) goto fail;
   *handle = p;
   return GS_OK;
@@ -163,24 +165,16 @@ static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, v
   if (!x_dev || !y_dev) return GS_ERR_INVALID_ARG;
   if (!aligned16(x_dev) || !aligned16(y_dev)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (algo == GS_ALGO_AUTO) algo = T >= kPrefillMinTokens ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
+  if (algo == GS_ALGO_AUTO)
+    algo = (T >= kPrefillMinTokens && p->G <= prefill_max_chunks()) ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
   if (algo == GS_ALGO_PREFILL) return launch_prefill(x_dev, p, T, y_dev, s);
   // decode family: token blocks of at most decode_max_tokens()
   const int64_t blk = decode_max_tokens();
   for (int64_t t0 = 0; t0 < T; t0 += blk) {
     const int64_t tb = T - t0 < blk ? T - t0 : blk;
-    DecodeLayer L;
-    std::memset(&L, 0, sizeof(L));
-    L.x = static_cast<const uint16_t*>(x_dev) + t0 * p->in;
-    L.tiles = p->tiles;
-    L.win_off16 = p->win_off16;
-    L.kmask16 = p->kmask16;
-    L.y = static_cast<uint16_t*>(y_dev) + t0 * p->out;
-    L.out = (int32_t)p->out;
-    L.in = (int32_t)p->in;
-    L.G = p->G;
-    L.nw16 = p->nw16;
-    const gs_status st = launch_decode(&L, 1, (int)tb, s);
+    const void* xb = static_cast<const uint16_t*>(x_dev) + t0 * p->in;
+    void* yb = static_cast<uint16_t*>(y_dev) + t0 * p->out;
+    const gs_status st = launch_decode(&p, &xb, &yb, 1, (int)tb, s);
     if (st != GS_OK) return st;
   }
   return GS_OK;
@@ -210,25 +204,24 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (T >= kPrefillMinTokens) {
     for (int i = 0; i < n; ++i) {
-      const gs_status st = launch_prefill(xs_dev[i], ps[i], T, ys_dev[i], s);
+      const gs_status st = linear_impl(xs_dev[i], ps[i], T, ys_dev[i], stream, GS_ALGO_AUTO);
       if (st != GS_OK) return st;
     }
     return GS_OK;
   }
-  std::vector<DecodeLayer> L(n);
-  for (int i = 0; i < n; ++i) {
-    std::memset(&L[i], 0, sizeof(DecodeLayer));
-    L[i].x = static_cast<const uint16_t*>(xs_dev[i]);
-    L[i].tiles = ps[i]->tiles;
-    L[i].win_off16 = ps[i]->win_off16;
-    L[i].kmask16 = ps[i]->kmask16;
-    L[i].y = static_cast<uint16_t*>(ys_dev[i]);
-    L[i].out = (int32_t)ps[i]->out;
-    L[i].in = (int32_t)ps[i]->in;
-    L[i].G = ps[i]->G;
-    L[i].nw16 = ps[i]->nw16;
+  const int64_t blk = decode_max_tokens();
+  std::vector<const void*> xb(n);
+  std::vector<void*> yb(n);
+  for (int64_t t0 = 0; t0 < T; t0 += blk) {
+    const int64_t tb = T - t0 < blk ? T - t0 : blk;
+    for (int i = 0; i < n; ++i) {
+      xb[i] = static_cast<const uint16_t*>(xs_dev[i]) + t0 * ps[i]->in;
+      yb[i] = static_cast<uint16_t*>(ys_dev[i]) + t0 * ps[i]->out;
+    }
+    const gs_status st = launch_decode(ps, xb.data(), yb.data(), n, (int)tb, s);
+    if (st != GS_OK) return st;
   }
-  return launch_decode(L.data(), n, (int)T, s);
+  return GS_OK;
 }
 
 gs_status gs_unpack(const gs_packed* p, void* W_hat_dev, void* stream) {

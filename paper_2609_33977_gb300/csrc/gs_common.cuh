@@ -6,7 +6,7 @@
 #include <cstdint>
 #include <cstddef>
 
-#include "../../include/groupsparse.h"
+#include "groupsparse.h"
 
 namespace gs {
 
@@ -32,6 +32,13 @@ struct gs_packed {
   int32_t* win_off16; // [G][nw16+1]
   uint16_t* kmask16;  // [G][nw16]
   size_t device_bytes;
+  // decode kernel: window-major metadata and split-reduction scratch
+  int32_t nblk64;     // ceil(out / 64)
+  int32_t dec_cpu;    // chunks per decode work unit
+  int32_t dec_nsplit; // work units per 64-row block = ceil(G / dec_cpu)
+  int4* dmeta;        // [nblk64][G]: {first packed row of the block's slice, kept masks of its 4 windows, 0}
+  float* dec_ws;      // [nblk64][dec_nsplit][4][16 tokens][16 rows] partial sums (dec_nsplit > 1)
+  int32_t* dec_cnt;   // [nblk64][4] arrival counters (self-resetting)
   // tcgen05 prefill: TMA descriptors over the tiles (box heights 128/64/32/16 rows)
   alignas(64) unsigned char wmaps[4][128];
   bool wmaps_valid;
@@ -49,21 +56,15 @@ gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s);
 gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
 
 // decode.cu
-struct DecodeLayer {
-  const uint16_t* x;        // [T][in]
-  const uint16_t* tiles;    // [kept][256]
-  const int32_t* win_off16; // [G][nw16+1]
-  const uint16_t* kmask16;  // [G][nw16]
-  uint16_t* y;              // [T][out]
-  int32_t out, in, G, nw16;
-  int32_t cta_begin;        // first CTA of this layer in the launch
-  int32_t nblk;             // ceil(out / 128)
-};
-gs_status launch_decode(const DecodeLayer* layers, int n, int T, cudaStream_t s);
+gs_status decode_prepare(gs_packed* p, cudaStream_t s);   // allocates + builds the decode metadata
+void decode_release(gs_packed* p);
+gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void* const* ys, int n, int T,
+                        cudaStream_t s);
 int decode_max_tokens();
 
 // prefill.cu
 gs_status prefill_prepare_weight_maps(gs_packed* p);
 gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, cudaStream_t s);
+int prefill_max_chunks();
 
 }  // namespace gs

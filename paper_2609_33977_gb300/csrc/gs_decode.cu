@@ -1,16 +1,28 @@
 // Decode-regime group-sparse linear (few tokens, HBM-bound):
 //   y[t, r] = sum over kept groups (r, c) of sum_k x[t, 256c+k] W[r, 256c+k]   (Eq. 1)
 //
-// Work decomposition.  A warp owns a 16-row output window and walks the
-// chunks of its chunk range.  For chunk c it loads the kept rows of its window
-// (each a 512-byte packed group, 16 bytes per lane, coalesced in 64-byte runs)
-// straight into mma.sync A fragments, placing every kept row at its window
-// position and leaving pruned rows zero.  The x chunk forms the B fragment.
-// Because the MMA row is the output row, the fp32 accumulator stays in
-// registers across all chunks: no scatter, no atomics, a fixed summation
-// order.  A CTA is eight such warps (128 rows); S CTAs of a thread-block
-// cluster split the chunks of the same 128 rows and reduce their partial sums
-// through distributed shared memory in rank order (deterministic).
+// Work units.  A unit is (64-row block, range of chunks) of one layer, sized to
+// about 128 KB of kept weights.  Persistent CTAs walk their units in a snake
+// order over a longest-first unit list, so every CTA streams a similar number
+// of bytes and the pipeline never restarts between units.
+//
+// Data movement.  Inside a chunk the kept rows of a 64-row block are one
+// contiguous slice of the packed tiles, so a producer warp streams each chunk's
+// slice with a single bulk copy (cp.async.bulk) into a shared-memory ring, and
+// the chunk's x rows with one bulk copy per token; only kept bytes move.  The
+// producer also stages each unit's per-chunk metadata (slice start + the
+// 16-bit kept masks of the four 16-row windows).
+//
+// Compute.  Consumer warp w owns rows 16w..16w+15 of the block.  It builds
+// mma.sync A fragments from the slice, placing every kept row at its window
+// position (pruned rows stay zero), with the x chunk as the B fragment.  The
+// MMA row is the output row, so the fp32 accumulator stays in registers for
+// the whole unit: no scatter and no atomics on y.
+//
+// Reduction.  When a block's chunks are split over several units, each warp
+// writes its 16-row partial to the handle's workspace and bumps the window's
+// arrival counter; the last arriver adds the partials in split order (so the
+// result does not depend on arrival order), writes y and resets the counter.
 //
 // K permutation.  Within a 32-wide k block b, lane (g, q) holds the eight
 // consecutive weights k = 32b + 8q + 0..7 of rows g and g+8 and the same eight
@@ -18,229 +30,443 @@
 // 2b+1; the logical-to-physical k map depends only on (b, q), so A and B agree
 // and every physical k is used exactly once.
 #include "gs_common.cuh"
+#include "gs_sm100.cuh"
 
-#include <cooperative_groups.h>
 #include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
 #include <vector>
-
-namespace cg = cooperative_groups;
 
 namespace gs {
 namespace {
+using namespace sm100;
 
-constexpr int kDecWarps = 8;                 // 16-row windows per CTA
-constexpr int kDecRows = kDecWarps * kWin16;  // 128 rows per CTA
+constexpr int kDW = 4;                        // consumer warps = 16-row windows per block
+constexpr int kRows = kDW * kWin16;           // 64 rows per block
+constexpr int kThreadsDec = (kDW + 1) * 32;   // + one producer warp
 constexpr int kMaxBatch = 32;
-constexpr int kMaxNT = 8;                    // up to 64 tokens per launch
+constexpr int kMaxT = 16;                     // tokens per launch (two 8-token MMA tiles)
+constexpr int kSlots = 2;                     // ring depth (per CTA; two CTAs per SM)
+constexpr int kWBytes = kRows * kTileBytes;   // 32 KB: the largest 64-row slice
+constexpr int kXRow = kTileBytes + 16;        // x chunk row (512 B) padded by 16 B: conflict-free fragment reads
+constexpr int kSlotBytes = ((kWBytes + kMaxT * kXRow) + 1023) / 1024 * 1024;
+constexpr int kMaxCpu = 64;                   // chunks per unit
+constexpr int kMetaSlots = 2;
+constexpr int kDecSmemBytes = kSlots * kSlotBytes + kMetaSlots * kMaxCpu * 16 + 1024;
+constexpr int kPartFloats = kMaxT * kWin16;   // one warp's partial: 16 tokens x 16 rows
+constexpr int64_t kUnitBytes = 128 * 1024;    // target kept bytes per unit
+constexpr uint64_t kDecWaitLimitNs = 2000000000ull;
+constexpr uint64_t kDecDrainLimitNs = 200000000ull;
 
-struct DecodeParams {
-  DecodeLayer layers[kMaxBatch];
-  int32_t n_layers;
-  int32_t T;
-  int32_t S;
+struct DecLayer {
+  const uint16_t* x;     // [T][in]
+  const uint16_t* tiles; // [kept][256]
+  const int4* dmeta;     // [nblk][G]
+  uint16_t* y;           // [T][out]
+  float* ws;             // [nblk][nsplit][4][kPartFloats]
+  int32_t* cnt;          // [nblk][4]
+  int32_t out, in, G, nblk, cpu, nsplit;
+  int32_t unit_begin;
 };
 
-__device__ __forceinline__ uint4 ld_stream16(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
-  return v;
+struct DecParams {
+  DecLayer L[kMaxBatch];
+  int32_t n_layers;
+  int32_t T;
+  int32_t n_units;
+  int* err;
+};
+
+__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
-__device__ __forceinline__ uint4 ld_cached16(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
-  return v;
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                          uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint16_t f32_to_bf16_rn(float f) {
-  return __bfloat16_as_ushort(__float2bfloat16_rn(f));
+__device__ __forceinline__ uint16_t f32_to_bf16_rn(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+
+// kept mask of window w (0..3) from a metadata entry
+__device__ __forceinline__ uint32_t meta_mask(const int4& m, int w) {
+  const uint32_t v = (uint32_t)(w < 2 ? m.y : m.z);
+  return (w & 1) ? (v >> 16) : (v & 0xFFFFu);
+}
+
+struct Unit {
+  int l, blk, c0, nC;
+};
+
+// k-th unit of this CTA (snake order over the unit list); false when done
+__device__ __forceinline__ bool unit_of(const DecParams& P, int k, Unit& U) {
+  const int n = gridDim.x, b = blockIdx.x;
+  const int64_t u = (int64_t)k * n + ((k & 1) ? (n - 1 - b) : b);
+  if (u >= P.n_units) return false;
+  int l = 0;
+  while (l + 1 < P.n_layers && P.L[l + 1].unit_begin <= u) ++l;
+  const DecLayer& L = P.L[l];
+  const int r = (int)(u - L.unit_begin);
+  U.l = l;
+  U.blk = r / L.nsplit;
+  const int split = r % L.nsplit;
+  U.c0 = split * L.cpu;
+  U.nC = min(L.G, U.c0 + L.cpu) - U.c0;
+  return true;
 }
 
 template <int NT>
-__global__ void __launch_bounds__(kDecWarps * 32) k_decode(const __grid_constant__ DecodeParams P) {
-  const int S = P.S;
-  const int cl = blockIdx.x / S;     // cluster index = (layer, 128-row block)
-  const int s = blockIdx.x % S;      // rank inside the cluster = chunk split
-  int l = 0;
-  while (l + 1 < P.n_layers && P.layers[l + 1].cta_begin <= cl) ++l;
-  const DecodeLayer& L = P.layers[l];
-  const int blk = cl - L.cta_begin;
+__global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant__ DecParams P) {
+  extern __shared__ uint8_t dsmem_raw[];
+  __shared__ __align__(8) uint64_t w_full[kSlots];
+  __shared__ __align__(8) uint64_t w_empty[kSlots];
+  __shared__ __align__(8) uint64_t m_full[kMetaSlots];
+  __shared__ __align__(8) uint64_t m_empty[kMetaSlots];
+  __shared__ int abort_s;
+  uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
+  int4* meta = reinterpret_cast<int4*>(ring + kSlots * kSlotBytes);   // [kMetaSlots][kMaxCpu]
+
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = lane >> 2, q = lane & 3;
-  const int w16 = blk * kDecWarps + warp;
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < kSlots; ++k) {
+      mbar_init(&w_full[k], 1);
+      mbar_init(&w_empty[k], kDW);
+    }
+    for (int k = 0; k < kMetaSlots; ++k) {
+      mbar_init(&m_full[k], 1);
+      mbar_init(&m_empty[k], kDW);
+    }
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  volatile int* abort_flag = &abort_s;
   const int T = P.T;
 
-  float acc[NT][4];
+  if (warp == kDW) {
+    // ------------------------------------------------------------ producer warp
+    uint32_t q = 0;              // chunks issued so far (ring sequence number)
+    bool ok = true;
+    Unit U;
+    bool have = unit_of(P, 0, U);
+    int4 pre[kMaxCpu / 32];      // this lane's metadata entries of the next unit to stage
+    auto prefetch = [&](const Unit& V, bool hv) {
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) acc[nt][i] = 0.f;
-
-  if (w16 < L.nw16) {
-    const int c0 = (int)((int64_t)s * L.G / S), c1 = (int)((int64_t)(s + 1) * L.G / S);
-    const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
-    const int64_t xrow = L.in / 8;   // uint4 per x row
-    const uint4* xbase = reinterpret_cast<const uint4*>(L.x);
-    for (int c = c0; c < c1; ++c) {
-      const uint32_t km = L.kmask16[(int64_t)c * L.nw16 + w16];
-      if (km == 0u) continue;
-      const int32_t base = L.win_off16[(int64_t)c * (L.nw16 + 1) + w16];
-      const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
-      const uint4* tg = reinterpret_cast<const uint4*>(L.tiles) + (int64_t)(base + __popc(km & lo_g)) * 32 + q;
-      const uint4* tg8 = reinterpret_cast<const uint4*>(L.tiles) + (int64_t)(base + __popc(km & lo_g8)) * 32 + q;
-      uint4 a[8], a8[8];
-#pragma unroll
-      for (int b = 0; b < 8; ++b) {
-        a[b] = kg ? ld_stream16(tg + 4 * b) : make_uint4(0u, 0u, 0u, 0u);
-        a8[b] = kg8 ? ld_stream16(tg8 + 4 * b) : make_uint4(0u, 0u, 0u, 0u);
+      for (int j = 0; j < kMaxCpu / 32; ++j) {
+        const int i = lane + 32 * j;
+        pre[j] = (hv && i < V.nC) ? __ldg(P.L[V.l].dmeta + (int64_t)V.blk * P.L[V.l].G + V.c0 + i)
+                                  : make_int4(0, 0, 0, 0);
       }
+    };
+    prefetch(U, have);
+    for (int k = 0; have && ok; ++k) {
+      const int ms = k % kMetaSlots;
+      if (!mbar_wait_bounded(&m_empty[ms], ((uint32_t)(k / kMetaSlots) & 1u) ^ 1u, abort_flag, P.err,
+                             kDecWaitLimitNs, kDevErrTimeout)) {
+        ok = false;
+        break;
+      }
+      int4* mrow = meta + ms * kMaxCpu;
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        const int tok = nt * 8 + g;
-        const uint4* xr = xbase + (int64_t)tok * xrow + (int64_t)c * 32 + q;
-#pragma unroll
-        for (int b = 0; b < 8; ++b) {
-          const uint4 xv = tok < T ? ld_cached16(xr + 4 * b) : make_uint4(0u, 0u, 0u, 0u);
-          mma16816(acc[nt], a[b].x, a8[b].x, a[b].y, a8[b].y, xv.x, xv.y);
-          mma16816(acc[nt], a[b].z, a8[b].z, a[b].w, a8[b].w, xv.z, xv.w);
+      for (int j = 0; j < kMaxCpu / 32; ++j)
+        if (lane + 32 * j < U.nC) mrow[lane + 32 * j] = pre[j];
+      __threadfence_block();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&m_full[ms]);   // release: the staged entries are visible to consumers
+      Unit V;
+      const bool have_v = unit_of(P, k + 1, V);
+      prefetch(V, have_v);                       // in flight while this unit's copies are issued
+      if (lane == 0) {
+        const DecLayer& L = P.L[U.l];
+        for (int i = 0; i < U.nC && ok; ++i, ++q) {
+          const int slot = (int)(q % kSlots);
+          if (!mbar_wait_bounded(&w_empty[slot], ((q / kSlots) & 1u) ^ 1u, abort_flag, P.err, kDecWaitLimitNs,
+                                 kDevErrTimeout)) {
+            ok = false;
+            break;
+          }
+          const int4 m = mrow[i];
+          const uint32_t cnt = __popc((uint32_t)m.y) + __popc((uint32_t)m.z);
+          const uint32_t bytes = cnt * (uint32_t)kTileBytes;
+          uint8_t* dst = ring + slot * kSlotBytes;
+          fence_proxy_async_smem();
+          mbar_arrive_expect_tx(&w_full[slot], bytes + (cnt ? (uint32_t)T * kTileBytes : 0u));
+          if (cnt) {
+            bulk_copy_g2s(dst, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[slot]);
+            const uint16_t* xc = L.x + (int64_t)(U.c0 + i) * kGroupIn;
+            for (int t = 0; t < T; ++t)
+              bulk_copy_g2s(dst + kWBytes + t * kXRow, xc + (int64_t)t * L.in, kTileBytes, &w_full[slot]);
+          }
         }
       }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      q = __shfl_sync(0xffffffffu, q, 0);
+      U = V;
+      have = have_v;
     }
-  }
-
-  const int row0 = blk * kDecRows;
-  if (S == 1) {
-    if (w16 < L.nw16) {
+    if (lane == 0 && !ok) {
+      // let copies already in flight land before the CTA retires
+      for (uint32_t i = q > (uint32_t)kSlots ? q - kSlots : 0u; i < q; ++i) {
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(&w_full[i % kSlots], (i / kSlots) & 1u))
+          if (globaltimer_ns() - t0 > kDecDrainLimitNs) break;
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ consumer warps
+    const int g = lane >> 2, qd = lane & 3;
+    const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
+    uint32_t q = 0;
+    bool ok = true;
+    Unit U;
+    for (int k = 0; ok && unit_of(P, k, U); ++k) {
+      const DecLayer& L = P.L[U.l];
+      const int ms = k % kMetaSlots;
+      if (!mbar_wait_bounded(&m_full[ms], (uint32_t)(k / kMetaSlots) & 1u, abort_flag, P.err, kDecWaitLimitNs,
+                             kDevErrTimeout)) {
+        ok = false;
+        break;
+      }
+      const int4* mrow = meta + ms * kMaxCpu;
+      float acc[NT][4], acc2[NT][4];   // two chains (even / odd k blocks) halve the MMA dependency depth
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          const int tok = nt * 8 + 2 * q + j;
-          const int r = row0 + warp * kWin16 + g;
-          if (tok < T) {
-            if (r < L.out) L.y[(int64_t)tok * L.out + r] = f32_to_bf16_rn(acc[nt][j]);
-            if (r + 8 < L.out) L.y[(int64_t)tok * L.out + r + 8] = f32_to_bf16_rn(acc[nt][2 + j]);
+        for (int i = 0; i < 4; ++i) acc[nt][i] = acc2[nt][i] = 0.f;
+      for (int i = 0; i < U.nC; ++i, ++q) {
+        const int4 m = mrow[i];
+        const uint32_t km = meta_mask(m, warp);
+        int base = 0;
+#pragma unroll
+        for (int w = 0; w < kDW; ++w)
+          if (w < warp) base += __popc(meta_mask(m, w));
+        const int slot = (int)(q % kSlots);
+        if (!mbar_wait_bounded(&w_full[slot], (q / kSlots) & 1u, abort_flag, P.err, kDecWaitLimitNs,
+                               kDevErrTimeout)) {
+          ok = false;
+          break;
+        }
+        if (km != 0u) {
+          const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
+          const uint4* sl = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
+          uint4 xv[NT][8];
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            const int tok = nt * 8 + g;
+            const uint4* xr = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kWBytes + tok * kXRow) + qd;
+#pragma unroll
+            for (int b = 0; b < 8; ++b) xv[nt][b] = tok < T ? xr[4 * b] : make_uint4(0u, 0u, 0u, 0u);
+          }
+          const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + qd;
+          const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + qd;
+#pragma unroll
+          for (int b = 0; b < 8; ++b) {
+            const uint4 a = kg ? tg[4 * b] : make_uint4(0u, 0u, 0u, 0u);
+            const uint4 a8 = kg8 ? tg8[4 * b] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              mma16816(acc[nt], a.x, a8.x, a.y, a8.y, xv[nt][b].x, xv[nt][b].y);
+              mma16816(acc2[nt], a.z, a8.z, a.w, a8.w, xv[nt][b].z, xv[nt][b].w);
+            }
           }
         }
-    }
-    return;
-  }
-
-  // chunk-split reduction across the cluster through distributed shared memory
-  __shared__ float red[kDecWarps][NT * 8][kWin16 + 1];
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      red[warp][nt * 8 + 2 * q + j][g] = acc[nt][j];
-      red[warp][nt * 8 + 2 * q + j][g + 8] = acc[nt][2 + j];
-    }
-  cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();
-  const int Tl = T < NT * 8 ? T : NT * 8;
-  for (int wi = s; wi < kDecWarps; wi += S) {
-    if (blk * kDecWarps + wi >= L.nw16) break;
-    for (int e = threadIdx.x; e < Tl * kWin16; e += blockDim.x) {
-      const int tok = e / kWin16, i = e % kWin16;
-      float sum = 0.f;
-      for (int rk = 0; rk < S; ++rk) {
-        const float* rred = cluster.map_shared_rank(&red[0][0][0], rk);
-        sum += rred[(wi * (NT * 8) + tok) * (kWin16 + 1) + i];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&w_empty[slot]);
       }
-      const int r = row0 + wi * kWin16 + i;
-      if (r < L.out) L.y[(int64_t)tok * L.out + r] = f32_to_bf16_rn(sum);
+      if (!ok) break;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&m_empty[ms]);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[nt][i] += acc2[nt][i];
+
+      // ---- unit result: this warp's 16 rows x T tokens
+      const int r0 = U.blk * kRows + warp * kWin16;
+      if (L.nsplit == 1) {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const int tok = nt * 8 + 2 * qd + j;
+            if (tok < T) {
+              if (r0 + g < L.out) L.y[(int64_t)tok * L.out + r0 + g] = f32_to_bf16_rn(acc[nt][j]);
+              if (r0 + g + 8 < L.out) L.y[(int64_t)tok * L.out + r0 + g + 8] = f32_to_bf16_rn(acc[nt][2 + j]);
+            }
+          }
+      } else {
+        const int split = U.c0 / L.cpu;
+        float* part = L.ws + (((int64_t)U.blk * L.nsplit + split) * kDW + warp) * kPartFloats;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const int tok = nt * 8 + 2 * qd + j;
+            part[tok * kWin16 + g] = acc[nt][j];
+            part[tok * kWin16 + g + 8] = acc[nt][2 + j];
+          }
+        __threadfence();
+        __syncwarp();
+        int last = 0;
+        int32_t* cnt = L.cnt + U.blk * kDW + warp;
+        if (lane == 0) last = (atomicAdd(cnt, 1) == L.nsplit - 1);
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
+          __threadfence();
+          const float* base_ws = L.ws + ((int64_t)U.blk * L.nsplit * kDW + warp) * kPartFloats;
+          const int Tl = T < NT * 8 ? T : NT * 8;
+          for (int e = lane; e < Tl * kWin16; e += 32) {
+            // issue every partial's load first, then add them in split order
+            float sum = 0.f;
+            for (int s0 = 0; s0 < L.nsplit; s0 += 8) {
+              float v[8];
+#pragma unroll
+              for (int u = 0; u < 8; ++u)
+                v[u] = s0 + u < L.nsplit ? __ldcg(base_ws + (int64_t)(s0 + u) * kDW * kPartFloats + e) : 0.f;
+#pragma unroll
+              for (int u = 0; u < 8; ++u) sum += v[u];
+            }
+            const int tok = e / kWin16, i = e % kWin16;
+            if (r0 + i < L.out) L.y[(int64_t)tok * L.out + r0 + i] = f32_to_bf16_rn(sum);
+          }
+          if (lane == 0) *cnt = 0;
+        }
+      }
     }
   }
-  cluster.sync();
+  __syncthreads();
 }
 
-int g_num_sms = 0;
+// metadata of 64-row block b, chunk c: first packed row of the block's slice and
+// the kept masks of its four 16-row windows
+__global__ void k_decode_meta(const int32_t* __restrict__ win_off16, const uint16_t* __restrict__ kmask16,
+                              int32_t G, int32_t nw16, int32_t nblk, int4* __restrict__ dmeta) {
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;   // e = b * G + c
+  if (e >= (int64_t)nblk * G) return;
+  const int b = (int)(e / G), c = (int)(e % G);
+  const int w0 = kDW * b;
+  uint32_t km[kDW];
+#pragma unroll
+  for (int w = 0; w < kDW; ++w) km[w] = (w0 + w < nw16) ? kmask16[(int64_t)c * nw16 + w0 + w] : 0u;
+  dmeta[e] = make_int4(win_off16[(int64_t)c * (nw16 + 1) + w0], (int)(km[0] | (km[1] << 16)),
+                       (int)(km[2] | (km[3] << 16)), 0);
+}
 
-int num_sms() {
-  if (g_num_sms == 0) {
+int sm_count_dec() {
+  static int n = 0;
+  if (n == 0) {
     int dev = 0;
     cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (g_num_sms <= 0) g_num_sms = 148;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
   }
-  return g_num_sms;
+  return n;
 }
 
 template <int NT>
-cudaError_t launch_nt(const DecodeParams& P, int grid, cudaStream_t s) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid, 1, 1);
-  cfg.blockDim = dim3(kDecWarps * 32, 1, 1);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  int na = 0;
-  if (P.S > 1) {
-    attr[na].id = cudaLaunchAttributeClusterDimension;
-    attr[na].val.clusterDim.x = P.S;
-    attr[na].val.clusterDim.y = 1;
-    attr[na].val.clusterDim.z = 1;
-    ++na;
-  }
-  cfg.attrs = attr;
-  cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, k_decode<NT>, P);
+cudaError_t launch_nt(const DecParams& P, int grid, cudaStream_t s) {
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, []() {
+    attr_err = cudaFuncSetAttribute(k_decode<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  k_decode<NT><<<grid, kThreadsDec, kDecSmemBytes, s>>>(P);
+  return cudaGetLastError();
 }
 
 }  // namespace
 
-int decode_max_tokens() { return kMaxNT * 8; }
+int decode_max_tokens() { return kMaxT; }
 
-gs_status launch_decode(const DecodeLayer* layers, int n, int T, cudaStream_t s) {
-  if (n <= 0 || T <= 0) return GS_OK;
-  if (n > kMaxBatch || T > kMaxNT * 8) return GS_ERR_UNSUPPORTED;
-  // Longest-work layers first: CTAs are dispatched roughly in index order, so
-  // the layers with the most kept groups per CTA start first.
-  std::vector<int> order(n);
-  for (int i = 0; i < n; ++i) order[i] = i;
-  std::vector<double> work(n);
-  int64_t blocks = 0;
-  int minG = 1 << 30;
-  for (int i = 0; i < n; ++i) {
-    const int nblk = (layers[i].out + kDecRows - 1) / kDecRows;
-    blocks += nblk;
-    minG = std::min(minG, layers[i].G);
-    work[i] = (double)layers[i].G;   // chunks per 128-row block (density-independent proxy)
+gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
+  p->nblk64 = (int32_t)((p->out + kRows - 1) / kRows);
+  // chunks per unit: about kUnitBytes of kept weights per unit
+  const double per_chunk = p->kept > 0 ? 512.0 * (double)p->kept / ((double)p->G * (double)p->nblk64) : 512.0;
+  int cpu = (int)std::floor((double)kUnitBytes / std::max(per_chunk, 1.0) + 0.5);
+  cpu = std::max(1, std::min(cpu, std::min(p->G, kMaxCpu)));
+  p->dec_cpu = cpu;
+  p->dec_nsplit = (p->G + cpu - 1) / cpu;
+  const size_t nmeta = (size_t)p->nblk64 * (size_t)p->G;
+  if (cudaMalloc(&p->dmeta, nmeta * sizeof(int4)) != cudaSuccess) return GS_ERR_OOM;
+  p->device_bytes += nmeta * sizeof(int4);
+  if (p->dec_nsplit > 1) {
+    const size_t nws = (size_t)p->nblk64 * p->dec_nsplit * kDW * kPartFloats;
+    const size_t ncnt = (size_t)p->nblk64 * kDW;
+    if (cudaMalloc(&p->dec_ws, nws * sizeof(float)) != cudaSuccess) return GS_ERR_OOM;
+    if (cudaMalloc(&p->dec_cnt, ncnt * sizeof(int32_t)) != cudaSuccess) return GS_ERR_OOM;
+    if (cudaMemsetAsync(p->dec_cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) return GS_ERR_CUDA;
+    p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
   }
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return work[a] > work[b]; });
-  // chunk splits: enough CTAs for about two per SM, at most 8 (portable cluster), at most G
-  const int want = 2 * num_sms();
-  int S = (int)((want + blocks - 1) / blocks);
-  S = std::max(1, std::min(S, std::min(8, minG)));
+  const int64_t n = (int64_t)nmeta;
+  k_decode_meta<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p->win_off16, p->kmask16, p->G, p->nw16, p->nblk64,
+                                                           p->dmeta);
+  note_launch();
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
 
-  DecodeParams P = {};
+void decode_release(gs_packed* p) {
+  if (p->dmeta) cudaFree(p->dmeta);
+  if (p->dec_ws) cudaFree(p->dec_ws);
+  if (p->dec_cnt) cudaFree(p->dec_cnt);
+  p->dmeta = nullptr;
+  p->dec_ws = nullptr;
+  p->dec_cnt = nullptr;
+}
+
+gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void* const* ys, int n, int T,
+                        cudaStream_t s) {
+  if (n <= 0 || T <= 0) return GS_OK;
+  if (n > kMaxBatch || T > kMaxT) return GS_ERR_UNSUPPORTED;
+  // longest units first (bytes per unit), so the snake schedule balances
+  std::vector<int> order(n);
+  std::vector<double> unit_bytes(n);
+  for (int i = 0; i < n; ++i) {
+    order[i] = i;
+    const gs_packed* p = ps[i];
+    unit_bytes[i] = (double)p->kept / std::max(1, p->nblk64 * p->dec_nsplit);
+  }
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return unit_bytes[a] > unit_bytes[b]; });
+  DecParams P;
+  std::memset(&P, 0, sizeof(P));
   P.n_layers = n;
   P.T = T;
-  P.S = S;
-  int32_t cl = 0;
+  P.err = device_error_flag();
+  if (!P.err) return GS_ERR_CUDA;
+  int64_t units = 0;
   for (int k = 0; k < n; ++k) {
-    P.layers[k] = layers[order[k]];
-    P.layers[k].nblk = (layers[order[k]].out + kDecRows - 1) / kDecRows;
-    P.layers[k].cta_begin = cl;
-    cl += P.layers[k].nblk;
+    const gs_packed* p = ps[order[k]];
+    DecLayer& L = P.L[k];
+    L.x = static_cast<const uint16_t*>(xs[order[k]]);
+    L.tiles = p->tiles;
+    L.dmeta = p->dmeta;
+    L.y = static_cast<uint16_t*>(ys[order[k]]);
+    L.ws = p->dec_ws;
+    L.cnt = p->dec_cnt;
+    L.out = (int32_t)p->out;
+    L.in = (int32_t)p->in;
+    L.G = p->G;
+    L.nblk = p->nblk64;
+    L.cpu = p->dec_cpu;
+    L.nsplit = p->dec_nsplit;
+    L.unit_begin = (int32_t)units;
+    units += (int64_t)p->nblk64 * p->dec_nsplit;
   }
-  const int grid = cl * S;
-  cudaError_t e;
-  if (T <= 8) e = launch_nt<1>(P, grid, s);
-  else if (T <= 16) e = launch_nt<2>(P, grid, s);
-  else if (T <= 32) e = launch_nt<4>(P, grid, s);
-  else e = launch_nt<8>(P, grid, s);
+  if (units > INT32_MAX) return GS_ERR_UNSUPPORTED;
+  P.n_units = (int32_t)units;
+  const int grid = (int)std::min<int64_t>(units, 2 * (int64_t)sm_count_dec());
+  const cudaError_t e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);
   note_launch();
   return e == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }

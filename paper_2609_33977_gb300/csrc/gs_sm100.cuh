@@ -43,18 +43,32 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// try_wait that may suspend the thread in hardware for up to `hint_ns` while
+// the phase is incomplete (no busy spinning); returns whether the phase completed.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
 
 // Bounded wait: returns false when the CTA-wide abort flag is raised or when
 // the wait exceeds `limit_ns` (then it raises the flag and records the error).
+// `abort_flag` may be null (the wait then only ends on completion or timeout).
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                                   int* err_flag, uint64_t limit_ns, int err_code) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (abort_flag && *abort_flag) return false;
     if (globaltimer_ns() - t0 > limit_ns) {
-      *abort_flag = 1;
+      if (abort_flag) *abort_flag = 1;
       atomicExch(err_flag, err_code);
       return false;
     }
