@@ -46,6 +46,10 @@ struct gs_packed {
 
 namespace gs {
 
+// 2-D bf16 TMA descriptor (map: 128-byte, 64-byte aligned buffer); false on failure
+bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                         uint32_t box_outer, bool swizzle128);
+
 // library-owned per-device error flag (allocated on first use)
 int* device_error_flag();
 void note_launch(int64_t n = 1);

@@ -2,14 +2,16 @@
 //   y[t, r] = sum over kept groups (r, c) of sum_k x[t, 256c+k] W[r, 256c+k]   (Eq. 1)
 //
 // Work units.  A unit is (64-row block, range of chunks) of one layer, sized to
-// about 128 KB of kept weights.  Persistent CTAs walk their units in a snake
+// about 256 KB of kept weights.  Persistent CTAs walk their units in a snake
 // order over a longest-first unit list, so every CTA streams a similar number
 // of bytes and the pipeline never restarts between units.
 //
 // Data movement.  Inside a chunk the kept rows of a 64-row block are one
 // contiguous slice of the packed tiles, so a producer warp streams each chunk's
-// slice with a single bulk copy (cp.async.bulk) into a shared-memory ring, and
-// the chunk's x rows with one bulk copy per token; only kept bytes move.  The
+// slice with a single bulk copy (cp.async.bulk) into a byte-granular
+// shared-memory ring (each chunk takes exactly its slice + x rows, so the ring
+// holds several chunks in flight), and the chunk's x rows with one 2-D TMA
+// load; only kept bytes move.  The
 // producer also stages each unit's per-chunk metadata (slice start + the
 // 16-bit kept masks of the four 16-row windows).
 //
@@ -32,6 +34,8 @@
 #include "gs_common.cuh"
 #include "gs_sm100.cuh"
 
+#include <cuda.h>
+
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -47,19 +51,19 @@ constexpr int kRows = kDW * kWin16;           // 64 rows per block
 constexpr int kThreadsDec = (kDW + 1) * 32;   // + one producer warp
 constexpr int kMaxBatch = 32;
 constexpr int kMaxT = 16;                     // tokens per launch (two 8-token MMA tiles)
-constexpr int kSlots = 2;                     // ring depth (per CTA; two CTAs per SM)
-constexpr int kWBytes = kRows * kTileBytes;   // 32 KB: the largest 64-row slice
-constexpr int kXRow = kTileBytes + 16;        // x chunk row (512 B) padded by 16 B: conflict-free fragment reads
-constexpr int kSlotBytes = ((kWBytes + kMaxT * kXRow) + 1023) / 1024 * 1024;
+constexpr int kRingBytes = 104 * 1024;       // byte ring per CTA (two CTAs per SM)
+constexpr int kRingSeq = 16;                  // chunks that may be in flight (barrier ring)
+constexpr int kXRow = kTileBytes;             // x chunk row (512 B), one 2-D TMA box per chunk
 constexpr int kMaxCpu = 64;                   // chunks per unit
 constexpr int kMetaSlots = 2;
-constexpr int kDecSmemBytes = kSlots * kSlotBytes + kMetaSlots * kMaxCpu * 16 + 1024;
+constexpr int kDecSmemBytes = kRingBytes + kMetaSlots * kMaxCpu * 16 + 1024;
 constexpr int kPartFloats = kMaxT * kWin16;   // one warp's partial: 16 tokens x 16 rows
-constexpr int64_t kUnitBytes = 128 * 1024;    // target kept bytes per unit
+constexpr int64_t kUnitBytes = 256 * 1024;    // target kept bytes per unit
 constexpr uint64_t kDecWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDecDrainLimitNs = 200000000ull;
 
 struct DecLayer {
+  CUtensorMap xmap;      // x [T][in], box 256 x T (one chunk of every token per load)
   const uint16_t* x;     // [T][in]
   const uint16_t* tiles; // [kept][256]
   const int4* dmeta;     // [nblk][G]
@@ -128,17 +132,18 @@ __device__ __forceinline__ bool unit_of(const DecParams& P, int k, Unit& U) {
 template <int NT>
 __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant__ DecParams P) {
   extern __shared__ uint8_t dsmem_raw[];
-  __shared__ __align__(8) uint64_t w_full[kSlots];
-  __shared__ __align__(8) uint64_t w_empty[kSlots];
+  __shared__ __align__(8) uint64_t w_full[kRingSeq];
+  __shared__ __align__(8) uint64_t w_empty[kRingSeq];
+  __shared__ uint32_t w_off[kRingSeq];   // ring offset of each in-flight chunk
   __shared__ __align__(8) uint64_t m_full[kMetaSlots];
   __shared__ __align__(8) uint64_t m_empty[kMetaSlots];
   __shared__ int abort_s;
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
-  int4* meta = reinterpret_cast<int4*>(ring + kSlots * kSlotBytes);   // [kMetaSlots][kMaxCpu]
+  int4* meta = reinterpret_cast<int4*>(ring + kRingBytes);   // [kMetaSlots][kMaxCpu]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int k = 0; k < kSlots; ++k) {
+    for (int k = 0; k < kRingSeq; ++k) {
       mbar_init(&w_full[k], 1);
       mbar_init(&w_empty[k], kDW);
     }
@@ -156,6 +161,9 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   if (warp == kDW) {
     // ------------------------------------------------------------ producer warp
     uint32_t q = 0;              // chunks issued so far (ring sequence number)
+    uint32_t oldest = 0;         // oldest chunk not yet known to be released
+    uint64_t head = 0, tail = 0; // virtual byte offsets: allocated / released
+    uint64_t end_v[kRingSeq];    // virtual end offset of each in-flight chunk
     bool ok = true;
     Unit U;
     bool have = unit_of(P, 0, U);
@@ -189,23 +197,36 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       if (lane == 0) {
         const DecLayer& L = P.L[U.l];
         for (int i = 0; i < U.nC && ok; ++i, ++q) {
-          const int slot = (int)(q % kSlots);
-          if (!mbar_wait_bounded(&w_empty[slot], ((q / kSlots) & 1u) ^ 1u, abort_flag, P.err, kDecWaitLimitNs,
-                                 kDevErrTimeout)) {
-            ok = false;
-            break;
-          }
           const int4 m = mrow[i];
           const uint32_t cnt = __popc((uint32_t)m.y) + __popc((uint32_t)m.z);
           const uint32_t bytes = cnt * (uint32_t)kTileBytes;
-          uint8_t* dst = ring + slot * kSlotBytes;
+          const uint32_t need = cnt ? ((bytes + (uint32_t)T * kXRow + 127u) & ~127u) : 0u;   // 128-B aligned starts
+          // allocate `need` contiguous bytes; a chunk that would straddle the end starts over at 0
+          uint64_t start = head;
+          if (need && (start % kRingBytes) + need > (uint64_t)kRingBytes) start += kRingBytes - start % kRingBytes;
+          // wait for the oldest chunks until the allocation fits and a barrier pair is free
+          while (ok && (start + need - tail > (uint64_t)kRingBytes || q - oldest >= (uint32_t)kRingSeq)) {
+            const uint32_t j = oldest % kRingSeq;
+            if (!mbar_wait_bounded(&w_empty[j], (oldest / kRingSeq) & 1u, abort_flag, P.err, kDecWaitLimitNs,
+                                   kDevErrTimeout)) {
+              ok = false;
+              break;
+            }
+            tail = end_v[j];
+            ++oldest;
+          }
+          if (!ok) break;
+          const uint32_t e = q % kRingSeq;
+          const uint32_t off = (uint32_t)(start % kRingBytes);
+          w_off[e] = off;
+          end_v[e] = start + need;
+          head = start + need;
+          uint8_t* dst = ring + off;
           fence_proxy_async_smem();
-          mbar_arrive_expect_tx(&w_full[slot], bytes + (cnt ? (uint32_t)T * kTileBytes : 0u));
+          mbar_arrive_expect_tx(&w_full[e], cnt ? bytes + (uint32_t)T * kTileBytes : 0u);
           if (cnt) {
-            bulk_copy_g2s(dst, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[slot]);
-            const uint16_t* xc = L.x + (int64_t)(U.c0 + i) * kGroupIn;
-            for (int t = 0; t < T; ++t)
-              bulk_copy_g2s(dst + kWBytes + t * kXRow, xc + (int64_t)t * L.in, kTileBytes, &w_full[slot]);
+            bulk_copy_g2s(dst, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
+            tma_load_2d(dst + bytes, &L.xmap, &w_full[e], (U.c0 + i) * kGroupIn, 0);
           }
         }
       }
@@ -216,9 +237,9 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     }
     if (lane == 0 && !ok) {
       // let copies already in flight land before the CTA retires
-      for (uint32_t i = q > (uint32_t)kSlots ? q - kSlots : 0u; i < q; ++i) {
+      for (uint32_t i = q > (uint32_t)kRingSeq ? q - kRingSeq : 0u; i < q; ++i) {
         const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait(&w_full[i % kSlots], (i / kSlots) & 1u))
+        while (!mbar_try_wait(&w_full[i % kRingSeq], (i / kRingSeq) & 1u))
           if (globaltimer_ns() - t0 > kDecDrainLimitNs) break;
       }
     }
@@ -251,20 +272,22 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 #pragma unroll
         for (int w = 0; w < kDW; ++w)
           if (w < warp) base += __popc(meta_mask(m, w));
-        const int slot = (int)(q % kSlots);
-        if (!mbar_wait_bounded(&w_full[slot], (q / kSlots) & 1u, abort_flag, P.err, kDecWaitLimitNs,
+        const int slot = (int)(q % kRingSeq);
+        if (!mbar_wait_bounded(&w_full[slot], (q / kRingSeq) & 1u, abort_flag, P.err, kDecWaitLimitNs,
                                kDevErrTimeout)) {
           ok = false;
           break;
         }
         if (km != 0u) {
           const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
-          const uint4* sl = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes);
+          const uint8_t* cbase = ring + w_off[slot];
+          const uint4* sl = reinterpret_cast<const uint4*>(cbase);
+          const uint32_t xoff = (uint32_t)(__popc((uint32_t)m.y) + __popc((uint32_t)m.z)) * (uint32_t)kTileBytes;
           uint4 xv[NT][8];
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int tok = nt * 8 + g;
-            const uint4* xr = reinterpret_cast<const uint4*>(ring + slot * kSlotBytes + kWBytes + tok * kXRow) + qd;
+            const uint4* xr = reinterpret_cast<const uint4*>(cbase + xoff + tok * kXRow) + qd;
 #pragma unroll
             for (int b = 0; b < 8; ++b) xv[nt][b] = tok < T ? xr[4 * b] : make_uint4(0u, 0u, 0u, 0u);
           }
@@ -350,7 +373,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 
 // metadata of 64-row block b, chunk c: first packed row of the block's slice and
 // the kept masks of its four 16-row windows
-__global__ void k_decode_meta(const int32_t* __restrict__ win_off16, const uint16_t* __restrict__ kmask16,
+__global__ void k_pack_decode_meta(const int32_t* __restrict__ win_off16, const uint16_t* __restrict__ kmask16,
                               int32_t G, int32_t nw16, int32_t nblk, int4* __restrict__ dmeta) {
   const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;   // e = b * G + c
   if (e >= (int64_t)nblk * G) return;
@@ -410,7 +433,7 @@ gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
     p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
   }
   const int64_t n = (int64_t)nmeta;
-  k_decode_meta<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p->win_off16, p->kmask16, p->G, p->nw16, p->nblk64,
+  k_pack_decode_meta<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p->win_off16, p->kmask16, p->G, p->nw16, p->nblk64,
                                                            p->dmeta);
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
@@ -449,6 +472,8 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     const gs_packed* p = ps[order[k]];
     DecLayer& L = P.L[k];
     L.x = static_cast<const uint16_t*>(xs[order[k]]);
+    if (!encode_tmap_2d_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)kGroupIn, (uint32_t)T, false))
+      return GS_ERR_CUDA;
     L.tiles = p->tiles;
     L.dmeta = p->dmeta;
     L.y = static_cast<uint16_t*>(ys[order[k]]);

@@ -387,37 +387,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
 }
 
 // ------------------------------------------------------------------ host side
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, []() {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  });
-  return fn;
-}
-
-bool encode_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
-                    uint32_t box_outer) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return false;
-  const cuuint64_t dims[2] = {inner, outer};
-  const cuuint64_t strides[1] = {inner * 2};
-  const cuuint32_t box[2] = {box_inner, box_outer};
-  const cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 int sm_count() {
   static int n = 0;
   if (n == 0) {
@@ -437,7 +406,7 @@ gs_status prefill_prepare_weight_maps(gs_packed* p) {
   static_assert(sizeof(CUtensorMap) == 128, "CUtensorMap size");
   for (int h = 0; h < 4; ++h) {
     CUtensorMap m;
-    if (!encode_2d_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, kBK, (uint32_t)(128 >> h)))
+    if (!encode_tmap_2d_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, kBK, (uint32_t)(128 >> h), true))
       return GS_ERR_CUDA;
     std::memcpy(p->wmaps[h], &m, sizeof(m));
   }
@@ -463,7 +432,7 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
 
   PrefillParams P;
   std::memset(&P, 0, sizeof(P));
-  if (!encode_2d_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBK, kBM)) return GS_ERR_CUDA;
+  if (!encode_tmap_2d_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBK, kBM, true)) return GS_ERR_CUDA;
   for (int h = 0; h < 4; ++h) std::memcpy(&P.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
   P.row_idx = p->row_idx;
   P.win_off16 = p->win_off16;
