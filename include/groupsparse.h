@@ -135,6 +135,35 @@ gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t*
 gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* row_idx_host,
                            uint16_t* tiles_host, int32_t* win_off16_host, uint16_t* kmask16_host);
 
+/*
+ * gs_pack_index_noalloc - the index part of gs_pack (per-chunk offsets, per
+ * 16-row-window offsets and kept masks, exactly as gs_packed_export reports
+ * them) computed without allocating any device memory.  The paper has no
+ * counterpart; this entry point exists for callers that cannot allocate device
+ * memory when they pack: code running inside a CUDA graph capture, where
+ * cudaMalloc is not allowed, and runtimes that hand out all device memory from
+ * their own fixed arena.
+ *
+ * mask_dev       uint8 [out][in/256] row-major; nonzero = keep.  Read only.
+ * out, in        out >= 1; in >= 256 and a multiple of 256.
+ * offsets_dev    int64 [in/256 + 1], caller-owned, overwritten.
+ * win_off16_dev  int32 [in/256][ceil(out/16) + 1], caller-owned, overwritten.
+ * kmask16_dev    uint16 [in/256][ceil(out/16)], caller-owned, overwritten.
+ * Temporary counts live in one fixed array in the library's device memory
+ * (2^20 entries of int32, held by every GPU that loads the library until the
+ * process exits); (in/256) * ceil(out/16) above 2^20 returns
+ * GS_ERR_UNSUPPORTED before anything is launched.  All calls share that array:
+ * calls whose kernels overlap on the GPU (different streams without ordering)
+ * race and must be serialized by the caller.  Every entry a call reads is
+ * written by the same call first, so nothing needs clearing between calls.
+ * The first call on a device looks up the array's device address (with that
+ * device current) and caches it; make that first call before any stream
+ * capture.  Asynchronous on `stream`.
+ * Errors: INVALID_ARG (nulls, sizes), UNSUPPORTED (beyond the fixed array), CUDA.
+ */
+gs_status gs_pack_index_noalloc(const uint8_t* mask_dev, int64_t out, int64_t in, int64_t* offsets_dev,
+                                int32_t* win_off16_dev, uint16_t* kmask16_dev, void* stream);
+
 /* Releases the handle and its device buffers (NULL is a no-op). */
 void gs_free(gs_packed* p);
 

@@ -6,6 +6,8 @@
 // 16-bit kept mask.
 #include "gs_common.cuh"
 
+#include <mutex>
+
 namespace gs {
 namespace {
 
@@ -215,3 +217,62 @@ gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s) {
 }
 
 }  // namespace gs
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the packing index step (count + scan).
+//
+// The per-(chunk, 16-row window) counts that gs_pack keeps in a cudaMalloc'd
+// temporary live here in a fixed array in the library's own device memory, so
+// gs_pack_index_noalloc never allocates.  Every call reuses (and overwrites)
+// the same array; the count kernel writes every entry it later reads, so no
+// entry needs clearing between calls.  Calls whose kernels overlap on the GPU
+// (concurrent streams) race on this array and must be serialized.
+// ---------------------------------------------------------------------------
+namespace gs {
+namespace {
+
+constexpr int64_t kNoAllocMaxEntries = int64_t(1) << 20;   // chunks x 16-row windows (4 MiB of int32)
+static __device__ __align__(256) int32_t g_noalloc_counts[kNoAllocMaxEntries];
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+int32_t* g_noalloc_ptr[kNoAllocMaxDevices] = {nullptr};
+
+// Device address of the counts array on the current device; resolved once per
+// device (with that device current) and cached.
+gs_status noalloc_counts_address(int32_t** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return GS_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    int32_t* ptr = nullptr;
+    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&ptr), g_noalloc_counts) != cudaSuccess || !ptr)
+      return GS_ERR_CUDA;
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return GS_OK;
+}
+
+}  // namespace
+}  // namespace gs
+
+extern "C" gs_status gs_pack_index_noalloc(const uint8_t* mask_dev, int64_t out, int64_t in, int64_t* offsets_dev,
+                                           int32_t* win_off16_dev, uint16_t* kmask16_dev, void* stream) {
+  using namespace gs;
+  if (!mask_dev || !offsets_dev || !win_off16_dev || !kmask16_dev) return GS_ERR_INVALID_ARG;
+  if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX || in % kGroupIn != 0) return GS_ERR_INVALID_ARG;
+  const int64_t G = in / kGroupIn;
+  const int64_t nw16 = (out + kWin16 - 1) / kWin16;
+  if (G * nw16 > kNoAllocMaxEntries) return GS_ERR_UNSUPPORTED;   // beyond the fixed scratch array
+  int32_t* counts = nullptr;
+  const gs_status st = noalloc_counts_address(&counts);
+  if (st != GS_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t E = G * nw16;
+  k_pack_count<<<grid_for(E, 256), 256, 0, s>>>(mask_dev, (int32_t)out, (int32_t)G, (int32_t)nw16, kmask16_dev,
+                                                counts);
+  k_pack_scan<<<1, kScanThreads, 0, s>>>(counts, (int32_t)G, (int32_t)nw16, win_off16_dev, offsets_dev);
+  note_launch(2);
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
