@@ -1,22 +1,23 @@
 // Prefill-regime group-sparse linear (many tokens, tensor-core bound):
 //   y[t, r] = sum over kept groups (r, c) of X_c[t, :] . W[r, 256c : 256c+256]   (Eq. 1)
 //
-// Tile = 128 tokens x 192 output rows (a "window").  For every chunk c the kept
+// Tile = 128 tokens x 160 output rows (a "window").  For every chunk c the kept
 // rows of the window form one contiguous slice of the packed tiles (rows are
 // ascending inside a chunk), so the slice is a dense K-major operand that TMA
-// loads as-is.  Per (chunk, slice of <= 160 kept rows) one tcgen05 MMA chain
-// computes D[128 tok x n] = X_c . W_slice^T into a TMEM scratch buffer; the
-// epilogue warps then add scratch column j into accumulator column
-// row_idx[j] - 192*window (TMEM-resident, 192 columns).  W (.) M is never
+// loads as-is.  Per chunk one tcgen05 MMA chain computes D[128 tok x n] =
+// X_c . W_slice^T (n <= 160 kept rows) into a TMEM scratch buffer; the
+// epilogue warps then gather each window row's scratch column (or a zero
+// column when the row is pruned in that chunk) into the TMEM-resident
+// 128 x 160 accumulator.  W (.) M is never
 // materialised and pruned groups cost neither bytes nor FLOPs.  Two scratch
 // buffers let the MMA of the next slice overlap the scatter-add of this one.
 //
 // Roles (one CTA per SM, persistent over tiles):
 //   warp 0      TMA producer (X box 128x64, W boxes of 128/64/32/16 rows)
 //   warp 1      TMEM allocator + single-thread MMA issuer
-//   warps 2..9  epilogue: scatter-add, then accumulator -> bf16 y
+//   warps 2..9  epilogue: gather-add into the accumulator, then accumulator -> bf16 y
 // Each warp stages the window's per-chunk slice bounds in shared memory at the
-// start of a tile, so no role waits on global metadata per item.  Every
+// start of a tile; the epilogue prefetches its blocks' masks one item ahead.  Every
 // mbarrier wait is bounded; a wait that runs out raises a CTA-wide abort flag
 // and the library's device error flag, and all roles wind down.
 #include "gs_common.cuh"
@@ -31,9 +32,11 @@ namespace {
 using namespace sm100;
 
 constexpr int kBM = 128;                      // tokens per tile (TMEM lanes)
-constexpr int kFW = 192;                      // output rows per tile (accumulator columns)
+constexpr int kFW = 160;                      // output rows per tile (accumulator columns)
 constexpr int kHalf = kFW / 2;                // accumulator columns owned by one epilogue warp
-constexpr int kNMax = 160;                    // kept rows per MMA item (scratch columns)
+constexpr int kBlkRows = kWin16;              // accumulator block handled per gather round
+constexpr int kBlocksPerHalf = kHalf / kBlkRows;   // 5
+constexpr int kNMax = kFW;                    // kept rows per MMA item: a whole window's slice always fits
 constexpr int kBK = 64;                       // k per pipeline stage: one 128-byte swizzle row
 constexpr int kKSteps = kGroupIn / kBK;       // 4 stages per 256-wide chunk
 constexpr int kStages = 5;
@@ -44,24 +47,25 @@ constexpr int kEpiWarps = 8;
 constexpr int kWarps = 2 + kEpiWarps;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMaxG = 256;                    // chunks per layer handled by this kernel (in <= 65536)
-constexpr int kMetaInts = 3 * kMaxG;          // per warp: slice start, end, and first row of the upper half
+constexpr int kMetaInts = 2 * kMaxG;          // per warp: slice start and end per chunk
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCol = 0;
 constexpr uint32_t kScrCol = kFW;             // two scratch buffers of kNMax columns
+constexpr uint32_t kZeroCol = kScrCol + 2 * kNMax;   // 32 columns kept at 0.0 (gather target of pruned rows)
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
 constexpr int kSmemBytes = kStages * kStageBytes + kWarps * kMetaInts * 4 + 1024;
 
-static_assert(kScrCol + 2 * kNMax <= kTmemCols, "TMEM budget");
+static_assert(kZeroCol + 32 <= kTmemCols, "TMEM budget");
 static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
-static_assert(kFW % 16 == 0 && kHalf % 32 == 0 && kNMax % 32 == 0, "tile shape");
+static_assert(kFW % 32 == 0 && kHalf % kBlkRows == 0 && kNMax % 16 == 0, "tile shape");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 struct PrefillParams {
   CUtensorMap xmap;        // x [T][in] bf16, box 64 x 128
   CUtensorMap wmap[4];     // tiles [kept][256] bf16, box 64 x {128, 64, 32, 16}
-  const int32_t* row_idx;
   const int32_t* win_off16;
+  const uint16_t* kmask16;
   uint16_t* y;
   int32_t out, G, nw16, T;
   int32_t n_m, n_w;
@@ -74,58 +78,57 @@ __device__ __forceinline__ uint32_t pack_bf16x2(uint32_t lo, uint32_t hi) {
 }
 
 // Per-warp copy of a tile's slice bounds: for chunk c the window's kept rows
-// are packed rows [p0[c], p1[c]); rows of the upper accumulator half start at pm[c].
+// are packed rows [p0[c], p1[c]).
 struct TileMeta {
   int32_t* p0;
   int32_t* p1;
-  int32_t* pm;
 };
 
 __device__ __forceinline__ void load_tile_meta(const PrefillParams& P, int w, int lane, const TileMeta& M) {
   const int wlo = (kFW / kWin16) * w;
   const int whi = min(wlo + kFW / kWin16, P.nw16);
-  const int wmid = min(wlo + kHalf / kWin16, P.nw16);
   for (int c = lane; c < P.G; c += 32) {
     const int32_t* wo = P.win_off16 + (int64_t)c * (P.nw16 + 1);
     M.p0[c] = wo[wlo];
     M.p1[c] = wo[whi];
-    M.pm[c] = wo[wmid];
   }
   __syncwarp();
 }
 
-// Items of a tile: chunk c = 0..G-1, slice cut into pieces of <= kNMax rows.
-struct Item {
-  int c, start, end;
-};
-__device__ __forceinline__ bool item_scan(const PrefillParams& P, const TileMeta& M, int c0, Item& it) {
-  for (int c = c0; c < P.G; ++c) {
-    const int p0 = M.p0[c], p1 = M.p1[c];
-    if (p1 > p0) {
-      it.c = c;
-      it.start = p0;
-      it.end = p1;
-      return true;
-    }
-  }
-  return false;
-}
-__device__ __forceinline__ bool item_next(const PrefillParams& P, const TileMeta& M, Item& it) {
-  if (it.start + kNMax < it.end) {
-    it.start += kNMax;
-    return true;
-  }
-  return item_scan(P, M, it.c + 1, it);
+// Items of a tile: the chunks whose window slice is non-empty, in order.
+__device__ __forceinline__ int item_next(const PrefillParams& P, const TileMeta& M, int c) {
+  for (++c; c < P.G; ++c)
+    if (M.p1[c] > M.p0[c]) return c;
+  return P.G;
 }
 
-// lane l receives the output rows of item columns l, 32+l, ..., 128+l
-__device__ __forceinline__ void load_dst(const PrefillParams& P, const Item& it, bool have, int lane,
-                                         int (&d)[kNMax / 32]) {
-#pragma unroll
-  for (int b = 0; b < kNMax / 32; ++b) {
-    const int j = it.start + 32 * b + lane;
-    d[b] = (have && j < it.end && j < it.start + kNMax) ? __ldg(P.row_idx + j) : 0;
+// lanes 0..4 fetch (window offset, kept mask) of the five 16-row blocks of an
+// epilogue warp's accumulator half for chunk c
+__device__ __forceinline__ void load_blocks(const PrefillParams& P, int c, int wblk0, int lane, int& woff,
+                                            uint32_t& km) {
+  const int wi = wblk0 + lane;
+  woff = 0;
+  km = 0u;
+  if (c < P.G && lane < kBlocksPerHalf && wi < P.nw16) {
+    woff = __ldg(P.win_off16 + (int64_t)c * (P.nw16 + 1) + wi);
+    km = __ldg(P.kmask16 + (int64_t)c * P.nw16 + wi);
   }
+}
+
+__device__ __forceinline__ void tmem_ld_x16b(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+        "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
 }
 
 __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
@@ -141,7 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int32_t* meta_base = reinterpret_cast<int32_t*>(smem + kStages * kStageBytes) + warp * kMetaInts;
-  const TileMeta M{meta_base, meta_base + kMaxG, meta_base + 2 * kMaxG};
+  const TileMeta M{meta_base, meta_base + kMaxG};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -179,11 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
       const int m = t % P.n_m, w = t / P.n_m;
       load_tile_meta(P, w, lane, M);
       if (lane == 0) {
-        Item it;
-        bool have = item_scan(P, M, 0, it);
-        for (; have && ok; have = item_next(P, M, it)) {
-          const int n = min(kNMax, it.end - it.start);
-          const int nr = (n + 15) & ~15;
+        for (int c = item_next(P, M, -1); c < P.G && ok; c = item_next(P, M, c)) {
+          const int start = M.p0[c];
+          const int nr = (M.p1[c] - start + 15) & ~15;
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kWaitLimitNs,
                                    kDevErrTimeout)) {
@@ -193,13 +194,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
             uint8_t* sx = smem + stage * kStageBytes;
             uint8_t* sw = sx + kXStageBytes;
             mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(kXStageBytes + nr * kBK * 2));
-            tma_load_2d(sx, &P.xmap, &full_bar[stage], it.c * kGroupIn + ks * kBK, m * kBM);
+            tma_load_2d(sx, &P.xmap, &full_bar[stage], c * kGroupIn + ks * kBK, m * kBM);
             int rr = 0;
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
               const int hh = 128 >> h;
               while (nr - rr >= hh) {
-                tma_load_2d(sw + rr * (kBK * 2), &P.wmap[h], &full_bar[stage], ks * kBK, it.start + rr);
+                tma_load_2d(sw + rr * (kBK * 2), &P.wmap[h], &full_bar[stage], ks * kBK, start + rr);
                 rr += hh;
               }
             }
@@ -233,11 +234,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
       const int w = t / P.n_m;
       load_tile_meta(P, w, lane, M);
       if (lane == 0) {
-        Item it;
-        bool have = item_scan(P, M, 0, it);
-        for (; have && ok; have = item_next(P, M, it)) {
-          const int n = min(kNMax, it.end - it.start);
-          const int nr = (n + 15) & ~15;
+        for (int c = item_next(P, M, -1); c < P.G && ok; c = item_next(P, M, c)) {
+          const int nr = (M.p1[c] - M.p0[c] + 15) & ~15;
           if (!mbar_wait_bounded(&sempty_bar[buf], se_ph[buf] ^ 1u, abort_flag, P.err, kWaitLimitNs,
                                  kDevErrTimeout)) {
             ok = false;
@@ -281,38 +279,42 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
   } else {
     // ------------------------------------------------------------ epilogue
     // Warp (q, h): TMEM lane quarter q (tokens 32q..32q+31) and accumulator
-    // half h (columns kHalf*h .. kHalf*h + kHalf - 1, window rows likewise).
-    // Kept rows are ascending inside an item, so the item's columns landing in
-    // half 0 are a prefix [0, jsplit) and the rest land in half 1: every
-    // accumulator column is only ever touched by one warp.
+    // half h (window rows 80h .. 80h+79, five 16-row blocks).  For each item
+    // (chunk) and block the warp gathers its rows' scratch columns: row i of
+    // a block with kept mask m reads scratch column b0 + popc(m & (2^i - 1))
+    // when kept and a column held at zero otherwise, then adds the 16 values
+    // into the block with one 16-column load and store.  Every accumulator
+    // column belongs to one warp, and no single-column TMEM store is needed.
     const int ew = warp - 2;
     const int q = warp & 3;
     const int h = ew >> 2;
     const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-    const uint32_t t_acc = tmem + lane_off + kAccCol;
+    const uint32_t t_acc = tmem + lane_off + kAccCol + (uint32_t)(kHalf * h);
     const uint32_t t_scr = tmem + lane_off + kScrCol;
+    const uint32_t t_zero = tmem + lane_off + kZeroCol;
+    tmem_st_x32_zero(t_zero);
     int buf = 0;
     uint32_t sf_ph[2] = {0u, 0u};
     bool ok = true;
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
       const int m = t % P.n_m, w = t / P.n_m;
-      const int r0 = w * kFW;
+      const int r0 = w * kFW + kHalf * h;
+      const int wblk0 = (kFW / kWin16) * w + kBlocksPerHalf * h;
       load_tile_meta(P, w, lane, M);
+      {
+        const uint32_t z[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
 #pragma unroll
-      for (int col = 0; col < kHalf; col += 32) tmem_st_x32_zero(t_acc + kHalf * h + col);
+        for (int k = 0; k < kBlocksPerHalf; ++k) tmem_st_x16(t_acc + kBlkRows * k, z);
+      }
       tmem_wait_st();
-      Item it;
-      bool have = item_scan(P, M, 0, it);
-      int dreg[kNMax / 32];
-      load_dst(P, it, have, lane, dreg);
-      while (have && ok) {
-        Item nx = it;
-        const bool have_nx = item_next(P, M, nx);
-        int ndreg[kNMax / 32];
-        load_dst(P, nx, have_nx, lane, ndreg);            // prefetch the next item's rows
-        const int n = min(kNMax, it.end - it.start);
-        const int jsplit = min(max(M.pm[it.c] - it.start, 0), n);
-        const int jlo = h ? jsplit : 0, jhi = h ? n : jsplit;
+      int c = item_next(P, M, -1);
+      int woff, nwoff;
+      uint32_t km, nkm;
+      load_blocks(P, c, wblk0, lane, woff, km);
+      while (c < P.G && ok) {
+        const int cn = item_next(P, M, c);
+        load_blocks(P, cn, wblk0, lane, nwoff, nkm);      // prefetch the next item's block metadata
+        const int p0 = M.p0[c];
         if (!mbar_wait_bounded(&sfull_bar[buf], sf_ph[buf], abort_flag, P.err, kWaitLimitNs, kDevErrTimeout)) {
           ok = false;
           break;
@@ -321,56 +323,54 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
         tc_fence_after();
         const uint32_t scr = t_scr + (uint32_t)(buf * kNMax);
 #pragma unroll
-        for (int b = 0; b < kNMax / 32; ++b) {
-          if (32 * b + 32 <= jlo || 32 * b >= jhi) continue;
-          uint32_t sv[32], av[32], col[32];
-          tmem_ld_x32(scr + (uint32_t)(32 * b), sv);
+        for (int k = 0; k < kBlocksPerHalf; ++k) {
+          const uint32_t mk = __shfl_sync(0xffffffffu, km, k);
+          if (mk == 0u) continue;
+          const int b0 = __shfl_sync(0xffffffffu, woff, k) - p0;   // scratch column of the block's first kept row
+          const int li = lane & (kBlkRows - 1);
+          const uint32_t my_addr = ((mk >> li) & 1u) ? scr + (uint32_t)(b0 + __popc(mk & ((1u << li) - 1u))) : t_zero;
+          uint32_t a[kBlkRows], g[kBlkRows];
+          tmem_ld_x16b(t_acc + kBlkRows * k, a);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            col[j] = (uint32_t)(__shfl_sync(0xffffffffu, dreg[b], j) - r0);
-            av[j] = 0u;
-            if (32 * b + j >= jlo && 32 * b + j < jhi) av[j] = tmem_ld_x1(t_acc + col[j]);
-          }
+          for (int i = 0; i < kBlkRows; ++i) g[i] = tmem_ld_x1(__shfl_sync(0xffffffffu, my_addr, i));
           tmem_wait_ld();
-          reg_fence(sv);
-          reg_fence(av);
+          reg_fence(a);
+          reg_fence(g);
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (32 * b + j >= jlo && 32 * b + j < jhi)
-              tmem_st_x1(t_acc + col[j], __float_as_uint(__uint_as_float(av[j]) + __uint_as_float(sv[j])));
+          for (int i = 0; i < kBlkRows; ++i) a[i] = __float_as_uint(__uint_as_float(a[i]) + __uint_as_float(g[i]));
+          tmem_st_x16(t_acc + kBlkRows * k, a);
         }
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sempty_bar[buf]);
         buf ^= 1;
-        it = nx;
-        have = have_nx;
-#pragma unroll
-        for (int b = 0; b < kNMax / 32; ++b) dreg[b] = ndreg[b];
+        c = cn;
+        woff = nwoff;
+        km = nkm;
       }
       if (!ok) break;
-      // own accumulator half -> bf16 y rows [r0 + kHalf*h, r0 + kHalf*h + kHalf) of token tok
+      // own accumulator half -> bf16 y rows [r0, r0 + kHalf) of token tok
       const int tok = m * kBM + 32 * q + lane;
       uint16_t* yrow = P.y + (int64_t)tok * P.out;
       const bool vec_ok = (P.out & 7) == 0;
 #pragma unroll 1
-      for (int col = 0; col < kHalf; col += 32) {
-        uint32_t v[32];
-        tmem_ld_x32(t_acc + kHalf * h + col, v);
+      for (int col = 0; col < kHalf; col += kBlkRows) {
+        uint32_t v[kBlkRows];
+        tmem_ld_x16b(t_acc + col, v);
         tmem_wait_ld();
         reg_fence(v);
-        const int rb = r0 + kHalf * h + col;
+        const int rb = r0 + col;
         if (tok < P.T && rb < P.out) {
-          if (vec_ok && rb + 32 <= P.out) {
+          if (vec_ok && rb + kBlkRows <= P.out) {
             uint4* dst = reinterpret_cast<uint4*>(yrow + rb);
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+            for (int u = 0; u < 2; ++u)
               dst[u] = make_uint4(pack_bf16x2(v[8 * u + 0], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
                                   pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
           } else {
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
+            for (int i = 0; i < kBlkRows; ++i)
               if (rb + i < P.out) yrow[rb + i] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[i])));
           }
         }
@@ -434,8 +434,8 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
   std::memset(&P, 0, sizeof(P));
   if (!encode_tmap_2d_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBK, kBM, true)) return GS_ERR_CUDA;
   for (int h = 0; h < 4; ++h) std::memcpy(&P.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
-  P.row_idx = p->row_idx;
   P.win_off16 = p->win_off16;
+  P.kmask16 = p->kmask16;
   P.y = static_cast<uint16_t*>(y);
   P.out = (int32_t)p->out;
   P.G = p->G;
