@@ -106,6 +106,24 @@ class ClockSampler:
                 "power_w_max": max((float(r[3]) for r in rows if r[3].replace(".", "").isdigit()), default=None)}
 
 
+# ----------------------------------------------------------------------------- multi-rank helpers
+def max_over_ranks(x: float, dist=None, device=None) -> float:
+    """The maximum of a per-rank float over all ranks (the job's wall time is the
+    slowest rank's); identity without a process group."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank_step: float, steps: int, elapsed_max: float, world: int) -> float:
+    """Throughput of the whole job: every rank processes the same units per step
+    (independent replicas), divided by the slowest rank's time."""
+    return world * units_per_rank_step * steps / elapsed_max
+
+
 # ----------------------------------------------------------------------------- traffic record
 def kernel_source_hash(name: str) -> str:
     return hashlib.sha256((ROOT / "paper_2609_33977_gb300" / "csrc" / name).read_bytes()).hexdigest()[:16]
@@ -315,13 +333,9 @@ def run_ours(args):
     # graph replays do not go through the library's launch counter: count the
     # kernels they contain (one decode launch per token batch per step)
     launches = args.steps * launches_per_step + (gs.launch_count() - n0)
-    elapsed = ev0.elapsed_time(ev1) / 1e3
-    if dist is not None:
-        t = torch.tensor([elapsed], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = max_over_ranks(ev0.elapsed_time(ev1) / 1e3, dist, dev)
     tokens_per_step = sum(DECODE_T)
-    value = world * tokens_per_step * args.steps / elapsed
+    value = whole_job_rate(tokens_per_step, args.steps, elapsed, world)
     bytes_per_step = sum(decode_bytes(layers, T) for T in DECODE_T)
     achieved_gbs = bytes_per_step * args.steps / elapsed / 1e9
 
