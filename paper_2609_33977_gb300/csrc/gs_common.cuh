@@ -39,8 +39,8 @@ struct gs_packed {
   int4* dmeta;        // [nblk64][G]: {first packed row of the block's slice, kept masks of its 4 windows, 0}
   float* dec_ws;      // [nblk64][dec_nsplit][4][16 tokens][16 rows] partial sums (dec_nsplit > 1)
   int32_t* dec_cnt;   // [nblk64][4] arrival counters (self-resetting)
-  // tcgen05 prefill: TMA descriptors over the tiles (box heights 128/64/32/16 rows)
-  alignas(64) unsigned char wmaps[4][128];
+  // tcgen05 prefill: slab TMA descriptors over the tiles, box heights 16, 32, ..., 160 rows
+  alignas(64) unsigned char wmaps[10][128];
   bool wmaps_valid;
 };
 
@@ -49,6 +49,13 @@ namespace gs {
 // 2-D bf16 TMA descriptor (map: 128-byte, 64-byte aligned buffer); false on failure
 bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
                          uint32_t box_outer, bool swizzle128);
+
+// 3-D "slab" bf16 descriptor over a row-major [rows][row_elems] matrix: a box
+// of box_rows rows x box_slabs 64-element slabs lands in shared memory as
+// box_slabs consecutive [box_rows][64] blocks, each with the 128-byte swizzle
+// that tcgen05's K-major operand descriptors expect.  row_elems % 64 == 0.
+bool encode_tmap_slabs_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows, uint32_t box_rows,
+                            uint32_t box_slabs);
 
 // library-owned per-device error flag (allocated on first use)
 int* device_error_flag();

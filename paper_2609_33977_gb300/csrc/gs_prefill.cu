@@ -5,21 +5,30 @@
 // rows of the window form one contiguous slice of the packed tiles (rows are
 // ascending inside a chunk), so the slice is a dense K-major operand that TMA
 // loads as-is.  Per chunk one tcgen05 MMA chain computes D[128 tok x n] =
-// X_c . W_slice^T (n <= 160 kept rows) into a TMEM scratch buffer; the
-// epilogue warps then gather each window row's scratch column (or a zero
-// column when the row is pruned in that chunk) into the TMEM-resident
-// 128 x 160 accumulator.  W (.) M is never
-// materialised and pruned groups cost neither bytes nor FLOPs.  Two scratch
-// buffers let the MMA of the next slice overlap the scatter-add of this one.
+// X_c . W_slice^T (n <= 160 kept rows, rounded up to 16) into one of three
+// TMEM scratch buffers; the epilogue warps then add each window row's scratch
+// column (a zero column for rows pruned in chunk c) into the window
+// accumulator, which they hold in registers.  W (.) M
+// is never materialised and pruned groups cost neither bytes nor FLOPs.
+//
+// Copies: a pipeline stage carries 128 of the chunk's 256 k as two 64-wide
+// slabs, fetched with one 3-D TMA box for X (128 rows x 2 slabs) and one for
+// the W slice (n rows x 2 slabs, from a descriptor whose box height is n).
+// TMA issue costs a fixed ~60-120 cycles per box whatever its size, so two
+// large boxes per stage keep the producer far below the copy time.
 //
 // Roles (one CTA per SM, persistent over tiles):
-//   warp 0      TMA producer (X box 128x64, W boxes of 128/64/32/16 rows)
+//   warp 0      TMA producer
 //   warp 1      TMEM allocator + single-thread MMA issuer
-//   warps 2..9  epilogue: gather-add into the accumulator, then accumulator -> bf16 y
+//   warps 2..17 epilogue: warp (q, g) owns tokens 32q..32q+31 (its TMEM lane
+//               quarter) and window rows 40g..40g+39: 40 fp32 accumulators
+//               per thread, updated from 40 single-column TMEM loads per chunk
+//               (pruned rows read a zero column) with one wait, then written
+//               to y as bf16 at the end of the tile.
 // Each warp stages the window's per-chunk slice bounds in shared memory at the
-// start of a tile; the epilogue prefetches its blocks' masks one item ahead.  Every
-// mbarrier wait is bounded; a wait that runs out raises a CTA-wide abort flag
-// and the library's device error flag, and all roles wind down.
+// start of a tile; the epilogue prefetches its blocks' masks four chunks ahead.
+// Every mbarrier wait is bounded; a wait that runs out raises a CTA-wide abort
+// flag and the library's device error flag, and all roles wind down.
 #include "gs_common.cuh"
 #include "gs_sm100.cuh"
 
@@ -31,160 +40,186 @@ namespace gs {
 namespace {
 using namespace sm100;
 
-constexpr int kBM = 128;                      // tokens per tile (TMEM lanes)
-constexpr int kFW = 160;                      // output rows per tile (accumulator columns)
-constexpr int kHalf = kFW / 2;                // accumulator columns owned by one epilogue warp
-constexpr int kBlkRows = kWin16;              // accumulator block handled per gather round
-constexpr int kBlocksPerHalf = kHalf / kBlkRows;   // 5
+constexpr int kBM = 128;                      // tokens per CTA (TMEM lanes); a CTA pair covers 256
+constexpr int kPairM = 2 * kBM;               // tokens per pair tile
+constexpr int kFW = 160;                      // output rows per tile (a window)
+constexpr int kGroups = 4;                    // epilogue warps per TMEM lane quarter
+constexpr int kRowsPerWarp = kFW / kGroups;   // 40 window rows per epilogue warp
+constexpr int kBlkRows = kWin16;              // rows per kept-mask block
+constexpr int kMetaBlocks = 3;                // 16-row blocks a warp's 40 rows can touch
 constexpr int kNMax = kFW;                    // kept rows per MMA item: a whole window's slice always fits
-constexpr int kBK = 64;                       // k per pipeline stage: one 128-byte swizzle row
-constexpr int kKSteps = kGroupIn / kBK;       // 4 stages per 256-wide chunk
-constexpr int kStages = 5;
-constexpr int kXStageBytes = kBM * kBK * 2;   // 16 KB
-constexpr int kWStageBytes = kNMax * kBK * 2; // 20 KB
-constexpr int kStageBytes = kXStageBytes + kWStageBytes;
-constexpr int kEpiWarps = 8;
+constexpr int kNMaps = kNMax / 16;            // W descriptors, box heights 8, 16, ..., 80 (half a slice each)
+constexpr int kBK = 64;                       // k per slab: one 128-byte swizzle row
+constexpr int kSlabs = 2;                     // slabs per pipeline stage (a stage carries 128 k)
+constexpr int kKSteps = kGroupIn / (kBK * kSlabs);   // 2 stages per 256-wide chunk
+constexpr int kStages = 4;
+constexpr int kXSlabBytes = kBM * kBK * 2;    // 16 KB
+constexpr int kXStageBytes = kSlabs * kXSlabBytes;
+constexpr int kWStageBytes = kSlabs * (kNMax / 2) * kBK * 2;   // 20 KB: this CTA's half of the largest slice
+constexpr int kStageBytes = kXStageBytes + kWStageBytes;       // 52 KB
+constexpr int kScrBufs = 3;                   // TMEM scratch buffers (MMA runs up to two chunks ahead)
+constexpr int kEpiWarps = 4 * kGroups;
 constexpr int kWarps = 2 + kEpiWarps;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMaxG = 256;                    // chunks per layer handled by this kernel (in <= 65536)
-constexpr int kMetaInts = 2 * kMaxG;          // per warp: slice start and end per chunk
+constexpr int kMetaInts = 2 * kMaxG;          // producer / MMA warp: a tile's item list (int2 per chunk)
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAccCol = 0;
-constexpr uint32_t kScrCol = kFW;             // two scratch buffers of kNMax columns
-constexpr uint32_t kZeroCol = kScrCol + 2 * kNMax;   // 32 columns kept at 0.0 (gather target of pruned rows)
+constexpr int kAcc = kRowsPerWarp;            // 40 accumulators per epilogue thread
+constexpr uint32_t kZeroCol = kScrBufs * kNMax;   // 32 columns held at 0.0: the gather source of pruned rows
+constexpr int kTblBytes = 2 * kEpiWarps * kAcc * 4;   // per epilogue warp, two chunks: the TMEM address of each row
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
-constexpr int kSmemBytes = kStages * kStageBytes + kWarps * kMetaInts * 4 + 1024;
+constexpr int kSmemBytes = kStages * kStageBytes + 2 * kMetaInts * 4 + kTblBytes + 1024;
 
-static_assert(kZeroCol + 32 <= kTmemCols, "TMEM budget");
-static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
-static_assert(kFW % 32 == 0 && kHalf % kBlkRows == 0 && kNMax % 16 == 0, "tile shape");
+static_assert(kZeroCol + 32 <= kTmemCols, "TMEM budget (scratch buffers + zero columns)");
+static_assert(kStageBytes % 1024 == 0 && kXSlabBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+static_assert(kFW % 32 == 0 && kRowsPerWarp % 8 == 0 && kNMax % 16 == 0, "tile shape");
+static_assert(kRowsPerWarp <= 32 + 8, "the address table is built in two lane rounds");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 struct PrefillParams {
-  CUtensorMap xmap;        // x [T][in] bf16, box 64 x 128
-  CUtensorMap wmap[4];     // tiles [kept][256] bf16, box 64 x {128, 64, 32, 16}
+  CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 2
+  CUtensorMap wmap[kNMaps];  // tiles as (64, kept, 4) slabs, box 64 x 8(i+1) x 2
   const int32_t* win_off16;
   const uint16_t* kmask16;
   uint16_t* y;
   int32_t out, G, nw16, T;
-  int32_t n_m, n_w;
+  int32_t n_m, n_w;          // pair tiles: ceil(T / 256) x ceil(out / 160)
   int* err;
 };
 
-__device__ __forceinline__ uint32_t pack_bf16x2(uint32_t lo, uint32_t hi) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(lo), __uint_as_float(hi));
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// Per-warp copy of a tile's slice bounds: for chunk c the window's kept rows
-// are packed rows [p0[c], p1[c]).
-struct TileMeta {
-  int32_t* p0;
-  int32_t* p1;
-};
-
-__device__ __forceinline__ void load_tile_meta(const PrefillParams& P, int w, int lane, const TileMeta& M) {
+// Items of a tile: the chunks whose window slice (kept rows = packed rows
+// [p0, p1)) is non-empty, in chunk order.  The warp builds the list in shared
+// memory, 32 chunks per round: entry = {chunk | (rows rounded up to 16) << 16, p0}.
+__device__ __forceinline__ int load_tile_items(const PrefillParams& P, int w, int lane, int2* items) {
   const int wlo = (kFW / kWin16) * w;
   const int whi = min(wlo + kFW / kWin16, P.nw16);
-  for (int c = lane; c < P.G; c += 32) {
-    const int32_t* wo = P.win_off16 + (int64_t)c * (P.nw16 + 1);
-    M.p0[c] = wo[wlo];
-    M.p1[c] = wo[whi];
+  int n = 0;
+  for (int c0 = 0; c0 < P.G; c0 += 32) {
+    const int c = c0 + lane;
+    int p0 = 0, p1 = 0;
+    if (c < P.G) {
+      const int32_t* wo = P.win_off16 + (int64_t)c * (P.nw16 + 1);
+      p0 = wo[wlo];
+      p1 = wo[whi];
+    }
+    const bool nonempty = p1 > p0;
+    const uint32_t ballot = __ballot_sync(0xffffffffu, nonempty);
+    if (nonempty)
+      items[n + __popc(ballot & ((1u << lane) - 1u))] = make_int2(c | (((p1 - p0 + 15) & ~15) << 16), p0);
+    n += __popc(ballot);
   }
   __syncwarp();
+  return n;
 }
 
-// Items of a tile: the chunks whose window slice is non-empty, in order.
-__device__ __forceinline__ int item_next(const PrefillParams& P, const TileMeta& M, int c) {
-  for (++c; c < P.G; ++c)
-    if (M.p1[c] > M.p0[c]) return c;
-  return P.G;
-}
-
-// lanes 0..4 fetch (window offset, kept mask) of the five 16-row blocks of an
-// epilogue warp's accumulator half for chunk c
-__device__ __forceinline__ void load_blocks(const PrefillParams& P, int c, int wblk0, int lane, int& woff,
-                                            uint32_t& km) {
-  const int wi = wblk0 + lane;
+// Chunk c's metadata for an epilogue warp: lanes 0..2 fetch (window offset,
+// kept mask) of the 16-row blocks its 40 rows touch (from block wblk0); lanes
+// 30 and 31 fetch the window slice's start and end.  Chunks past the last read as empty.
+__device__ __forceinline__ void load_chunk_meta(const PrefillParams& P, int c, int wlo, int whi, int wblk0, int lane,
+                                                int& bnd, int& woff, uint32_t& km) {
+  bnd = 0;
   woff = 0;
   km = 0u;
-  if (c < P.G && lane < kBlocksPerHalf && wi < P.nw16) {
-    woff = __ldg(P.win_off16 + (int64_t)c * (P.nw16 + 1) + wi);
+  if (c >= P.G) return;
+  const int32_t* wo = P.win_off16 + (int64_t)c * (P.nw16 + 1);
+  const int wi = wblk0 + lane;
+  if (lane < kMetaBlocks && wi < P.nw16) {
+    woff = __ldg(wo + wi);
     km = __ldg(P.kmask16 + (int64_t)c * P.nw16 + wi);
+  }
+  if (lane == 30) bnd = __ldg(wo + wlo);
+  if (lane == 31) bnd = __ldg(wo + whi);
+}
+
+// acc[0..n) += v[0..n), two lanes per packed f32x2 add
+template <int N>
+__device__ __forceinline__ void add_f32x2(float* acc, const uint32_t* v) {
+#pragma unroll
+  for (int j = 0; j < N; j += 2)
+    asm("{\n\t.reg .b64 a, b;\n\t"
+        "mov.b64 a, {%0, %1};\n\t"
+        "mov.b64 b, {%2, %3};\n\t"
+        "add.rn.f32x2 a, a, b;\n\t"
+        "mov.b64 {%0, %1}, a;\n\t}"
+        : "+f"(acc[j]), "+f"(acc[j + 1])
+        : "r"(v[j]), "r"(v[j + 1]));
+}
+
+// Single-column TMEM loads of N rows whose addresses sit in shared memory.
+template <int N>
+__device__ __forceinline__ void gather_rows(const uint32_t* tbl, uint32_t* v) {
+#pragma unroll
+  for (int j = 0; j < N; j += 4) {
+    const uint4 a = *reinterpret_cast<const uint4*>(tbl + j);
+    v[j + 0] = tmem_ld_x1(a.x);
+    v[j + 1] = tmem_ld_x1(a.y);
+    v[j + 2] = tmem_ld_x1(a.z);
+    v[j + 3] = tmem_ld_x1(a.w);
   }
 }
 
-__device__ __forceinline__ void tmem_ld_x16b(uint32_t taddr, uint32_t* v) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-        "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
-      : "r"(taddr)
-      : "memory");
-}
-__device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t* v) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
-      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
-        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
-      : "memory");
-}
-
-__global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ __align__(8) uint64_t empty_bar[kStages];
-  __shared__ __align__(8) uint64_t sfull_bar[2];
-  __shared__ __align__(8) uint64_t sempty_bar[2];
+  __shared__ __align__(8) uint64_t sfull_bar[kScrBufs];
+  __shared__ __align__(8) uint64_t sempty_bar[kScrBufs];
   __shared__ __align__(8) uint64_t drain_bar;
   __shared__ uint32_t tmem_base_s;
   __shared__ int abort_s;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int32_t* meta_base = reinterpret_cast<int32_t*>(smem + kStages * kStageBytes) + warp * kMetaInts;
-  const TileMeta M{meta_base, meta_base + kMaxG};
+  const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs), 1: peer
+  int2* items = reinterpret_cast<int2*>(smem + kStages * kStageBytes) + (warp < 2 ? warp : 0) * kMaxG;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kScrBufs; ++b) {
       mbar_init(&sfull_bar[b], 1);
-      mbar_init(&sempty_bar[b], kEpiWarps);
+      mbar_init(&sempty_bar[b], 2 * kEpiWarps);   // the epilogue warps of both CTAs
     }
     mbar_init(&drain_bar, 1);
     abort_s = 0;
     fence_mbar_init();
     prefetch_tmap(&P.xmap);
-    for (int h = 0; h < 4; ++h) prefetch_tmap(&P.wmap[h]);
+    for (int h = 0; h < kNMaps; ++h) prefetch_tmap(&P.wmap[h]);
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_s, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&tmem_base_s, kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   volatile int* abort_flag = &abort_s;
   const int n_tiles = P.n_m * P.n_w;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     uint32_t stage = 0, phase = 0;
-    int armed[kStages];
-    for (int s = 0; s < kStages; ++s) armed[s] = -1;
+    uint32_t armed = 0u, armed_par = 0u;   // per stage: a copy was issued / the phase it completes
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
       const int m = t % P.n_m, w = t / P.n_m;
-      load_tile_meta(P, w, lane, M);
+      const int n_items = load_tile_items(P, w, lane, items);
       if (lane == 0) {
-        for (int c = item_next(P, M, -1); c < P.G && ok; c = item_next(P, M, c)) {
-          const int start = M.p0[c];
-          const int nr = (M.p1[c] - start + 15) & ~15;
+        for (int it = 0; it < n_items && ok; ++it) {
+          const int2 e = items[it];
+          const int c = e.x & 0xFFFF, nr = e.x >> 16, start = e.y;
+          const int hn = nr >> 1;   // slice rows held by each CTA of the pair
+          const CUtensorMap* wm = &P.wmap[(hn >> 3) - 1];
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kWaitLimitNs,
                                    kDevErrTimeout)) {
@@ -192,19 +227,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
               break;
             }
             uint8_t* sx = smem + stage * kStageBytes;
-            uint8_t* sw = sx + kXStageBytes;
-            mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(kXStageBytes + nr * kBK * 2));
-            tma_load_2d(sx, &P.xmap, &full_bar[stage], c * kGroupIn + ks * kBK, m * kBM);
-            int rr = 0;
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const int hh = 128 >> h;
-              while (nr - rr >= hh) {
-                tma_load_2d(sw + rr * (kBK * 2), &P.wmap[h], &full_bar[stage], ks * kBK, start + rr);
-                rr += hh;
-              }
-            }
-            armed[stage] = (int)phase;
+            // both CTAs' copies complete on the leader's full barrier, which
+            // expects the bytes of the two halves
+            if (rank == 0)
+              mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(2 * kXStageBytes + nr * kSlabs * kBK * 2));
+            const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+            tma_load_3d_pair(sx, &P.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+            tma_load_3d_pair(sx + kXStageBytes, wm, fb, 0, start + (int)rank * hn, ks * kSlabs);
+            armed |= 1u << stage;
+            armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
@@ -214,37 +245,37 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
-    if (lane == 0 && !ok) {
+    if (lane == 0 && !ok && rank == 0) {
       // let copies already in flight land before the CTA retires
       for (int s = 0; s < kStages; ++s) {
-        if (armed[s] < 0) continue;
+        if (!((armed >> s) & 1u)) continue;
         const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait(&full_bar[s], (uint32_t)armed[s]))
+        while (!mbar_try_wait(&full_bar[s], (armed_par >> s) & 1u))
           if (globaltimer_ns() - t0 > kDrainLimitNs) break;
       }
     }
     __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 && rank == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader CTA)
     uint32_t stage = 0, phase = 0;
     int buf = 0;
-    uint32_t se_ph[2] = {0u, 0u};
+    uint32_t se_ph = 0u;   // bit b: parity of scratch buffer b's next release
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
       const int w = t / P.n_m;
-      load_tile_meta(P, w, lane, M);
+      const int n_items = load_tile_items(P, w, lane, items);
       if (lane == 0) {
-        for (int c = item_next(P, M, -1); c < P.G && ok; c = item_next(P, M, c)) {
-          const int nr = (M.p1[c] - M.p0[c] + 15) & ~15;
-          if (!mbar_wait_bounded(&sempty_bar[buf], se_ph[buf] ^ 1u, abort_flag, P.err, kWaitLimitNs,
-                                 kDevErrTimeout)) {
+        for (int it = 0; it < n_items && ok; ++it) {
+          const int nr = items[it].x >> 16;
+          if (!mbar_wait_bounded_cluster(&sempty_bar[buf], ((se_ph >> buf) & 1u) ^ 1u, abort_flag, P.err,
+                                         kWaitLimitNs, kDevErrTimeout)) {
             ok = false;
             break;
           }
-          se_ph[buf] ^= 1u;
+          se_ph ^= 1u << buf;
           tc_fence_after();
-          const uint32_t d = tmem + kScrCol + (uint32_t)(buf * kNMax);
-          const uint32_t idesc = idesc_bf16_f32(kBM, nr);
+          const uint32_t d = tmem + (uint32_t)(buf * kNMax);
+          const uint32_t idesc = idesc_bf16_f32(kPairM, nr);
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&full_bar[stage], phase, abort_flag, P.err, kWaitLimitNs, kDevErrTimeout)) {
               ok = false;
@@ -252,126 +283,144 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
             }
             tc_fence_after();
             const uint32_t sx = smem_u32(smem + stage * kStageBytes);
-            const uint64_t ad = sdesc_sw128(sx);
-            const uint64_t bd = sdesc_sw128(sx + kXStageBytes);
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-              mma_bf16_ss(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc, (ks | kk) != 0 ? 1u : 0u);
-            mma_commit(&empty_bar[stage]);
+            for (int j = 0; j < kSlabs; ++j) {
+              const uint64_t ad = sdesc_sw128(sx + j * kXSlabBytes);
+              const uint64_t bd = sdesc_sw128(sx + kXStageBytes + j * (nr >> 1) * (kBK * 2));
+#pragma unroll
+              for (int kk = 0; kk < kBK / 16; ++kk)
+                mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
+                                 (ks | j | kk) != 0 ? 1u : 0u);
+            }
+            mma_commit_pair_mc(&empty_bar[stage], 0x3);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
             }
           }
           if (!ok) break;
-          mma_commit(&sfull_bar[buf]);
-          buf ^= 1;
+          mma_commit_pair_mc(&sfull_bar[buf], 0x3);
+          if (++buf == kScrBufs) buf = 0;
         }
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
     if (lane == 0) {
       // all MMAs issued by this thread have completed once drain_bar flips
-      mma_commit(&drain_bar);
+      mma_commit_pair(&drain_bar);
       mbar_wait_bounded(&drain_bar, 0u, nullptr, P.err, kWaitLimitNs, kDevErrTimeout);
     }
     __syncwarp();
-  } else {
+  } else if (warp >= 2) {
     // ------------------------------------------------------------ epilogue
-    // Warp (q, h): TMEM lane quarter q (tokens 32q..32q+31) and accumulator
-    // half h (window rows 80h .. 80h+79, five 16-row blocks).  For each item
-    // (chunk) and block the warp gathers its rows' scratch columns: row i of
-    // a block with kept mask m reads scratch column b0 + popc(m & (2^i - 1))
-    // when kept and a column held at zero otherwise, then adds the 16 values
-    // into the block with one 16-column load and store.  Every accumulator
-    // column belongs to one warp, and no single-column TMEM store is needed.
+    // Warp (q, g): TMEM lane quarter q (tokens 32q..32q+31) and window rows
+    // 40g .. 40g+39.
     const int ew = warp - 2;
     const int q = warp & 3;
-    const int h = ew >> 2;
-    const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-    const uint32_t t_acc = tmem + lane_off + kAccCol + (uint32_t)(kHalf * h);
-    const uint32_t t_scr = tmem + lane_off + kScrCol;
-    const uint32_t t_zero = tmem + lane_off + kZeroCol;
+    const int g = ew >> 2;
+    const uint32_t t_scr = tmem + ((uint32_t)(32 * q) << 16);
+    const uint32_t t_zero = t_scr + kZeroCol;
     tmem_st_x32_zero(t_zero);
+    tmem_wait_st();
+    uint32_t* tbl = reinterpret_cast<uint32_t*>(smem + kStages * kStageBytes + 2 * kMetaInts * 4) + ew * 2 * kAcc;
     int buf = 0;
-    uint32_t sf_ph[2] = {0u, 0u};
+    uint32_t sf_ph = 0u;   // bit b: parity of scratch buffer b's next fill
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
       const int m = t % P.n_m, w = t / P.n_m;
-      const int r0 = w * kFW + kHalf * h;
-      const int wblk0 = (kFW / kWin16) * w + kBlocksPerHalf * h;
-      load_tile_meta(P, w, lane, M);
-      {
-        const uint32_t z[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+      const int r0 = w * kFW + kRowsPerWarp * g;
+      const int wblk0 = (kFW / kWin16) * w + (kRowsPerWarp * g) / kBlkRows;
+      const int rsh = (kRowsPerWarp * g) % kBlkRows;   // the warp's first row within block wblk0
+      float acc[kAcc];
 #pragma unroll
-        for (int k = 0; k < kBlocksPerHalf; ++k) tmem_st_x16(t_acc + kBlkRows * k, z);
-      }
-      tmem_wait_st();
-      int c = item_next(P, M, -1);
-      int woff, nwoff;
-      uint32_t km, nkm;
-      load_blocks(P, c, wblk0, lane, woff, km);
-      while (c < P.G && ok) {
-        const int cn = item_next(P, M, c);
-        load_blocks(P, cn, wblk0, lane, nwoff, nkm);      // prefetch the next item's block metadata
-        const int p0 = M.p0[c];
-        if (!mbar_wait_bounded(&sfull_bar[buf], sf_ph[buf], abort_flag, P.err, kWaitLimitNs, kDevErrTimeout)) {
-          ok = false;
-          break;
-        }
-        sf_ph[buf] ^= 1u;
-        tc_fence_after();
+      for (int i = 0; i < kAcc; ++i) acc[i] = 0.f;
+      // per chunk: the window's slice bounds and this half's block metadata,
+      // prefetched four chunks ahead into four register slots.  The loop is
+      // unrolled by four so a slot is read (its load long complete) and only
+      // then reloaded; no register copy ever waits on a load in flight.
+      const int wlo = (kFW / kWin16) * w, whi = min(wlo + kFW / kWin16, P.nw16);
+      int bnd0, bnd1, bnd2, bnd3, wo0, wo1, wo2, wo3;
+      uint32_t km0, km1, km2, km3;
+      load_chunk_meta(P, 0, wlo, whi, wblk0, lane, bnd0, wo0, km0);
+      load_chunk_meta(P, 1, wlo, whi, wblk0, lane, bnd1, wo1, km1);
+      load_chunk_meta(P, 2, wlo, whi, wblk0, lane, bnd2, wo2, km2);
+      load_chunk_meta(P, 3, wlo, whi, wblk0, lane, bnd3, wo3, km3);
+      // Gather addresses of a chunk (its metadata slot), for scratch buffer
+      // `buf`: row r of the warp (window row 40g + r: block k, bit i; kept
+      // mask m, first kept row at scratch column b0) reads scratch column
+      // b0 + popc(m & (2^i - 1)) when kept and a zero column when pruned.
+      // The lanes compute the 40 addresses (rows lane, lane + 32).
+      auto build_table = [&](uint32_t* t, int bnd, int woff, uint32_t km) {
+        const int p0 = __shfl_sync(0xffffffffu, bnd, 30);
         const uint32_t scr = t_scr + (uint32_t)(buf * kNMax);
 #pragma unroll
-        for (int k = 0; k < kBlocksPerHalf; ++k) {
-          const uint32_t mk = __shfl_sync(0xffffffffu, km, k);
-          if (mk == 0u) continue;
-          const int b0 = __shfl_sync(0xffffffffu, woff, k) - p0;   // scratch column of the block's first kept row
-          const int li = lane & (kBlkRows - 1);
-          const uint32_t my_addr = ((mk >> li) & 1u) ? scr + (uint32_t)(b0 + __popc(mk & ((1u << li) - 1u))) : t_zero;
-          uint32_t a[kBlkRows], g[kBlkRows];
-          tmem_ld_x16b(t_acc + kBlkRows * k, a);
-#pragma unroll
-          for (int i = 0; i < kBlkRows; ++i) g[i] = tmem_ld_x1(__shfl_sync(0xffffffffu, my_addr, i));
-          tmem_wait_ld();
-          reg_fence(a);
-          reg_fence(g);
-#pragma unroll
-          for (int i = 0; i < kBlkRows; ++i) a[i] = __float_as_uint(__uint_as_float(a[i]) + __uint_as_float(g[i]));
-          tmem_st_x16(t_acc + kBlkRows * k, a);
+        for (int rr = 0; rr < 2; ++rr) {
+          const int r = lane + 32 * rr;
+          const int k = (r + rsh) >> 4, i = (r + rsh) & 15;
+          const uint32_t mk = __shfl_sync(0xffffffffu, km, k);   // lanes >= 3 hold no block: mask 0
+          const int wo = __shfl_sync(0xffffffffu, woff, k);
+          const uint32_t addr =
+              ((mk >> i) & 1u) ? scr + (uint32_t)(wo - p0 + __popc(mk & ((1u << i) - 1u))) : t_zero;
+          if (r < kAcc) t[r] = addr;
         }
-        tmem_wait_st();
-        tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sempty_bar[buf]);
-        buf ^= 1;
-        c = cn;
-        woff = nwoff;
-        km = nkm;
-      }
-      if (!ok) break;
-      // own accumulator half -> bf16 y rows [r0, r0 + kHalf) of token tok
-      const int tok = m * kBM + 32 * q + lane;
-      uint16_t* yrow = P.y + (int64_t)tok * P.out;
-      const bool vec_ok = (P.out & 7) == 0;
-#pragma unroll 1
-      for (int col = 0; col < kHalf; col += kBlkRows) {
-        uint32_t v[kBlkRows];
-        tmem_ld_x16b(t_acc + col, v);
+      };
+      // One chunk.  Its address table was built by the previous step, so the
+      // path from "scratch full" to "scratch free" holds only the table reads,
+      // the 40 TMEM loads and their wait; the next chunk's table is built
+      // after the buffer is handed back, then the loaded values are added.
+      auto step = [&](int c, int& bnd, int& wo, uint32_t& kmr, int bnd_n, int wo_n, uint32_t km_n) {
+        const int p0 = __shfl_sync(0xffffffffu, bnd, 30), p1 = __shfl_sync(0xffffffffu, bnd, 31);
+        load_chunk_meta(P, c + 4, wlo, whi, wblk0, lane, bnd, wo, kmr);
+        uint32_t* t_cur = tbl + (c & 1) * kAcc;
+        uint32_t* t_next = tbl + ((c + 1) & 1) * kAcc;
+        if (p1 <= p0 || !ok) {
+          build_table(t_next, bnd_n, wo_n, km_n);
+          return;
+        }
+        if (!mbar_wait_bounded(&sfull_bar[buf], (sf_ph >> buf) & 1u, abort_flag, P.err, kWaitLimitNs,
+                               kDevErrTimeout)) {
+          ok = false;
+          return;
+        }
+        sf_ph ^= 1u << buf;
+        tc_fence_after();
+        uint32_t v[kAcc];
+        gather_rows<kAcc>(t_cur, v);
         tmem_wait_ld();
         reg_fence(v);
-        const int rb = r0 + col;
-        if (tok < P.T && rb < P.out) {
-          if (vec_ok && rb + kBlkRows <= P.out) {
-            uint4* dst = reinterpret_cast<uint4*>(yrow + rb);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&sempty_bar[buf]), 0));
+        if (++buf == kScrBufs) buf = 0;
+        build_table(t_next, bnd_n, wo_n, km_n);
+        add_f32x2<kAcc>(acc, v);
+      };
+      build_table(tbl, bnd0, wo0, km0);
+      for (int c = 0; c < P.G && ok; c += 4) {
+        step(c, bnd0, wo0, km0, bnd1, wo1, km1);
+        if (c + 1 < P.G) step(c + 1, bnd1, wo1, km1, bnd2, wo2, km2);
+        if (c + 2 < P.G) step(c + 2, bnd2, wo2, km2, bnd3, wo3, km3);
+        if (c + 3 < P.G) step(c + 3, bnd3, wo3, km3, bnd0, wo0, km0);
+      }
+      if (!ok) break;
+      // accumulators -> bf16 y rows [r0, r0 + 40) of token tok
+      const int tok = m * kPairM + (int)rank * kBM + 32 * q + lane;
+      if (tok < P.T) {
+        uint16_t* yrow = P.y + (int64_t)tok * P.out;
+        const bool vec_ok = (P.out & 7) == 0;
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
-              dst[u] = make_uint4(pack_bf16x2(v[8 * u + 0], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
-                                  pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
+        for (int k = 0; k < kAcc / 8; ++k) {
+          const int rb = r0 + 8 * k;
+          const float* a = acc + 8 * k;
+          if (vec_ok && rb + 8 <= P.out) {
+            *reinterpret_cast<uint4*>(yrow + rb) =
+                make_uint4(pack_bf16x2(a[0], a[1]), pack_bf16x2(a[2], a[3]), pack_bf16x2(a[4], a[5]),
+                           pack_bf16x2(a[6], a[7]));
           } else {
 #pragma unroll
-            for (int i = 0; i < kBlkRows; ++i)
-              if (rb + i < P.out) yrow[rb + i] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[i])));
+            for (int i = 0; i < 8; ++i)
+              if (rb + i < P.out) yrow[rb + i] = __bfloat16_as_ushort(__float2bfloat16_rn(a[i]));
           }
         }
       }
@@ -380,10 +429,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
 
   tc_fence_before();
   __syncthreads();
+  if (abort_s) {
+    // a role gave up: give copies the peer may still have in flight time to land
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 2000000ull) {
+    }
+  }
+  cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
+  cluster_sync_all();
 }
 
 // ------------------------------------------------------------------ host side
@@ -404,9 +461,10 @@ gs_status prefill_prepare_weight_maps(gs_packed* p) {
   p->wmaps_valid = false;
   if (p->kept == 0) return GS_OK;
   static_assert(sizeof(CUtensorMap) == 128, "CUtensorMap size");
-  for (int h = 0; h < 4; ++h) {
+  static_assert(sizeof(p->wmaps) / sizeof(p->wmaps[0]) == kNMaps, "one W descriptor per slice height");
+  for (int h = 0; h < kNMaps; ++h) {
     CUtensorMap m;
-    if (!encode_tmap_2d_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, kBK, (uint32_t)(128 >> h), true))
+    if (!encode_tmap_slabs_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, (uint32_t)(8 * (h + 1)), kSlabs))
       return GS_ERR_CUDA;
     std::memcpy(p->wmaps[h], &m, sizeof(m));
   }
@@ -432,8 +490,8 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
 
   PrefillParams P;
   std::memset(&P, 0, sizeof(P));
-  if (!encode_tmap_2d_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBK, kBM, true)) return GS_ERR_CUDA;
-  for (int h = 0; h < 4; ++h) std::memcpy(&P.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
+  if (!encode_tmap_slabs_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBM, kSlabs)) return GS_ERR_CUDA;
+  for (int h = 0; h < kNMaps; ++h) std::memcpy(&P.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
   P.win_off16 = p->win_off16;
   P.kmask16 = p->kmask16;
   P.y = static_cast<uint16_t*>(y);
@@ -441,12 +499,13 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
   P.G = p->G;
   P.nw16 = p->nw16;
   P.T = (int32_t)T;
-  P.n_m = (int32_t)((T + kBM - 1) / kBM);
+  P.n_m = (int32_t)((T + kPairM - 1) / kPairM);
   P.n_w = (int32_t)((p->out + kFW - 1) / kFW);
   P.err = device_error_flag();
   if (!P.err) return GS_ERR_CUDA;
   const int64_t tiles = (int64_t)P.n_m * P.n_w;
-  const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
+  const int64_t max_pairs = sm_count() / 2;
+  const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs (cluster dims 2)
   k_prefill<<<grid, kThreads, kSmemBytes, s>>>(P);
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;

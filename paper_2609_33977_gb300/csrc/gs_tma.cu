@@ -43,4 +43,19 @@ bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t o
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_tmap_slabs_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows, uint32_t box_rows,
+                            uint32_t box_slabs) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || row_elems % 64 != 0) return false;
+  // (element within slab, row, slab): the slab dimension advances 128 bytes
+  // inside a row, the row dimension a whole row.
+  const cuuint64_t dims[3] = {64, rows, row_elems / 64};
+  const cuuint64_t strides[2] = {row_elems * 2, 128};
+  const cuuint32_t box[3] = {64, box_rows, box_slabs};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(static_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace gs
