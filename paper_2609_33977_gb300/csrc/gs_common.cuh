@@ -34,11 +34,12 @@ struct gs_packed {
   size_t device_bytes;
   // decode kernel: window-major metadata and split-reduction scratch
   int32_t nblk64;     // ceil(out / 64)
-  int32_t dec_cpu;    // chunks per decode work unit
-  int32_t dec_nsplit; // work units per 64-row block = ceil(G / dec_cpu)
+  int32_t dec_cpu;    // chunks per decode work unit (about 256 KB of kept weights)
+  int32_t dec_cpu_fine;   // chunks per unit when the layer is scheduled last (a quarter of that)
+  int32_t dec_nsplit_max; // ceil(G / dec_cpu_fine): splits the workspace is sized for
   int4* dmeta;        // [nblk64][G]: {first packed row of the block's slice, kept masks of its 4 windows, 0}
-  float* dec_ws;      // [nblk64][dec_nsplit][4][16 tokens][16 rows] partial sums (dec_nsplit > 1)
-  int32_t* dec_cnt;   // [nblk64][4] arrival counters (self-resetting)
+  float* dec_ws;      // [nblk64][dec_nsplit_max][4][16 tokens][16 rows] partial sums
+  int32_t* dec_cnt;   // [nblk64][4] arrival counters, then {unit ticket, finished CTAs} (self-resetting)
   // tcgen05 prefill: slab TMA descriptors over the tiles, box heights 16, 32, ..., 160 rows
   alignas(64) unsigned char wmaps[10][128];
   bool wmaps_valid;

@@ -2,9 +2,10 @@
 //   y[t, r] = sum over kept groups (r, c) of sum_k x[t, 256c+k] W[r, 256c+k]   (Eq. 1)
 //
 // Work units.  A unit is (64-row block, range of chunks) of one layer, sized to
-// about 256 KB of kept weights.  Persistent CTAs walk their units in a snake
-// order over a longest-first unit list, so every CTA streams a similar number
-// of bytes and the pipeline never restarts between units.
+// about 256 KB of kept weights (a quarter of that when a launch has too few
+// units to spread over the CTAs).  Persistent CTAs take units from a shared
+// ticket counter in list order (largest layers first), so a CTA that runs
+// ahead takes more units, and the pipeline never restarts between units.
 //
 // Data movement.  Inside a chunk the kept rows of a 64-row block are one
 // contiguous slice of the packed tiles, so a producer warp streams each chunk's
@@ -79,6 +80,7 @@ struct DecParams {
   int32_t n_layers;
   int32_t T;
   int32_t n_units;
+  int32_t* sched;        // {next unit ticket, finished CTAs}: zero between launches
   int* err;
 };
 
@@ -112,11 +114,8 @@ struct Unit {
   int l, blk, c0, nC;
 };
 
-// k-th unit of this CTA (snake order over the unit list); false when done
-__device__ __forceinline__ bool unit_of(const DecParams& P, int k, Unit& U) {
-  const int n = gridDim.x, b = blockIdx.x;
-  const int64_t u = (int64_t)k * n + ((k & 1) ? (n - 1 - b) : b);
-  if (u >= P.n_units) return false;
+// unit u of the launch's unit list
+__device__ __forceinline__ void unit_at(const DecParams& P, int u, Unit& U) {
   int l = 0;
   while (l + 1 < P.n_layers && P.L[l + 1].unit_begin <= u) ++l;
   const DecLayer& L = P.L[l];
@@ -126,7 +125,6 @@ __device__ __forceinline__ bool unit_of(const DecParams& P, int k, Unit& U) {
   const int split = r % L.nsplit;
   U.c0 = split * L.cpu;
   U.nC = min(L.G, U.c0 + L.cpu) - U.c0;
-  return true;
 }
 
 template <int NT>
@@ -137,6 +135,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   __shared__ uint32_t w_off[kRingSeq];   // ring offset of each in-flight chunk
   __shared__ __align__(8) uint64_t m_full[kMetaSlots];
   __shared__ __align__(8) uint64_t m_empty[kMetaSlots];
+  __shared__ int unit_id[kMetaSlots];   // unit staged in each metadata slot (-1: no more units)
   __shared__ int abort_s;
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
   int4* meta = reinterpret_cast<int4*>(ring + kRingBytes);   // [kMetaSlots][kMaxCpu]
@@ -155,6 +154,12 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     fence_mbar_init();
   }
   __syncthreads();
+  // Programmatic dependent launch: the next launch in the stream may become
+  // resident as soon as SM slots free up, and this grid waits here until the
+  // grid before it has completed and its writes are visible (x may be its y;
+  // the ticket counter and split workspace may be shared with it).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   volatile int* abort_flag = &abort_s;
   const int T = P.T;
 
@@ -165,8 +170,16 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     uint64_t head = 0, tail = 0; // virtual byte offsets: allocated / released
     uint64_t end_v[kRingSeq];    // virtual end offset of each in-flight chunk
     bool ok = true;
-    Unit U;
-    bool have = unit_of(P, 0, U);
+    // Units come from the launch's ticket counter.  Lane 0 holds the ticket
+    // after next in `t_ahead`: it is taken two units early, so the atomic's
+    // round trip never delays the copies of the current unit.
+    int t_ahead = 0;
+    if (lane == 0) t_ahead = atomicAdd(P.sched, 1);
+    int u = __shfl_sync(0xffffffffu, t_ahead, 0);
+    if (lane == 0) t_ahead = atomicAdd(P.sched, 1);
+    bool have = u < P.n_units;
+    Unit U{0, 0, 0, 0};
+    if (have) unit_at(P, u, U);
     int4 pre[kMaxCpu / 32];      // this lane's metadata entries of the next unit to stage
     auto prefetch = [&](const Unit& V, bool hv) {
 #pragma unroll
@@ -177,22 +190,36 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       }
     };
     prefetch(U, have);
-    for (int k = 0; have && ok; ++k) {
+    for (int k = 0; ok; ++k) {
       const int ms = k % kMetaSlots;
       if (!mbar_wait_bounded(&m_empty[ms], ((uint32_t)(k / kMetaSlots) & 1u) ^ 1u, abort_flag, P.err,
                              kDecWaitLimitNs, kDevErrTimeout)) {
         ok = false;
         break;
       }
+      if (!have) {
+        // no more units: tell the consumers
+        if (lane == 0) {
+          unit_id[ms] = -1;
+          __threadfence_block();
+          mbar_arrive(&m_full[ms]);
+        }
+        __syncwarp();
+        break;
+      }
       int4* mrow = meta + ms * kMaxCpu;
 #pragma unroll
       for (int j = 0; j < kMaxCpu / 32; ++j)
         if (lane + 32 * j < U.nC) mrow[lane + 32 * j] = pre[j];
+      if (lane == 0) unit_id[ms] = u;
       __threadfence_block();
       __syncwarp();
       if (lane == 0) mbar_arrive(&m_full[ms]);   // release: the staged entries are visible to consumers
-      Unit V;
-      const bool have_v = unit_of(P, k + 1, V);
+      const int u_next = __shfl_sync(0xffffffffu, t_ahead, 0);
+      if (lane == 0 && u_next < P.n_units) t_ahead = atomicAdd(P.sched, 1);
+      const bool have_v = u_next < P.n_units;
+      Unit V{0, 0, 0, 0};
+      if (have_v) unit_at(P, u_next, V);
       prefetch(V, have_v);                       // in flight while this unit's copies are issued
       if (lane == 0) {
         const DecLayer& L = P.L[U.l];
@@ -233,6 +260,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       q = __shfl_sync(0xffffffffu, q, 0);
       U = V;
+      u = u_next;
       have = have_v;
     }
     if (lane == 0 && !ok) {
@@ -250,15 +278,18 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
     uint32_t q = 0;
     bool ok = true;
-    Unit U;
-    for (int k = 0; ok && unit_of(P, k, U); ++k) {
-      const DecLayer& L = P.L[U.l];
+    for (int k = 0; ok; ++k) {
       const int ms = k % kMetaSlots;
       if (!mbar_wait_bounded(&m_full[ms], (uint32_t)(k / kMetaSlots) & 1u, abort_flag, P.err, kDecWaitLimitNs,
                              kDevErrTimeout)) {
         ok = false;
         break;
       }
+      const int u = unit_id[ms];
+      if (u < 0) break;
+      Unit U;
+      unit_at(P, u, U);
+      const DecLayer& L = P.L[U.l];
       const int4* mrow = meta + ms * kMaxCpu;
       float acc[NT][4], acc2[NT][4];   // two chains (even / odd k blocks) halve the MMA dependency depth
 #pragma unroll
@@ -369,6 +400,15 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     }
   }
   __syncthreads();
+  // the last CTA to finish rewinds the ticket counter for the next launch
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(P.sched + 1, 1) == (int)gridDim.x - 1) {
+      P.sched[0] = 0;
+      P.sched[1] = 0;
+      __threadfence();
+    }
+  }
 }
 
 // metadata of 64-row block b, chunk c: first packed row of the block's slice and
@@ -405,8 +445,17 @@ cudaError_t launch_nt(const DecParams& P, int grid, cudaStream_t s) {
     attr_err = cudaFuncSetAttribute(k_decode<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
-  k_decode<NT><<<grid, kThreadsDec, kDecSmemBytes, s>>>(P);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreadsDec);
+  cfg.dynamicSmemBytes = kDecSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_decode<NT>, P);
 }
 
 }  // namespace
@@ -420,18 +469,17 @@ gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
   int cpu = (int)std::floor((double)kUnitBytes / std::max(per_chunk, 1.0) + 0.5);
   cpu = std::max(1, std::min(cpu, std::min(p->G, kMaxCpu)));
   p->dec_cpu = cpu;
-  p->dec_nsplit = (p->G + cpu - 1) / cpu;
+  p->dec_cpu_fine = std::max(1, cpu / 4);
+  p->dec_nsplit_max = (p->G + p->dec_cpu_fine - 1) / p->dec_cpu_fine;
   const size_t nmeta = (size_t)p->nblk64 * (size_t)p->G;
   if (cudaMalloc(&p->dmeta, nmeta * sizeof(int4)) != cudaSuccess) return GS_ERR_OOM;
   p->device_bytes += nmeta * sizeof(int4);
-  if (p->dec_nsplit > 1) {
-    const size_t nws = (size_t)p->nblk64 * p->dec_nsplit * kDW * kPartFloats;
-    const size_t ncnt = (size_t)p->nblk64 * kDW;
-    if (cudaMalloc(&p->dec_ws, nws * sizeof(float)) != cudaSuccess) return GS_ERR_OOM;
-    if (cudaMalloc(&p->dec_cnt, ncnt * sizeof(int32_t)) != cudaSuccess) return GS_ERR_OOM;
-    if (cudaMemsetAsync(p->dec_cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) return GS_ERR_CUDA;
-    p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
-  }
+  const size_t nws = (size_t)p->nblk64 * p->dec_nsplit_max * kDW * kPartFloats;
+  const size_t ncnt = (size_t)p->nblk64 * kDW + 2;   // + {unit ticket, finished CTAs}
+  if (cudaMalloc(&p->dec_ws, nws * sizeof(float)) != cudaSuccess) return GS_ERR_OOM;
+  if (cudaMalloc(&p->dec_cnt, ncnt * sizeof(int32_t)) != cudaSuccess) return GS_ERR_OOM;
+  if (cudaMemsetAsync(p->dec_cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) return GS_ERR_CUDA;
+  p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
   const int64_t n = (int64_t)nmeta;
   k_pack_decode_meta<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p->win_off16, p->kmask16, p->G, p->nw16, p->nblk64,
                                                            p->dmeta);
@@ -452,15 +500,20 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
                         cudaStream_t s) {
   if (n <= 0 || T <= 0) return GS_OK;
   if (n > kMaxBatch || T > kMaxT) return GS_ERR_UNSUPPORTED;
-  // longest units first (bytes per unit), so the snake schedule balances
+  // Unit list: layers in descending kept bytes.  When the list would not give
+  // every CTA a couple of units, all layers use quarter-size units (their
+  // split reductions cost more than a ragged end does otherwise).
   std::vector<int> order(n);
-  std::vector<double> unit_bytes(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return ps[a]->kept > ps[b]->kept; });
+  const int64_t max_grid = 2 * (int64_t)sm_count_dec();
+  int64_t coarse_units = 0;
   for (int i = 0; i < n; ++i) {
-    order[i] = i;
     const gs_packed* p = ps[i];
-    unit_bytes[i] = (double)p->kept / std::max(1, p->nblk64 * p->dec_nsplit);
+    coarse_units += (int64_t)p->nblk64 * ((p->G + p->dec_cpu - 1) / p->dec_cpu);
   }
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return unit_bytes[a] > unit_bytes[b]; });
+  const bool all_fine = coarse_units < 2 * max_grid;
+  std::vector<char> fine(n, all_fine ? 1 : 0);
   DecParams P;
   std::memset(&P, 0, sizeof(P));
   P.n_layers = n;
@@ -483,14 +536,15 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     L.in = (int32_t)p->in;
     L.G = p->G;
     L.nblk = p->nblk64;
-    L.cpu = p->dec_cpu;
-    L.nsplit = p->dec_nsplit;
+    L.cpu = fine[k] ? p->dec_cpu_fine : p->dec_cpu;
+    L.nsplit = (p->G + L.cpu - 1) / L.cpu;
     L.unit_begin = (int32_t)units;
-    units += (int64_t)p->nblk64 * p->dec_nsplit;
+    units += (int64_t)p->nblk64 * L.nsplit;
   }
   if (units > INT32_MAX) return GS_ERR_UNSUPPORTED;
   P.n_units = (int32_t)units;
-  const int grid = (int)std::min<int64_t>(units, 2 * (int64_t)sm_count_dec());
+  P.sched = ps[0]->dec_cnt + (size_t)ps[0]->nblk64 * kDW;
+  const int grid = (int)std::min<int64_t>(units, max_grid);
   const cudaError_t e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);
   note_launch();
   return e == cudaSuccess ? GS_OK : GS_ERR_CUDA;
