@@ -10,9 +10,11 @@
 // Data movement.  Inside a chunk the kept rows of a 64-row block are one
 // contiguous slice of the packed tiles, so a producer warp streams each chunk's
 // slice with a single bulk copy (cp.async.bulk) into a byte-granular
-// shared-memory ring (each chunk takes exactly its slice + x rows, so the ring
-// holds several chunks in flight), and the chunk's x rows with one 2-D TMA
-// load; only kept bytes move.  The
+// shared-memory ring (each chunk takes its x rows + slice, from a 1024-byte
+// aligned start, so the ring holds several chunks in flight), and the chunk's
+// x rows with one 3-D TMA box: four 64-wide slabs with the 128-byte swizzle,
+// which keeps the consumers' x fragment reads free of bank conflicts; only
+// kept bytes move.  The
 // producer also stages each unit's per-chunk metadata (slice start + the
 // 16-bit kept masks of the four 16-row windows).
 //
@@ -54,7 +56,7 @@ constexpr int kMaxBatch = 32;
 constexpr int kMaxT = 16;                     // tokens per launch (two 8-token MMA tiles)
 constexpr int kRingBytes = 104 * 1024;       // byte ring per CTA (two CTAs per SM)
 constexpr int kRingSeq = 16;                  // chunks that may be in flight (barrier ring)
-constexpr int kXRow = kTileBytes;             // x chunk row (512 B), one 2-D TMA box per chunk
+constexpr int kXRow = kTileBytes;             // x chunk row (512 B): one 3-D TMA box of 4 swizzled 64-wide slabs per chunk
 constexpr int kMaxCpu = 64;                   // chunks per unit
 constexpr int kMetaSlots = 2;
 constexpr int kDecSmemBytes = kRingBytes + kMetaSlots * kMaxCpu * 16 + 1024;
@@ -64,7 +66,7 @@ constexpr uint64_t kDecWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDecDrainLimitNs = 200000000ull;
 
 struct DecLayer {
-  CUtensorMap xmap;      // x [T][in], box 256 x T (one chunk of every token per load)
+  CUtensorMap xmap;      // x [T][in] as (64, T, in/64) slabs, box 64 x T x 4, 128-byte swizzle
   const uint16_t* x;     // [T][in]
   const uint16_t* tiles; // [kept][256]
   const int4* dmeta;     // [nblk][G]
@@ -227,9 +229,10 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           const int4 m = mrow[i];
           const uint32_t cnt = __popc((uint32_t)m.y) + __popc((uint32_t)m.z);
           const uint32_t bytes = cnt * (uint32_t)kTileBytes;
-          const uint32_t need = cnt ? ((bytes + (uint32_t)T * kXRow + 127u) & ~127u) : 0u;   // 128-B aligned starts
-          // allocate `need` contiguous bytes; a chunk that would straddle the end starts over at 0
-          uint64_t start = head;
+          const uint32_t need = cnt ? bytes + (uint32_t)T * kXRow : 0u;
+          // allocate `need` contiguous bytes from a 1024-byte boundary (the swizzled x box);
+          // a chunk that would straddle the end starts over at 0
+          uint64_t start = need ? (head + 1023u) & ~(uint64_t)1023u : head;
           if (need && (start % kRingBytes) + need > (uint64_t)kRingBytes) start += kRingBytes - start % kRingBytes;
           // wait for the oldest chunks until the allocation fits and a barrier pair is free
           while (ok && (start + need - tail > (uint64_t)kRingBytes || q - oldest >= (uint32_t)kRingSeq)) {
@@ -252,8 +255,8 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           fence_proxy_async_smem();
           mbar_arrive_expect_tx(&w_full[e], cnt ? bytes + (uint32_t)T * kTileBytes : 0u);
           if (cnt) {
-            bulk_copy_g2s(dst, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
-            tma_load_2d(dst + bytes, &L.xmap, &w_full[e], (U.c0 + i) * kGroupIn, 0);
+            tma_load_3d(dst, &L.xmap, &w_full[e], 0, 0, (U.c0 + i) * (kGroupIn / 64));
+            bulk_copy_g2s(dst + (uint32_t)T * kXRow, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
           }
         }
       }
@@ -312,15 +315,20 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
         if (km != 0u) {
           const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
           const uint8_t* cbase = ring + w_off[slot];
-          const uint4* sl = reinterpret_cast<const uint4*>(cbase);
-          const uint32_t xoff = (uint32_t)(__popc((uint32_t)m.y) + __popc((uint32_t)m.z)) * (uint32_t)kTileBytes;
+          const uint4* sl = reinterpret_cast<const uint4*>(cbase + T * kXRow);
+          // x: slab s = b/2 holds k 64s..64s+63 of every token as 128-byte rows
+          // (row index s*T + tok); 16-byte chunk c of a row sits at c ^ (row & 7)
           uint4 xv[NT][8];
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int tok = nt * 8 + g;
-            const uint4* xr = reinterpret_cast<const uint4*>(cbase + xoff + tok * kXRow) + qd;
 #pragma unroll
-            for (int b = 0; b < 8; ++b) xv[nt][b] = tok < T ? xr[4 * b] : make_uint4(0u, 0u, 0u, 0u);
+            for (int b = 0; b < 8; ++b) {
+              const int row = (b >> 1) * T + tok;
+              const int ch = (4 * (b & 1) + qd) ^ (row & 7);
+              xv[nt][b] = tok < T ? *reinterpret_cast<const uint4*>(cbase + row * 128 + ch * 16)
+                                  : make_uint4(0u, 0u, 0u, 0u);
+            }
           }
           const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + qd;
           const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + qd;
@@ -525,7 +533,7 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     const gs_packed* p = ps[order[k]];
     DecLayer& L = P.L[k];
     L.x = static_cast<const uint16_t*>(xs[order[k]]);
-    if (!encode_tmap_2d_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)kGroupIn, (uint32_t)T, false))
+    if (!encode_tmap_slabs_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)T, (uint32_t)(kGroupIn / 64)))
       return GS_ERR_CUDA;
     L.tiles = p->tiles;
     L.dmeta = p->dmeta;
