@@ -162,21 +162,53 @@ def test_block_workload_decode_batched(gs):
     assert gs.device_status() == gs.GS_OK
 
 
-@pytest.mark.parametrize("cfg,T", [(3, 2048), (4, 512), (5, 1024)])
-def test_stack_shapes_prefill_sampled(gs, cfg, T):
-    """First block of the 7B (with activation outliers), 13B and Qwen stacks at
-    prefill token counts; every layer checked on a deterministic token sample."""
-    w = wl.workload(cfg, 0.5)
-    k = wl.keep_counts(w)
-    for i in range(7):
+def stack_blocks(w, k):
+    """Blocks checked for a stack: the first, the last, and the blocks holding
+    the sparsest and the densest layer of the layer-adaptive allocation."""
+    groups = np.array([L.out * (L.inp // 256) for L in w.layers], dtype=np.float64)
+    dens = np.asarray(k, dtype=np.float64) / groups
+    nblk = len(w.layers) // 7
+    return sorted({0, nblk - 1, int(np.argmin(dens)) // 7, int(np.argmax(dens)) // 7})
+
+
+_stack_cache = {}
+
+
+def stack_layer(gs, w, k, i):
+    key = (w.cfg_id, w.density, i)
+    if key not in _stack_cache:
+        _stack_cache.clear()                  # one layer resident at a time (the stacks are GBs)
         Wb = wl.weight_bits(w, i)
         B = wl.group_mask(w, i, int(k[i]))
-        xb = wl.activation_bits(w, i, T)
-        p = packed(gs, Wb, B)
-        y = to_bits(gs.linear(to_dev(xb), p))
-        assert_within_bound(y, xb, Wb, B, tokens=sample_tokens(T, seed=i),
-                            what=f"cfg{cfg} {w.layers[i].name} T={T}")
-        del p
+        _stack_cache[key] = (Wb, B, packed(gs, Wb, B))
+    return _stack_cache[key]
+
+
+# (config, density, token counts): the full-size stacks of the 7B model with
+# activation outliers at prefill, the 13B model over its token sweep, and the
+# Qwen model over its density sweep at T = 1 and 1024.
+STACK_CASES = [(3, 0.5, (2048,)), (4, 0.5, (1, 16, 128, 512, 2048)), (5, 0.3, (1, 1024)), (5, 0.5, (1, 1024)),
+               (5, 0.7, (1, 1024))]
+
+
+@pytest.mark.parametrize("cfg,d,Ts", STACK_CASES)
+def test_stack_shapes_sampled(gs, cfg, d, Ts):
+    """Every layer of the checked blocks of a full-size stack (first, last, and the
+    blocks with the sparsest and densest layer), each at the config's token
+    counts, checked on a deterministic token sample (all tokens when T <= 16)."""
+    w = wl.workload(cfg, d)
+    k = wl.keep_counts(w)
+    assert int(k.sum()) == w.budget
+    for b in stack_blocks(w, k):
+        for i in range(7 * b, 7 * b + 7):
+            Wb, B, p = stack_layer(gs, w, k, i)
+            assert p.kept == int(k[i])
+            for T in Ts:
+                xb = wl.activation_bits(w, i, T)
+                y = to_bits(gs.linear(to_dev(xb), p))
+                assert_within_bound(y, xb, Wb, B, tokens=None if T <= 16 else sample_tokens(T, seed=i),
+                                    what=f"cfg{cfg} d={d} {w.layers[i].name} T={T}")
+    _stack_cache.clear()
     assert gs.device_status() == gs.GS_OK
 
 
