@@ -437,8 +437,10 @@ def run_ours(args):
 
     # ---- tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
     prefill = None
+    prefill_sweep = None
     if not args.no_prefill:
         prefill = measure_prefill(gs, torch, dev, stream, peaks)
+        prefill_sweep = measure_prefill_sweep(gs, torch, dev, stream, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -469,12 +471,30 @@ def run_ours(args):
         "dense_torch_bf16": dense,
         "pack": {"seconds": pack_s, "layers": 7, "GB/s_incl_alloc_and_sync": pack_bytes / pack_s / 1e9},
         "prefill": prefill,
+        "prefill_sweep": prefill_sweep,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def _time_block(gs, torch, stream, xd, ps, ys, algo, n=10):
+    """Seconds per pass over one block's 7 projections (CUDA events, after warm-up)."""
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            for i in range(len(ps)):
+                gs.linear_into(xd[i], ps[i], ys[i], algo=algo, stream=stream)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n):
+            for i in range(len(ps)):
+                gs.linear_into(xd[i], ps[i], ys[i], algo=algo, stream=stream)
+        b.record(stream)
+        b.synchronize()
+    return a.elapsed_time(b) / 1e3 / n
 
 
 def measure_prefill(gs, torch, dev, stream, peaks):
@@ -489,23 +509,14 @@ def measure_prefill(gs, torch, dev, stream, peaks):
     ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
     kept = sum(p.kept for p in ps)
     flops = 2.0 * T * 256 * kept
+    s_block = _time_block(gs, torch, stream, xd, ps, ys, gs.ALGO_PREFILL)
+    n = 10
     with torch.cuda.stream(stream):
-        for _ in range(3):
-            for i in range(7):
-                gs.linear_into(xd[i], ps[i], ys[i], algo=gs.ALGO_PREFILL, stream=stream)
-        n = 10
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(n):
-            for i in range(7):
-                gs.linear_into(xd[i], ps[i], ys[i], algo=gs.ALGO_PREFILL, stream=stream)
-        b.record(stream)
-        b.synchronize()
-        s_block = a.elapsed_time(b) / 1e3 / n
         # dense bf16 reference point on the unpruned weights
         for i in range(7):
             torch.matmul(xd[i], Wd[i].t())
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(n):
             for i in range(7):
@@ -526,6 +537,39 @@ def measure_prefill(gs, torch, dev, stream, peaks):
     del Wd, Bd, xd, ps, ys
     torch.cuda.empty_cache()
     return out
+
+
+def measure_prefill_sweep(gs, torch, dev, stream, peaks):
+    """Prefill kernel over the token counts of the 13B and Qwen stacks (first block
+    of each).  The attainable rate at a token count is min(tensor peak, kept FLOPs
+    over the time to stream the block's bytes at the measured HBM bandwidth)."""
+    tpk = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
+    bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"])) * 1e9
+    rows = []
+    for cfg, d, Ts, name in ((4, 0.5, (128, 512, 2048), "llama2-13b block 0"),
+                             (5, 0.5, (1024,), "qwen2.5-7b block 0, d=0.5")):
+        w = wl.workload(cfg, d, blocks=1)
+        k = wl.keep_counts(w)
+        Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
+        ps = [gs.pack(Wd[i], torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev)) for i in range(7)]
+        del Wd
+        kept = sum(p.kept for p in ps)
+        for T in Ts:
+            xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
+            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
+            s_block = _time_block(gs, torch, stream, xd, ps, ys, gs.ALGO_PREFILL)
+            flops = 2.0 * T * 256 * kept
+            nbytes = 512.0 * kept + sum(2.0 * T * (L.inp + L.out) for L in w.layers)
+            attainable = min(tpk, flops / (nbytes / bw) / 1e12)
+            tflops = flops / s_block / 1e12
+            rows.append({"workload": f"{name}, T={T}", "T": T, "kept_groups": kept, "ms_per_block": s_block * 1e3,
+                         "tokens/s": T / s_block, "TFLOP/s": tflops, "attainable_TFLOP/s": attainable,
+                         "frac_of_attainable": tflops / attainable, "frac_of_tensor_peak": tflops / tpk})
+            del xd, ys
+        del ps
+        torch.cuda.empty_cache()
+    assert gs.device_status() == gs.GS_OK
+    return rows
 
 
 def run_layer(args):
