@@ -29,11 +29,14 @@
 // arrival counter; the last arriver adds the partials in split order (so the
 // result does not depend on arrival order), writes y and resets the counter.
 //
-// K permutation.  Within a 32-wide k block b, lane (g, q) holds the eight
-// consecutive weights k = 32b + 8q + 0..7 of rows g and g+8 and the same eight
-// x values of token g.  Elements 0..3 feed MMA 2b, elements 4..7 feed MMA
-// 2b+1; the logical-to-physical k map depends only on (b, q), so A and B agree
-// and every physical k is used exactly once.
+// K permutation.  At step b (0..7) lane (g, q) holds the eight consecutive
+// weights of 16-byte chunk j = 8(b>>1) + 2q + (b&1) of rows g and g+8 (k = 8j
+// + 0..7) and the same eight x values of token g.  Elements 0..3 feed MMA 2b,
+// elements 4..7 feed MMA 2b+1; the logical-to-physical k map depends only on
+// (b, q), so A and B agree and every physical k is used exactly once.  The
+// four q lanes of a token read every other chunk of a 128-byte slab row, so
+// after the swizzle (chunk ^ row&7) tokens 2p and 2p+1, which share a
+// quarter-warp load phase, land on disjoint banks.
 #include "gs_common.cuh"
 #include "gs_sm100.cuh"
 
@@ -325,17 +328,18 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 #pragma unroll
             for (int b = 0; b < 8; ++b) {
               const int row = (b >> 1) * T + tok;
-              const int ch = (4 * (b & 1) + qd) ^ (row & 7);
+              const int ch = (2 * qd + (b & 1)) ^ (row & 7);
               xv[nt][b] = tok < T ? *reinterpret_cast<const uint4*>(cbase + row * 128 + ch * 16)
                                   : make_uint4(0u, 0u, 0u, 0u);
             }
           }
-          const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + qd;
-          const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + qd;
+          const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + 2 * qd;
+          const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + 2 * qd;
 #pragma unroll
           for (int b = 0; b < 8; ++b) {
-            const uint4 a = kg ? tg[4 * b] : make_uint4(0u, 0u, 0u, 0u);
-            const uint4 a8 = kg8 ? tg8[4 * b] : make_uint4(0u, 0u, 0u, 0u);
+            const int j = 8 * (b >> 1) + (b & 1);
+            const uint4 a = kg ? tg[j] : make_uint4(0u, 0u, 0u, 0u);
+            const uint4 a8 = kg8 ? tg8[j] : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               mma16816(acc[nt], a.x, a8.x, a.y, a8.y, xv[nt][b].x, xv[nt][b].y);
