@@ -3,9 +3,10 @@
 //
 // Work units.  A unit is (64-row block, range of chunks) of one layer, sized to
 // about 256 KB of kept weights (a quarter of that when a launch has too few
-// units to spread over the CTAs).  Persistent CTAs take units from a shared
-// ticket counter in list order (largest layers first), so a CTA that runs
-// ahead takes more units, and the pipeline never restarts between units.
+// units to spread over the CTAs).  Persistent CTA b starts on units b and
+// b + grid, then takes units from a shared ticket counter in list order
+// (largest layers first), so a CTA that runs ahead takes more units, and the
+// pipeline never restarts between units.
 //
 // Data movement.  Inside a chunk the kept rows of a 64-row block are one
 // contiguous slice of the packed tiles, so a producer warp streams each chunk's
@@ -65,6 +66,13 @@ constexpr int kMetaSlots = 2;
 constexpr int kDecSmemBytes = kRingBytes + kMetaSlots * kMaxCpu * 16 + 1024;
 constexpr int kPartFloats = kMaxT * kWin16;   // one warp's partial: 16 tokens x 16 rows
 constexpr int64_t kUnitBytes = 256 * 1024;    // target kept bytes per unit
+// Ring allocation never waits forever: a chunk that does not fit before the
+// ring's end starts over at offset 0, which with every earlier chunk released
+// asks for (ring end - head) + need bytes; that stays within the ring for any
+// head only while two largest chunks (all 64 rows kept, kMaxT x rows) plus the
+// 1024-byte alignment fit in it.
+static_assert(2 * (kRows * kTileBytes + kMaxT * kXRow) + 1023 <= kRingBytes,
+              "decode ring must hold two largest chunks plus alignment");
 constexpr uint64_t kDecWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDecDrainLimitNs = 200000000ull;
 
@@ -119,17 +127,18 @@ struct Unit {
   int l, blk, c0, nC;
 };
 
-// unit u of the launch's unit list
-__device__ __forceinline__ void unit_at(const DecParams& P, int u, Unit& U) {
+// unit u of the launch's unit list; lay[l] = {first unit, splits per block,
+// chunks per unit, chunks} of layer l, staged in shared memory
+__device__ __forceinline__ void unit_at(const int4* lay, int n_layers, int u, Unit& U) {
   int l = 0;
-  while (l + 1 < P.n_layers && P.L[l + 1].unit_begin <= u) ++l;
-  const DecLayer& L = P.L[l];
-  const int r = (int)(u - L.unit_begin);
+  while (l + 1 < n_layers && lay[l + 1].x <= u) ++l;
+  const int4 L = lay[l];
+  const int r = u - L.x;
   U.l = l;
-  U.blk = r / L.nsplit;
-  const int split = r % L.nsplit;
-  U.c0 = split * L.cpu;
-  U.nC = min(L.G, U.c0 + L.cpu) - U.c0;
+  U.blk = r / L.y;
+  const int split = r - U.blk * L.y;
+  U.c0 = split * L.z;
+  U.nC = min(L.w, U.c0 + L.z) - U.c0;
 }
 
 template <int NT>
@@ -138,10 +147,13 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   __shared__ __align__(8) uint64_t w_full[kRingSeq];
   __shared__ __align__(8) uint64_t w_empty[kRingSeq];
   __shared__ uint32_t w_off[kRingSeq];   // ring offset of each in-flight chunk
+  __shared__ uint32_t w_end[kRingSeq];   // its virtual end offset (producer bookkeeping)
   __shared__ __align__(8) uint64_t m_full[kMetaSlots];
   __shared__ __align__(8) uint64_t m_empty[kMetaSlots];
   __shared__ int unit_id[kMetaSlots];   // unit staged in each metadata slot (-1: no more units)
   __shared__ int abort_s;
+  __shared__ int4 lay[kMaxBatch];               // per layer: {first unit, splits per block, chunks per unit, chunks}
+  __shared__ const int4* lay_dmeta[kMaxBatch];  // per layer: chunk metadata
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
   int4* meta = reinterpret_cast<int4*>(ring + kRingBytes);   // [kMetaSlots][kMaxCpu]
 
@@ -158,13 +170,20 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     abort_s = 0;
     fence_mbar_init();
   }
+  if (threadIdx.x < P.n_layers) {
+    const DecLayer& L = P.L[threadIdx.x];
+    lay[threadIdx.x] = make_int4(L.unit_begin, L.nsplit, L.cpu, L.G);
+    lay_dmeta[threadIdx.x] = L.dmeta;
+  }
   __syncthreads();
   // Programmatic dependent launch: the next launch in the stream may become
-  // resident as soon as SM slots free up, and this grid waits here until the
-  // grid before it has completed and its writes are visible (x may be its y;
-  // the ticket counter and split workspace may be shared with it).
+  // resident as soon as SM slots free up.  Before touching anything the grid
+  // before it may write (x may be its y; the ticket counter and split
+  // workspace may be shared with it) a thread waits for that grid to complete
+  // (griddepcontrol.wait).  The packed tiles and chunk metadata are never
+  // written by a decode launch, so the producer streams its first unit's
+  // weight slices before it waits, overlapping the previous launch's end.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   volatile int* abort_flag = &abort_s;
   const int T = P.T;
 
@@ -172,25 +191,31 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     // ------------------------------------------------------------ producer warp
     uint32_t q = 0;              // chunks issued so far (ring sequence number)
     uint32_t oldest = 0;         // oldest chunk not yet known to be released
-    uint64_t head = 0, tail = 0; // virtual byte offsets: allocated / released
-    uint64_t end_v[kRingSeq];    // virtual end offset of each in-flight chunk
+    // Ring bookkeeping in 32-bit virtual byte offsets: `head` / `tail` =
+    // allocated / released, `hoff` = head's offset inside the ring.  Only
+    // differences below the ring size are ever taken, so the counters may wrap.
+    uint32_t head = 0, tail = 0, hoff = 0;
     bool ok = true;
-    // Units come from the launch's ticket counter.  Lane 0 holds the ticket
-    // after next in `t_ahead`: it is taken two units early, so the atomic's
-    // round trip never delays the copies of the current unit.
-    int t_ahead = 0;
-    if (lane == 0) t_ahead = atomicAdd(P.sched, 1);
-    int u = __shfl_sync(0xffffffffu, t_ahead, 0);
-    if (lane == 0) t_ahead = atomicAdd(P.sched, 1);
+    // CTA b starts with units b and b + grid; every later unit comes from the
+    // launch's ticket counter (ticket t = unit 2 grid + t).  `t_ahead` holds
+    // the unit after next: its ticket is taken two units early, so neither the
+    // start of the launch nor the atomic's round trip delays any copies.
+    const int n_static = 2 * (int)gridDim.x;
+    int u = (int)blockIdx.x;
+    int t_ahead = (int)(blockIdx.x + gridDim.x);
     bool have = u < P.n_units;
     Unit U{0, 0, 0, 0};
-    if (have) unit_at(P, u, U);
+    if (have) unit_at(lay, P.n_layers, u, U);
+    // Chunks of the first unit issued before the dependency wait: their x
+    // boxes follow once it returns (lane 0; `dep` = wait done).
+    bool dep = false;
+    uint32_t n_pend = 0;
     int4 pre[kMaxCpu / 32];      // this lane's metadata entries of the next unit to stage
     auto prefetch = [&](const Unit& V, bool hv) {
 #pragma unroll
       for (int j = 0; j < kMaxCpu / 32; ++j) {
         const int i = lane + 32 * j;
-        pre[j] = (hv && i < V.nC) ? __ldg(P.L[V.l].dmeta + (int64_t)V.blk * P.L[V.l].G + V.c0 + i)
+        pre[j] = (hv && i < V.nC) ? __ldg(lay_dmeta[V.l] + (int64_t)V.blk * lay[V.l].w + V.c0 + i)
                                   : make_int4(0, 0, 0, 0);
       }
     };
@@ -221,47 +246,74 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       __syncwarp();
       if (lane == 0) mbar_arrive(&m_full[ms]);   // release: the staged entries are visible to consumers
       const int u_next = __shfl_sync(0xffffffffu, t_ahead, 0);
-      if (lane == 0 && u_next < P.n_units) t_ahead = atomicAdd(P.sched, 1);
+      if (lane == 0 && dep && u_next < P.n_units) t_ahead = n_static + atomicAdd(P.sched, 1);
       const bool have_v = u_next < P.n_units;
       Unit V{0, 0, 0, 0};
-      if (have_v) unit_at(P, u_next, V);
+      if (have_v) unit_at(lay, P.n_layers, u_next, V);
       prefetch(V, have_v);                       // in flight while this unit's copies are issued
       if (lane == 0) {
         const DecLayer& L = P.L[U.l];
+        const uint32_t xbytes = (uint32_t)T * kXRow;
+        // first unit only: wait for the previous grid, then issue the pending
+        // x boxes and take the ticket of the unit after next
+        auto resolve = [&]() {
+          asm volatile("griddepcontrol.wait;" ::: "memory");
+          for (uint32_t i = 0; i < n_pend; ++i) {
+            const int4 mp = mrow[i];
+            if ((mp.y | mp.z) != 0)
+              tma_load_3d(ring + w_off[i], &L.xmap, &w_full[i], 0, 0, (U.c0 + (int)i) * (kGroupIn / 64));
+          }
+          if (u_next < P.n_units) t_ahead = n_static + atomicAdd(P.sched, 1);
+          dep = true;
+        };
+        int4 m_next = U.nC > 0 ? mrow[0] : make_int4(0, 0, 0, 0);
         for (int i = 0; i < U.nC && ok; ++i, ++q) {
-          const int4 m = mrow[i];
+          const int4 m = m_next;
+          if (i + 1 < U.nC) m_next = mrow[i + 1];
           const uint32_t cnt = __popc((uint32_t)m.y) + __popc((uint32_t)m.z);
           const uint32_t bytes = cnt * (uint32_t)kTileBytes;
-          const uint32_t need = cnt ? bytes + (uint32_t)T * kXRow : 0u;
+          const uint32_t need = cnt ? bytes + xbytes : 0u;
           // allocate `need` contiguous bytes from a 1024-byte boundary (the swizzled x box);
-          // a chunk that would straddle the end starts over at 0
-          uint64_t start = need ? (head + 1023u) & ~(uint64_t)1023u : head;
-          if (need && (start % kRingBytes) + need > (uint64_t)kRingBytes) start += kRingBytes - start % kRingBytes;
+          // a chunk that would straddle the end starts over at offset 0
+          uint32_t off = hoff, pad = 0u;
+          if (need) {
+            off = (hoff + 1023u) & ~1023u;
+            pad = off - hoff;
+            if (off + need > (uint32_t)kRingBytes) {
+              pad = (uint32_t)kRingBytes - hoff;
+              off = 0u;
+            }
+          }
+          const uint32_t start = head + pad;
+          const bool full = start + need - tail > (uint32_t)kRingBytes || q - oldest >= (uint32_t)kRingSeq;
+          if (full && !dep) resolve();   // releases need the pending x boxes
           // wait for the oldest chunks until the allocation fits and a barrier pair is free
-          while (ok && (start + need - tail > (uint64_t)kRingBytes || q - oldest >= (uint32_t)kRingSeq)) {
+          while (ok && (start + need - tail > (uint32_t)kRingBytes || q - oldest >= (uint32_t)kRingSeq)) {
             const uint32_t j = oldest % kRingSeq;
             if (!mbar_wait_bounded(&w_empty[j], (oldest / kRingSeq) & 1u, abort_flag, P.err, kDecWaitLimitNs,
                                    kDevErrTimeout)) {
               ok = false;
               break;
             }
-            tail = end_v[j];
+            tail = w_end[j];
             ++oldest;
           }
           if (!ok) break;
           const uint32_t e = q % kRingSeq;
-          const uint32_t off = (uint32_t)(start % kRingBytes);
           w_off[e] = off;
-          end_v[e] = start + need;
+          w_end[e] = start + need;
           head = start + need;
+          hoff = off + need;
           uint8_t* dst = ring + off;
           fence_proxy_async_smem();
-          mbar_arrive_expect_tx(&w_full[e], cnt ? bytes + (uint32_t)T * kTileBytes : 0u);
+          mbar_arrive_expect_tx(&w_full[e], cnt ? bytes + xbytes : 0u);
           if (cnt) {
-            tma_load_3d(dst, &L.xmap, &w_full[e], 0, 0, (U.c0 + i) * (kGroupIn / 64));
-            bulk_copy_g2s(dst + (uint32_t)T * kXRow, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
+            if (dep) tma_load_3d(dst, &L.xmap, &w_full[e], 0, 0, (U.c0 + i) * (kGroupIn / 64));
+            bulk_copy_g2s(dst + xbytes, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
           }
+          if (!dep) ++n_pend;
         }
+        if (!dep) resolve();
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       q = __shfl_sync(0xffffffffu, q, 0);
@@ -280,6 +332,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     __syncwarp();
   } else {
     // ------------------------------------------------------------ consumer warps
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int g = lane >> 2, qd = lane & 3;
     const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
     uint32_t q = 0;
@@ -294,7 +347,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       const int u = unit_id[ms];
       if (u < 0) break;
       Unit U;
-      unit_at(P, u, U);
+      unit_at(lay, P.n_layers, u, U);
       const DecLayer& L = P.L[U.l];
       const int4* mrow = meta + ms * kMaxCpu;
       float acc[NT][4], acc2[NT][4];   // two chains (even / odd k blocks) halve the MMA dependency depth
