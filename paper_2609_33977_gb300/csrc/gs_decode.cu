@@ -19,16 +19,21 @@
 // producer also stages each unit's per-chunk metadata (slice start + the
 // 16-bit kept masks of the four 16-row windows).
 //
-// Compute.  Consumer warp w owns rows 16w..16w+15 of the block.  It builds
+// Compute.  Two consumer warps own each 16-row window w of the block (rows
+// 16w..16w+15): one takes the unit's even chunks, the other its odd chunks,
+// so two chunks per window are in flight in the MMA pipeline.  A warp builds
 // mma.sync A fragments from the slice, placing every kept row at its window
 // position (pruned rows stay zero), with the x chunk as the B fragment.  The
 // MMA row is the output row, so the fp32 accumulator stays in registers for
-// the whole unit: no scatter and no atomics on y.
+// the whole unit: no scatter and no atomics on y.  At the unit's end the
+// odd-chunk warp hands its accumulator to the even-chunk warp through shared
+// memory, which adds it (a fixed order) and writes the result.
 //
-// Reduction.  When a block's chunks are split over several units, each warp
-// writes its 16-row partial to the handle's workspace and bumps the window's
-// arrival counter; the last arriver adds the partials in split order (so the
-// result does not depend on arrival order), writes y and resets the counter.
+// Reduction.  When a block's chunks are split over several units, the
+// even-chunk warp of each window writes its 16-row partial to the handle's
+// workspace and bumps the window's arrival counter; the last arriver adds the
+// partials in split order (so the result does not depend on arrival order),
+// writes y and resets the counter.
 //
 // K permutation.  At step b (0..7) lane (g, q) holds the eight consecutive
 // weights of 16-byte chunk j = 8(b>>1) + 2q + (b&1) of rows g and g+8 (k = 8j
@@ -53,9 +58,11 @@ namespace gs {
 namespace {
 using namespace sm100;
 
-constexpr int kDW = 4;                        // consumer warps = 16-row windows per block
+constexpr int kDW = 4;                        // 16-row windows per block
+constexpr int kCW = 2 * kDW;                  // consumer warps: two per window (even / odd chunks)
 constexpr int kRows = kDW * kWin16;           // 64 rows per block
-constexpr int kThreadsDec = (kDW + 1) * 32;   // + one producer warp
+constexpr int kThreadsDec = (kCW + 1) * 32;   // + one producer warp
+constexpr int kMaxNT = 2;                     // 8-token MMA tiles per launch
 constexpr int kMaxBatch = 32;
 constexpr int kMaxT = 16;                     // tokens per launch (two 8-token MMA tiles)
 constexpr int kRingBytes = 104 * 1024;       // byte ring per CTA (two CTAs per SM)
@@ -152,6 +159,9 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   __shared__ __align__(8) uint64_t m_empty[kMetaSlots];
   __shared__ int unit_id[kMetaSlots];   // unit staged in each metadata slot (-1: no more units)
   __shared__ int abort_s;
+  __shared__ __align__(8) uint64_t p_full[kDW];    // pair hand-off per window: accumulator written
+  __shared__ __align__(8) uint64_t p_empty[kDW];   // ... and consumed
+  __shared__ __align__(16) float pair_buf[kDW * 32 * 4 * kMaxNT];
   __shared__ int4 lay[kMaxBatch];               // per layer: {first unit, splits per block, chunks per unit, chunks}
   __shared__ const int4* lay_dmeta[kMaxBatch];  // per layer: chunk metadata
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
@@ -165,7 +175,11 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     }
     for (int k = 0; k < kMetaSlots; ++k) {
       mbar_init(&m_full[k], 1);
-      mbar_init(&m_empty[k], kDW);
+      mbar_init(&m_empty[k], kCW);
+    }
+    for (int k = 0; k < kDW; ++k) {
+      mbar_init(&p_full[k], 1);
+      mbar_init(&p_empty[k], 1);
     }
     abort_s = 0;
     fence_mbar_init();
@@ -187,7 +201,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   volatile int* abort_flag = &abort_s;
   const int T = P.T;
 
-  if (warp == kDW) {
+  if (warp == kCW) {
     // ------------------------------------------------------------ producer warp
     uint32_t q = 0;              // chunks issued so far (ring sequence number)
     uint32_t oldest = 0;         // oldest chunk not yet known to be released
@@ -333,8 +347,15 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   } else {
     // ------------------------------------------------------------ consumer warps
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    // Warp pair (win, win + kDW) owns the 16-row window win: the first warp
+    // takes a unit's even chunks, the second its odd chunks, so two chunks are
+    // in the MMA pipeline per window.  At the unit's end the second warp hands
+    // its accumulator to the first through shared memory, which adds it (a
+    // fixed order) and writes the result.
+    const int win = warp & (kDW - 1), par = warp / kDW;
     const int g = lane >> 2, qd = lane & 3;
     const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
+    float* pbuf = pair_buf + win * (32 * 4 * kMaxNT) + lane * (4 * kMaxNT);
     uint32_t q = 0;
     bool ok = true;
     for (int k = 0; ok; ++k) {
@@ -355,15 +376,16 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[nt][i] = acc2[nt][i] = 0.f;
-      for (int i = 0; i < U.nC; ++i, ++q) {
+      for (int i = par; i < U.nC; i += 2) {
+        const uint32_t qi = q + (uint32_t)i;   // ring sequence number of chunk i
         const int4 m = mrow[i];
-        const uint32_t km = meta_mask(m, warp);
+        const uint32_t km = meta_mask(m, win);
         int base = 0;
 #pragma unroll
         for (int w = 0; w < kDW; ++w)
-          if (w < warp) base += __popc(meta_mask(m, w));
-        const int slot = (int)(q % kRingSeq);
-        if (!mbar_wait_bounded(&w_full[slot], (q / kRingSeq) & 1u, abort_flag, P.err, kDecWaitLimitNs,
+          if (w < win) base += __popc(meta_mask(m, w));
+        const int slot = (int)(qi % kRingSeq);
+        if (!mbar_wait_bounded(&w_full[slot], (qi / kRingSeq) & 1u, abort_flag, P.err, kDecWaitLimitNs,
                                kDevErrTimeout)) {
           ok = false;
           break;
@@ -372,20 +394,6 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
           const uint8_t* cbase = ring + w_off[slot];
           const uint4* sl = reinterpret_cast<const uint4*>(cbase + T * kXRow);
-          // x: slab s = b/2 holds k 64s..64s+63 of every token as 128-byte rows
-          // (row index s*T + tok); 16-byte chunk c of a row sits at c ^ (row & 7)
-          uint4 xv[NT][8];
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            const int tok = nt * 8 + g;
-#pragma unroll
-            for (int b = 0; b < 8; ++b) {
-              const int row = (b >> 1) * T + tok;
-              const int ch = (2 * qd + (b & 1)) ^ (row & 7);
-              xv[nt][b] = tok < T ? *reinterpret_cast<const uint4*>(cbase + row * 128 + ch * 16)
-                                  : make_uint4(0u, 0u, 0u, 0u);
-            }
-          }
           const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + 2 * qd;
           const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + 2 * qd;
 #pragma unroll
@@ -395,14 +403,22 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
             const uint4 a8 = kg8 ? tg8[j] : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              mma16816(acc[nt], a.x, a8.x, a.y, a8.y, xv[nt][b].x, xv[nt][b].y);
-              mma16816(acc2[nt], a.z, a8.z, a.w, a8.w, xv[nt][b].z, xv[nt][b].w);
+              // x: slab s = b/2 holds k 64s..64s+63 of every token as 128-byte
+              // rows (row index s*T + tok); 16-byte chunk c of a row sits at c ^ (row & 7)
+              const int tok = nt * 8 + g;
+              const int row = (b >> 1) * T + tok;
+              const int ch = (2 * qd + (b & 1)) ^ (row & 7);
+              const uint4 xv = tok < T ? *reinterpret_cast<const uint4*>(cbase + row * 128 + ch * 16)
+                                       : make_uint4(0u, 0u, 0u, 0u);
+              mma16816(acc[nt], a.x, a8.x, a.y, a8.y, xv.x, xv.y);
+              mma16816(acc2[nt], a.z, a8.z, a.w, a8.w, xv.z, xv.w);
             }
           }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&w_empty[slot]);
       }
+      q += (uint32_t)U.nC;
       if (!ok) break;
       __syncwarp();
       if (lane == 0) mbar_arrive(&m_empty[ms]);
@@ -411,8 +427,37 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[nt][i] += acc2[nt][i];
 
-      // ---- unit result: this warp's 16 rows x T tokens
-      const int r0 = U.blk * kRows + warp * kWin16;
+      // ---- pair hand-off: the odd-chunk warp's accumulator joins the even one's
+      const uint32_t hpar = (uint32_t)k & 1u;
+      if (par) {
+        if (!mbar_wait_bounded(&p_empty[win], hpar ^ 1u, abort_flag, P.err, kDecWaitLimitNs, kDevErrTimeout)) {
+          ok = false;
+          break;
+        }
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+          *reinterpret_cast<float4*>(pbuf + 4 * nt) = make_float4(acc[nt][0], acc[nt][1], acc[nt][2], acc[nt][3]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[win]);
+        continue;
+      }
+      if (!mbar_wait_bounded(&p_full[win], hpar, abort_flag, P.err, kDecWaitLimitNs, kDevErrTimeout)) {
+        ok = false;
+        break;
+      }
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const float4 o = *reinterpret_cast<const float4*>(pbuf + 4 * nt);
+        acc[nt][0] += o.x;
+        acc[nt][1] += o.y;
+        acc[nt][2] += o.z;
+        acc[nt][3] += o.w;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_empty[win]);
+
+      // ---- unit result: this window's 16 rows x T tokens
+      const int r0 = U.blk * kRows + win * kWin16;
       if (L.nsplit == 1) {
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
@@ -426,7 +471,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           }
       } else {
         const int split = U.c0 / L.cpu;
-        float* part = L.ws + (((int64_t)U.blk * L.nsplit + split) * kDW + warp) * kPartFloats;
+        float* part = L.ws + (((int64_t)U.blk * L.nsplit + split) * kDW + win) * kPartFloats;
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -438,12 +483,12 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
         __threadfence();
         __syncwarp();
         int last = 0;
-        int32_t* cnt = L.cnt + U.blk * kDW + warp;
+        int32_t* cnt = L.cnt + U.blk * kDW + win;
         if (lane == 0) last = (atomicAdd(cnt, 1) == L.nsplit - 1);
         last = __shfl_sync(0xffffffffu, last, 0);
         if (last) {
           __threadfence();
-          const float* base_ws = L.ws + ((int64_t)U.blk * L.nsplit * kDW + warp) * kPartFloats;
+          const float* base_ws = L.ws + ((int64_t)U.blk * L.nsplit * kDW + win) * kPartFloats;
           const int Tl = T < NT * 8 ? T : NT * 8;
           for (int e = lane; e < Tl * kWin16; e += 32) {
             // issue every partial's load first, then add them in split order
