@@ -1,9 +1,10 @@
 // Decode-regime group-sparse linear (few tokens, HBM-bound):
 //   y[t, r] = sum over kept groups (r, c) of sum_k x[t, 256c+k] W[r, 256c+k]   (Eq. 1)
 //
-// Work units.  A unit is (64-row block, range of chunks) of one layer, sized to
-// about 256 KB of kept weights (a quarter of that when a launch has too few
-// units to spread over the CTAs).  Persistent CTA b starts on units b and
+// Work units.  A unit is (64-row block, range of chunks) of one layer: a
+// block's chunks are split into equal ranges of about 256 KB of kept weights
+// (a quarter of that when a launch has too few units to spread over the
+// CTAs).  Persistent CTA b starts on units b and
 // b + grid, then takes units from a shared ticket counter in list order
 // (largest layers first), so a CTA that runs ahead takes more units, and the
 // pipeline never restarts between units.
@@ -579,10 +580,15 @@ int decode_max_tokens() { return kMaxT; }
 
 gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
   p->nblk64 = (int32_t)((p->out + kRows - 1) / kRows);
-  // chunks per unit: about kUnitBytes of kept weights per unit
+  // Chunks per unit: a block's chunks are split into the whole number of
+  // units nearest to its kept bytes / kUnitBytes (at most kMaxCpu chunks
+  // each), of equal length.  Every split costs a partial write and a global
+  // reduction, so a block only slightly above kUnitBytes stays whole instead
+  // of leaving a one-chunk remainder unit.
   const double per_chunk = p->kept > 0 ? 512.0 * (double)p->kept / ((double)p->G * (double)p->nblk64) : 512.0;
-  int cpu = (int)std::floor((double)kUnitBytes / std::max(per_chunk, 1.0) + 0.5);
-  cpu = std::max(1, std::min(cpu, std::min(p->G, kMaxCpu)));
+  int nsplit = (int)std::floor(per_chunk * (double)p->G / (double)kUnitBytes + 0.5);
+  nsplit = std::min(p->G, std::max(nsplit, std::max(1, (p->G + kMaxCpu - 1) / kMaxCpu)));
+  const int cpu = (p->G + nsplit - 1) / nsplit;
   p->dec_cpu = cpu;
   p->dec_cpu_fine = std::max(1, cpu / 4);
   p->dec_nsplit_max = (p->G + p->dec_cpu_fine - 1) / p->dec_cpu_fine;
