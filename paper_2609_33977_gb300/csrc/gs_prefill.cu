@@ -118,6 +118,20 @@ __device__ __forceinline__ int load_tile_items(const PrefillParams& P, int w, in
   return n;
 }
 
+// Read-only global loads kept at their place in the program: volatile asm is
+// not moved across the other volatile asm (barrier waits, TMEM traffic), so a
+// load issued chunks ahead of its use is not sunk down to that use.
+__device__ __forceinline__ int ld_pinned_s32(const int32_t* p) {
+  int v;
+  asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_pinned_u16(const uint16_t* p) {
+  uint16_t v;
+  asm volatile("ld.global.nc.b16 %0, [%1];" : "=h"(v) : "l"(p));
+  return v;
+}
+
 // Chunk c's metadata for an epilogue warp: lanes 0..2 fetch (window offset,
 // kept mask) of the 16-row blocks its 40 rows touch (from block wblk0); lanes
 // 30 and 31 fetch the window slice's start and end.  Chunks past the last read as empty.
@@ -130,11 +144,11 @@ __device__ __forceinline__ void load_chunk_meta(const PrefillParams& P, int c, i
   const int32_t* wo = P.win_off16 + (int64_t)c * (P.nw16 + 1);
   const int wi = wblk0 + lane;
   if (lane < kMetaBlocks && wi < P.nw16) {
-    woff = __ldg(wo + wi);
-    km = __ldg(P.kmask16 + (int64_t)c * P.nw16 + wi);
+    woff = ld_pinned_s32(wo + wi);
+    km = ld_pinned_u16(P.kmask16 + (int64_t)c * P.nw16 + wi);
   }
-  if (lane == 30) bnd = __ldg(wo + wlo);
-  if (lane == 31) bnd = __ldg(wo + whi);
+  if (lane == 30) bnd = ld_pinned_s32(wo + wlo);
+  if (lane == 31) bnd = ld_pinned_s32(wo + whi);
 }
 
 // acc[0..n) += v[0..n), two lanes per packed f32x2 add
