@@ -364,54 +364,77 @@ def run_ours(args):
                              "tokens/s": T / us * 1e6}
 
     # ---- end to end through the public API with host buffers
-    xh = {T: torch.cat([xx.reshape(-1) for xx in xs[T]]).cpu().pin_memory() for T in DECODE_T}
-    xd_flat = {T: torch.empty_like(xh[T], device=dev) for T in DECODE_T}
-    xd_views = {}
-    for T in DECODE_T:
-        off = 0
-        views = []
-        for d in layers:
-            n = T * d["L"].inp
-            views.append(xd_flat[T][off:off + n].view(T, d["L"].inp))
-            off += n
-        xd_views[T] = views
-    yd_flat = {T: torch.empty(sum(T * d["L"].out for d in layers), dtype=torch.bfloat16, device=dev)
-               for T in DECODE_T}
-    yd_views = {}
-    for T in DECODE_T:
-        off = 0
-        views = []
-        for d in layers:
-            n = T * d["L"].out
-            views.append(yd_flat[T][off:off + n].view(T, d["L"].out))
-            off += n
-        yd_views[T] = views
-    yh = {T: torch.empty(yd_flat[T].shape, dtype=torch.bfloat16).pin_memory() for T in DECODE_T}
-    h2d = sum(xh[T].numel() * 2 for T in DECODE_T)
-    d2h = sum(yh[T].numel() * 2 for T in DECODE_T)
+    # One pinned host buffer per direction holds a step's inputs (x of every
+    # projection for T = 1, 4, 16, back to back) and its results.  The device
+    # side alternates between two copies of each, so a step's copies overlap
+    # the neighbouring steps' launches; events order every buffer's reuse.
+    y_len = {T: sum(T * d["L"].out for d in layers) for T in DECODE_T}
+    xh_all = torch.cat([torch.cat([xx.reshape(-1) for xx in xs[T]]) for T in DECODE_T]).cpu().pin_memory()
+    yh_all = torch.empty(sum(y_len.values()), dtype=torch.bfloat16).pin_memory()
+    xd_all = [torch.empty_like(xh_all, device=dev) for _ in range(2)]
+    yd_all = [torch.empty_like(yh_all, device=dev) for _ in range(2)]
+
+    def layer_views(buf, dim):
+        out, off = {}, 0
+        for T in DECODE_T:
+            views = []
+            for d in layers:
+                n = T * getattr(d["L"], dim)
+                views.append(buf[off:off + n].view(T, getattr(d["L"], dim)))
+                off += n
+            out[T] = views
+        return out
+
+    xv = [layer_views(xd_all[k], "inp") for k in range(2)]
+    yv = [layer_views(yd_all[k], "out") for k in range(2)]
+    h2d = xh_all.numel() * 2
+    d2h = yh_all.numel() * 2
     e2e_steps = max(20, min(args.steps, 2000))
-    with torch.cuda.stream(stream):
-        def e2e_step(i):
-            c = i % R
+    h2d_stream = torch.cuda.Stream(device=dev)
+    d2h_stream = torch.cuda.Stream(device=dev)
+    x_ready = [torch.cuda.Event() for _ in range(2)]
+    k_done = [torch.cuda.Event() for _ in range(2)]
+    y_read = [torch.cuda.Event() for _ in range(2)]
+    used = [False, False]
+
+    def e2e_step(i):
+        c, k = i % R, i % 2
+        if used[k]:
+            h2d_stream.wait_event(k_done[k])    # the launches two steps back have read this x buffer
+        with torch.cuda.stream(h2d_stream):
+            xd_all[k].copy_(xh_all, non_blocking=True)
+            x_ready[k].record(h2d_stream)
+        stream.wait_event(x_ready[k])
+        if used[k]:
+            stream.wait_event(y_read[k])        # the copy two steps back has read this y buffer
+        with torch.cuda.stream(stream):
             for T in DECODE_T:
-                xd_flat[T].copy_(xh[T], non_blocking=True)
-                gs.linear_batched_into(xd_views[T], packs[c], yd_views[T], stream=stream)
-                yh[T].copy_(yd_flat[T], non_blocking=True)
-        for i in range(5):
-            e2e_step(i)
-        stream.synchronize()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for i in range(e2e_steps):
-            e2e_step(i)
-        b.record(stream)
-        b.synchronize()
+                gs.linear_batched_into(xv[k][T], packs[c], yv[k][T], stream=stream)
+            k_done[k].record(stream)
+        d2h_stream.wait_event(k_done[k])
+        with torch.cuda.stream(d2h_stream):
+            yh_all.copy_(yd_all[k], non_blocking=True)
+            y_read[k].record(d2h_stream)
+        used[k] = True
+
+    for i in range(5):
+        e2e_step(i)
+    torch.cuda.synchronize(dev)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    h2d_stream.wait_event(a)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    stream.wait_event(y_read[(e2e_steps - 1) % 2])    # the last step's results are on the host
+    b.record(stream)
+    b.synchronize()
+    torch.cuda.synchronize(dev)
     e2e_s = a.elapsed_time(b) / 1e3
     e2e_value = world * tokens_per_step * e2e_steps / e2e_s
     # results of the e2e path equal the device-resident path
-    for T in DECODE_T:
-        assert torch.equal(yh[T].to(dev), torch.cat([yy.reshape(-1) for yy in ys[T]])), "e2e result mismatch"
+    y_dev = torch.cat([torch.cat([yy.reshape(-1) for yy in ys[T]]) for T in DECODE_T])
+    assert torch.equal(yh_all.to(dev), y_dev), "e2e result mismatch"
 
     # ---- dense bf16 torch matmul on the unpruned weights (reference point)
     dense = {}
@@ -463,8 +486,10 @@ def run_ours(args):
                      "frac_of_8TBs_nominal": achieved_gbs / 8000.0},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "steps": e2e_steps, "how": "pinned host x -> device, gs_linear_batched, device y -> pinned host; "
-                                         "per token batch, through the Python binding (no graph)"},
+                "steps": e2e_steps, "how": "per step: one pinned host -> device copy of every x (T = 1, 4, 16), three "
+                                         "gs_linear_batched calls through the Python binding (no graph), one device -> "
+                                         "pinned host copy of every y; copies on their own streams, device buffers "
+                                         "alternating between steps so copies overlap neighbouring launches"},
         "gpu_launches": launches,
         "clocks": clock_rec,
         "per_T": per_T,

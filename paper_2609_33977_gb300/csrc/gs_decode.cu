@@ -65,6 +65,7 @@ constexpr int kRows = kDW * kWin16;           // 64 rows per block
 constexpr int kThreadsDec = (kCW + 1) * 32;   // + one producer warp
 constexpr int kMaxNT = 2;                     // 8-token MMA tiles per launch
 constexpr int kMaxBatch = 32;
+constexpr int kSmallBatch = 8;
 constexpr int kMaxT = 16;                     // tokens per launch (two 8-token MMA tiles)
 constexpr int kRingBytes = 104 * 1024;       // byte ring per CTA (two CTAs per SM)
 constexpr int kRingSeq = 16;                  // chunks that may be in flight (barrier ring)
@@ -96,8 +97,12 @@ struct DecLayer {
   int32_t unit_begin;
 };
 
+// Launch parameters for up to MB layers.  Launches of at most kSmallBatch
+// layers use the small instance: the parameter block (about 256 B per layer)
+// is copied with every launch.
+template <int MB>
 struct DecParams {
-  DecLayer L[kMaxBatch];
+  DecLayer L[MB];
   int32_t n_layers;
   int32_t T;
   int32_t n_units;
@@ -154,8 +159,8 @@ __device__ __forceinline__ void unit_at(const int4* lay, int n_layers, int u, Un
   U.nC = min(L.w, U.c0 + L.z) - U.c0;
 }
 
-template <int NT>
-__global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant__ DecParams P) {
+template <int NT, int MB>
+__global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant__ DecParams<MB> P) {
   extern __shared__ uint8_t dsmem_raw[];
   __shared__ __align__(8) uint64_t w_full[kRingSeq];
   __shared__ __align__(8) uint64_t w_empty[kRingSeq];
@@ -168,8 +173,8 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   __shared__ __align__(8) uint64_t p_full[kDW];    // pair hand-off per window: accumulator written
   __shared__ __align__(8) uint64_t p_empty[kDW];   // ... and consumed
   __shared__ __align__(16) float pair_buf[kDW * 32 * 4 * kMaxNT];
-  __shared__ int4 lay[kMaxBatch];               // per layer: {first unit, splits per block, chunks per unit, chunks}
-  __shared__ const int4* lay_dmeta[kMaxBatch];  // per layer: chunk metadata
+  __shared__ int4 lay[MB];                      // per layer: {first unit, splits per block, chunks per unit, chunks}
+  __shared__ const int4* lay_dmeta[MB];         // per layer: chunk metadata
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~uintptr_t(1023));
   int4* meta = reinterpret_cast<int4*>(ring + kRingBytes);   // [kMetaSlots][kMaxCpu]
 
@@ -553,12 +558,12 @@ int sm_count_dec() {
   return n;
 }
 
-template <int NT>
-cudaError_t launch_nt(const DecParams& P, int grid, cudaStream_t s) {
+template <int NT, int MB>
+cudaError_t launch_nt(const DecParams<MB>& P, int grid, cudaStream_t s) {
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, []() {
-    attr_err = cudaFuncSetAttribute(k_decode<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
+    attr_err = cudaFuncSetAttribute(k_decode<NT, MB>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
   cudaLaunchConfig_t cfg = {};
@@ -571,7 +576,7 @@ cudaError_t launch_nt(const DecParams& P, int grid, cudaStream_t s) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_decode<NT>, P);
+  return cudaLaunchKernelEx(&cfg, k_decode<NT, MB>, P);
 }
 
 }  // namespace
@@ -639,7 +644,7 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
   }
   const bool all_fine = coarse_units < 2 * max_grid;
   std::vector<char> fine(n, all_fine ? 1 : 0);
-  DecParams P;
+  DecParams<kMaxBatch> P;
   std::memset(&P, 0, sizeof(P));
   P.n_layers = n;
   P.T = T;
@@ -670,7 +675,19 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
   P.n_units = (int32_t)units;
   P.sched = ps[0]->dec_cnt + (size_t)ps[0]->nblk64 * kDW;
   const int grid = (int)std::min<int64_t>(units, max_grid);
-  const cudaError_t e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);
+  cudaError_t e;
+  if (n <= kSmallBatch) {
+    DecParams<kSmallBatch> Q;
+    std::memcpy(Q.L, P.L, sizeof(Q.L));
+    Q.n_layers = P.n_layers;
+    Q.T = P.T;
+    Q.n_units = P.n_units;
+    Q.sched = P.sched;
+    Q.err = P.err;
+    e = T <= 8 ? launch_nt<1>(Q, grid, s) : launch_nt<2>(Q, grid, s);
+  } else {
+    e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);
+  }
   note_launch();
   return e == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }
