@@ -162,6 +162,32 @@ def test_block_workload_decode_batched(gs):
     assert gs.device_status() == gs.GS_OK
 
 
+@pytest.mark.parametrize("n", [9, 12, 32])
+def test_decode_batched_many_layers(gs, n):
+    """More layers in one decode launch than the small parameter block holds
+    (up to the 32-layer limit), with mixed shapes and densities, the split and
+    unsplit unit paths, and T = 3 and 16."""
+    import torch
+    outs = [64, 200, 256, 512, 1000, 1024]
+    inps = [256, 512, 1024, 2048, 2816]
+    dens = [0.2, 0.5, 0.8, 1.0, 0.05]
+    Ws, Bs, ps = [], [], []
+    for i in range(n):
+        out, inp, d = outs[i % len(outs)], inps[(3 * i) % len(inps)], dens[(5 * i) % len(dens)]
+        Wb, B = layer(out, inp, d, 500 + i)
+        Ws.append(Wb)
+        Bs.append(B)
+        ps.append(packed(gs, Wb, B))
+    for T in (3, 16):
+        xs = [wl.random_activation_bits(T, W.shape[1], seed=700 + 17 * i + T) for i, W in enumerate(Ws)]
+        xd = [to_dev(x) for x in xs]
+        ys = [torch.empty((T, W.shape[0]), dtype=torch.bfloat16, device="cuda") for W in Ws]
+        gs.linear_batched_into(xd, ps, ys)
+        for i in range(n):
+            assert_within_bound(to_bits(ys[i]), xs[i], Ws[i], Bs[i], what=f"batched n={n} layer {i} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
 def stack_blocks(w, k):
     """Blocks checked for a stack: the first, the last, and the blocks holding
     the sparsest and the densest layer of the layer-adaptive allocation."""
