@@ -506,17 +506,17 @@ def run_ours(args):
 
 
 def _time_block(gs, torch, stream, xd, ps, ys, algo, n=10):
-    """Seconds per pass over one block's 7 projections (CUDA events, after warm-up)."""
+    """Seconds per pass over one block's 7 projections (CUDA events, after warm-up);
+    one batched call per pass (T >= 33 takes the tensor-core prefill kernel)."""
+    assert algo == gs.ALGO_PREFILL and xd[0].shape[0] >= 33
     with torch.cuda.stream(stream):
         for _ in range(3):
-            for i in range(len(ps)):
-                gs.linear_into(xd[i], ps[i], ys[i], algo=algo, stream=stream)
+            gs.linear_batched_into(xd, ps, ys, stream=stream)
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(n):
-            for i in range(len(ps)):
-                gs.linear_into(xd[i], ps[i], ys[i], algo=algo, stream=stream)
+            gs.linear_batched_into(xd, ps, ys, stream=stream)
         b.record(stream)
         b.synchronize()
     return a.elapsed_time(b) / 1e3 / n

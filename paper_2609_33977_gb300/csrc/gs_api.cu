@@ -203,11 +203,21 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
   if (T == 0) return GS_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (T >= kPrefillMinTokens) {
+    // layers the prefill kernel takes share batched launches; any other goes alone
+    std::vector<const void*> xp;
+    std::vector<const gs_packed*> pp;
+    std::vector<void*> yp;
     for (int i = 0; i < n; ++i) {
-      const gs_status st = linear_impl(xs_dev[i], ps[i], T, ys_dev[i], stream, GS_ALGO_AUTO);
-      if (st != GS_OK) return st;
+      if (ps[i]->G <= prefill_max_chunks()) {
+        xp.push_back(xs_dev[i]);
+        pp.push_back(ps[i]);
+        yp.push_back(ys_dev[i]);
+      } else {
+        const gs_status st = linear_impl(xs_dev[i], ps[i], T, ys_dev[i], stream, GS_ALGO_AUTO);
+        if (st != GS_OK) return st;
+      }
     }
-    return GS_OK;
+    return launch_prefill_batched(xp.data(), pp.data(), (int)pp.size(), T, yp.data(), s);
   }
   const int64_t blk = decode_max_tokens();
   std::vector<const void*> xb(n);

@@ -77,6 +77,8 @@ int decode_max_tokens();
 // prefill.cu
 gs_status prefill_prepare_weight_maps(gs_packed* p);
 gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, cudaStream_t s);
+gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T,
+                                 void* const* ys, cudaStream_t s);
 int prefill_max_chunks();
 
 }  // namespace gs

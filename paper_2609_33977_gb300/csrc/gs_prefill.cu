@@ -33,7 +33,9 @@
 #include "gs_sm100.cuh"
 
 #include <cuda.h>
+#include <algorithm>
 #include <cstring>
+#include <vector>
 #include <mutex>
 
 namespace gs {
@@ -77,16 +79,31 @@ static_assert(kFW % 32 == 0 && kRowsPerWarp % 8 == 0 && kNMax % 16 == 0, "tile s
 static_assert(kRowsPerWarp <= 32 + 8, "the address table is built in two lane rounds");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
-struct PrefillParams {
+// One launch covers up to kMaxLayers layers with the same T; the pairs walk
+// one list of tiles, layer after layer (tile_begin = first tile of a layer).
+constexpr int kMaxLayers = 8;
+struct PrefillLayer {
   CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 2
   CUtensorMap wmap[kNMaps];  // tiles as (64, kept, 4) slabs, box 64 x 8(i+1) x 2
   const int32_t* win_off16;
   const uint16_t* kmask16;
   uint16_t* y;
-  int32_t out, G, nw16, T;
+  int32_t out, G, nw16;
   int32_t n_m, n_w;          // pair tiles: ceil(T / 256) x ceil(out / 160)
+  int32_t tile_begin;
+};
+struct PrefillParams {
+  PrefillLayer L[kMaxLayers];
+  int32_t n_layers, T, n_tiles;
   int* err;
 };
+
+// layer of global tile t
+__device__ __forceinline__ int tile_layer(const PrefillParams& P, int t) {
+  int l = 0;
+  while (l + 1 < P.n_layers && P.L[l + 1].tile_begin <= t) ++l;
+  return l;
+}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
@@ -96,7 +113,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // Items of a tile: the chunks whose window slice (kept rows = packed rows
 // [p0, p1)) is non-empty, in chunk order.  The warp builds the list in shared
 // memory, 32 chunks per round: entry = {chunk | (rows rounded up to 16) << 16, p0}.
-__device__ __forceinline__ int load_tile_items(const PrefillParams& P, int w, int lane, int2* items) {
+__device__ __forceinline__ int load_tile_items(const PrefillLayer& P, int w, int lane, int2* items) {
   const int wlo = (kFW / kWin16) * w;
   const int whi = min(wlo + kFW / kWin16, P.nw16);
   int n = 0;
@@ -135,7 +152,7 @@ __device__ __forceinline__ uint32_t ld_pinned_u16(const uint16_t* p) {
 // Chunk c's metadata for an epilogue warp: lanes 0..2 fetch (window offset,
 // kept mask) of the 16-row blocks its 40 rows touch (from block wblk0); lanes
 // 30 and 31 fetch the window slice's start and end.  Chunks past the last read as empty.
-__device__ __forceinline__ void load_chunk_meta(const PrefillParams& P, int c, int wlo, int whi, int wblk0, int lane,
+__device__ __forceinline__ void load_chunk_meta(const PrefillLayer& P, int c, int wlo, int whi, int wblk0, int lane,
                                                 int& bnd, int& woff, uint32_t& km) {
   bnd = 0;
   woff = 0;
@@ -205,8 +222,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     mbar_init(&drain_bar, 1);
     abort_s = 0;
     fence_mbar_init();
-    prefetch_tmap(&P.xmap);
-    for (int h = 0; h < kNMaps; ++h) prefetch_tmap(&P.wmap[h]);
+    for (int l = 0; l < P.n_layers; ++l) {
+      prefetch_tmap(&P.L[l].xmap);
+      for (int h = 0; h < kNMaps; ++h) prefetch_tmap(&P.L[l].wmap[h]);
+    }
   }
   if (warp == 1) {
     tmem_alloc_pair(&tmem_base_s, kTmemCols);
@@ -217,7 +236,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   volatile int* abort_flag = &abort_s;
-  const int n_tiles = P.n_m * P.n_w;
+  const int n_tiles = P.n_tiles;
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
 
   if (warp == 0) {
@@ -226,14 +245,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     uint32_t armed = 0u, armed_par = 0u;   // per stage: a copy was issued / the phase it completes
     bool ok = true;
     for (int t = pair; t < n_tiles && ok; t += n_pairs) {
-      const int m = t % P.n_m, w = t / P.n_m;
-      const int n_items = load_tile_items(P, w, lane, items);
+      const PrefillLayer& L = P.L[tile_layer(P, t)];
+      const int lt = t - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      const int n_items = load_tile_items(L, w, lane, items);
       if (lane == 0) {
         for (int it = 0; it < n_items && ok; ++it) {
           const int2 e = items[it];
           const int c = e.x & 0xFFFF, nr = e.x >> 16, start = e.y;
           const int hn = nr >> 1;   // slice rows held by each CTA of the pair
-          const CUtensorMap* wm = &P.wmap[(hn >> 3) - 1];
+          const CUtensorMap* wm = &L.wmap[(hn >> 3) - 1];
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kWaitLimitNs,
                                    kDevErrTimeout)) {
@@ -246,7 +267,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
             if (rank == 0)
               mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(2 * kXStageBytes + nr * kSlabs * kBK * 2));
             const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
-            tma_load_3d_pair(sx, &P.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+            tma_load_3d_pair(sx, &L.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
             tma_load_3d_pair(sx + kXStageBytes, wm, fb, 0, start + (int)rank * hn, ks * kSlabs);
             armed |= 1u << stage;
             armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
@@ -276,8 +297,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     uint32_t se_ph = 0u;   // bit b: parity of scratch buffer b's next release
     bool ok = true;
     for (int t = pair; t < n_tiles && ok; t += n_pairs) {
-      const int w = t / P.n_m;
-      const int n_items = load_tile_items(P, w, lane, items);
+      const PrefillLayer& L = P.L[tile_layer(P, t)];
+      const int w = (t - L.tile_begin) / L.n_m;
+      const int n_items = load_tile_items(L, w, lane, items);
       if (lane == 0) {
         for (int it = 0; it < n_items && ok; ++it) {
           const int nr = items[it].x >> 16;
@@ -341,7 +363,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     uint32_t sf_ph = 0u;   // bit b: parity of scratch buffer b's next fill
     bool ok = true;
     for (int t = pair; t < n_tiles && ok; t += n_pairs) {
-      const int m = t % P.n_m, w = t / P.n_m;
+      const PrefillLayer& L = P.L[tile_layer(P, t)];
+      const int lt = t - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
       const int r0 = w * kFW + kRowsPerWarp * g;
       const int wblk0 = (kFW / kWin16) * w + (kRowsPerWarp * g) / kBlkRows;
       const int rsh = (kRowsPerWarp * g) % kBlkRows;   // the warp's first row within block wblk0
@@ -352,13 +376,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
       // prefetched four chunks ahead into four register slots.  The loop is
       // unrolled by four so a slot is read (its load long complete) and only
       // then reloaded; no register copy ever waits on a load in flight.
-      const int wlo = (kFW / kWin16) * w, whi = min(wlo + kFW / kWin16, P.nw16);
+      const int wlo = (kFW / kWin16) * w, whi = min(wlo + kFW / kWin16, L.nw16);
       int bnd0, bnd1, bnd2, bnd3, wo0, wo1, wo2, wo3;
       uint32_t km0, km1, km2, km3;
-      load_chunk_meta(P, 0, wlo, whi, wblk0, lane, bnd0, wo0, km0);
-      load_chunk_meta(P, 1, wlo, whi, wblk0, lane, bnd1, wo1, km1);
-      load_chunk_meta(P, 2, wlo, whi, wblk0, lane, bnd2, wo2, km2);
-      load_chunk_meta(P, 3, wlo, whi, wblk0, lane, bnd3, wo3, km3);
+      load_chunk_meta(L, 0, wlo, whi, wblk0, lane, bnd0, wo0, km0);
+      load_chunk_meta(L, 1, wlo, whi, wblk0, lane, bnd1, wo1, km1);
+      load_chunk_meta(L, 2, wlo, whi, wblk0, lane, bnd2, wo2, km2);
+      load_chunk_meta(L, 3, wlo, whi, wblk0, lane, bnd3, wo3, km3);
       // Gather addresses of a chunk (its metadata slot), for scratch buffer
       // `buf`: row r of the warp (window row 40g + r: block k, bit i; kept
       // mask m, first kept row at scratch column b0) reads scratch column
@@ -385,7 +409,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
       // after the buffer is handed back, then the loaded values are added.
       auto step = [&](int c, int& bnd, int& wo, uint32_t& kmr, int bnd_n, int wo_n, uint32_t km_n) {
         const int p0 = __shfl_sync(0xffffffffu, bnd, 30), p1 = __shfl_sync(0xffffffffu, bnd, 31);
-        load_chunk_meta(P, c + 4, wlo, whi, wblk0, lane, bnd, wo, kmr);
+        load_chunk_meta(L, c + 4, wlo, whi, wblk0, lane, bnd, wo, kmr);
         uint32_t* t_cur = tbl + (c & 1) * kAcc;
         uint32_t* t_next = tbl + ((c + 1) & 1) * kAcc;
         if (p1 <= p0 || !ok) {
@@ -411,30 +435,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
         add_f32x2<kAcc>(acc, v);
       };
       build_table(tbl, bnd0, wo0, km0);
-      for (int c = 0; c < P.G && ok; c += 4) {
+      for (int c = 0; c < L.G && ok; c += 4) {
         step(c, bnd0, wo0, km0, bnd1, wo1, km1);
-        if (c + 1 < P.G) step(c + 1, bnd1, wo1, km1, bnd2, wo2, km2);
-        if (c + 2 < P.G) step(c + 2, bnd2, wo2, km2, bnd3, wo3, km3);
-        if (c + 3 < P.G) step(c + 3, bnd3, wo3, km3, bnd0, wo0, km0);
+        if (c + 1 < L.G) step(c + 1, bnd1, wo1, km1, bnd2, wo2, km2);
+        if (c + 2 < L.G) step(c + 2, bnd2, wo2, km2, bnd3, wo3, km3);
+        if (c + 3 < L.G) step(c + 3, bnd3, wo3, km3, bnd0, wo0, km0);
       }
       if (!ok) break;
       // accumulators -> bf16 y rows [r0, r0 + 40) of token tok
       const int tok = m * kPairM + (int)rank * kBM + 32 * q + lane;
       if (tok < P.T) {
-        uint16_t* yrow = P.y + (int64_t)tok * P.out;
-        const bool vec_ok = (P.out & 7) == 0;
+        uint16_t* yrow = L.y + (int64_t)tok * L.out;
+        const bool vec_ok = (L.out & 7) == 0;
 #pragma unroll
         for (int k = 0; k < kAcc / 8; ++k) {
           const int rb = r0 + 8 * k;
           const float* a = acc + 8 * k;
-          if (vec_ok && rb + 8 <= P.out) {
+          if (vec_ok && rb + 8 <= L.out) {
             *reinterpret_cast<uint4*>(yrow + rb) =
                 make_uint4(pack_bf16x2(a[0], a[1]), pack_bf16x2(a[2], a[3]), pack_bf16x2(a[4], a[5]),
                            pack_bf16x2(a[6], a[7]));
           } else {
 #pragma unroll
             for (int i = 0; i < 8; ++i)
-              if (rb + i < P.out) yrow[rb + i] = __bfloat16_as_ushort(__float2bfloat16_rn(a[i]));
+              if (rb + i < L.out) yrow[rb + i] = __bfloat16_as_ushort(__float2bfloat16_rn(a[i]));
           }
         }
       }
@@ -488,41 +512,74 @@ gs_status prefill_prepare_weight_maps(gs_packed* p) {
 
 int prefill_max_chunks() { return kMaxG; }
 
-gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, cudaStream_t s) {
-  if (T <= 0) return GS_OK;
-  if (p->kept == 0) {
-    return cudaMemsetAsync(y, 0, (size_t)T * (size_t)p->out * 2, s) == cudaSuccess ? GS_OK : GS_ERR_CUDA;
-  }
-  if (!p->wmaps_valid) return GS_ERR_CUDA;
-  if (p->G > kMaxG) return GS_ERR_UNSUPPORTED;
+gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T,
+                                 void* const* ys, cudaStream_t s) {
+  if (T <= 0 || n <= 0) return GS_OK;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, []() {
     attr_err = cudaFuncSetAttribute(k_prefill, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   });
   if (attr_err != cudaSuccess) return GS_ERR_CUDA;
-
-  PrefillParams P;
-  std::memset(&P, 0, sizeof(P));
-  if (!encode_tmap_slabs_bf16(&P.xmap, x, (uint64_t)p->in, (uint64_t)T, kBM, kSlabs)) return GS_ERR_CUDA;
-  for (int h = 0; h < kNMaps; ++h) std::memcpy(&P.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
-  P.win_off16 = p->win_off16;
-  P.kmask16 = p->kmask16;
-  P.y = static_cast<uint16_t*>(y);
-  P.out = (int32_t)p->out;
-  P.G = p->G;
-  P.nw16 = p->nw16;
-  P.T = (int32_t)T;
-  P.n_m = (int32_t)((T + kPairM - 1) / kPairM);
-  P.n_w = (int32_t)((p->out + kFW - 1) / kFW);
-  P.err = device_error_flag();
-  if (!P.err) return GS_ERR_CUDA;
-  const int64_t tiles = (int64_t)P.n_m * P.n_w;
+  // Layers with no kept group produce zeros; the others share launches of up
+  // to kMaxLayers, largest work per tile (kept groups per window) first, so
+  // the last tiles the pairs pick up are the short ones.
+  std::vector<int> order;
+  for (int i = 0; i < n; ++i) {
+    const gs_packed* p = ps[i];
+    if (p->kept == 0) {
+      if (cudaMemsetAsync(ys[i], 0, (size_t)T * (size_t)p->out * 2, s) != cudaSuccess) return GS_ERR_CUDA;
+      continue;
+    }
+    if (!p->wmaps_valid) return GS_ERR_CUDA;
+    if (p->G > kMaxG) return GS_ERR_UNSUPPORTED;
+    order.push_back(i);
+  }
+  auto tile_work = [&](int i) {
+    const gs_packed* p = ps[i];
+    return (double)p->kept / (double)((p->out + kFW - 1) / kFW);
+  };
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return tile_work(a) > tile_work(b); });
+  int* err = device_error_flag();
+  if (!err) return GS_ERR_CUDA;
   const int64_t max_pairs = sm_count() / 2;
-  const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs (cluster dims 2)
-  k_prefill<<<grid, kThreads, kSmemBytes, s>>>(P);
-  note_launch();
-  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+  for (size_t b0 = 0; b0 < order.size(); b0 += kMaxLayers) {
+    const int nb = (int)std::min<size_t>(kMaxLayers, order.size() - b0);
+    PrefillParams P;
+    std::memset(&P, 0, sizeof(P));
+    int64_t tiles = 0;
+    for (int k = 0; k < nb; ++k) {
+      const int i = order[b0 + k];
+      const gs_packed* p = ps[i];
+      PrefillLayer& L = P.L[k];
+      if (!encode_tmap_slabs_bf16(&L.xmap, xs[i], (uint64_t)p->in, (uint64_t)T, kBM, kSlabs)) return GS_ERR_CUDA;
+      for (int h = 0; h < kNMaps; ++h) std::memcpy(&L.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
+      L.win_off16 = p->win_off16;
+      L.kmask16 = p->kmask16;
+      L.y = static_cast<uint16_t*>(ys[i]);
+      L.out = (int32_t)p->out;
+      L.G = p->G;
+      L.nw16 = p->nw16;
+      L.n_m = (int32_t)((T + kPairM - 1) / kPairM);
+      L.n_w = (int32_t)((p->out + kFW - 1) / kFW);
+      L.tile_begin = (int32_t)tiles;
+      tiles += (int64_t)L.n_m * L.n_w;
+    }
+    if (tiles > INT32_MAX) return GS_ERR_UNSUPPORTED;
+    P.n_layers = nb;
+    P.T = (int32_t)T;
+    P.n_tiles = (int32_t)tiles;
+    P.err = err;
+    const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs (cluster dims 2)
+    k_prefill<<<grid, kThreads, kSmemBytes, s>>>(P);
+    note_launch();
+    if (cudaGetLastError() != cudaSuccess) return GS_ERR_CUDA;
+  }
+  return GS_OK;
+}
+
+gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, cudaStream_t s) {
+  return launch_prefill_batched(&x, &p, 1, T, &y, s);
 }
 
 }  // namespace gs

@@ -188,6 +188,33 @@ def test_decode_batched_many_layers(gs, n):
     assert gs.device_status() == gs.GS_OK
 
 
+@pytest.mark.parametrize("n,T", [(3, 200), (11, 300)])
+def test_prefill_batched_matches_single(gs, n, T):
+    """A batched prefill call (several layers with one T share launches of up
+    to 8 layers) gives bit for bit the single-layer results and stays within
+    the bound; layers without kept groups give zeros."""
+    import torch
+    shapes = [(4096, 4096, 0.5), (1000, 1024, 0.3), (512, 2816, 0.8), (300, 256, 0.0), (2048, 512, 1.0),
+              (160, 768, 0.5), (1100, 2048, 0.05)]
+    Ws, Bs, ps = [], [], []
+    for i in range(n):
+        out, inp, d = shapes[i % len(shapes)]
+        Wb, B = layer(out, inp, d, 900 + i)
+        Ws.append(Wb)
+        Bs.append(B)
+        ps.append(packed(gs, Wb, B))
+    xs = [wl.random_activation_bits(T, W.shape[1], seed=950 + i) for i, W in enumerate(Ws)]
+    xd = [to_dev(x) for x in xs]
+    ys = [torch.full((T, W.shape[0]), 7.0, dtype=torch.bfloat16, device="cuda") for W in Ws]
+    gs.linear_batched_into(xd, ps, ys)
+    toks = sample_tokens(T, seed=n)
+    for i in range(n):
+        y1 = gs.linear(xd[i], ps[i])
+        assert np.array_equal(to_bits(ys[i]), to_bits(y1)), f"layer {i}: batched != single"
+        assert_within_bound(to_bits(ys[i]), xs[i], Ws[i], Bs[i], tokens=toks, what=f"batched prefill layer {i}")
+    assert gs.device_status() == gs.GS_OK
+
+
 def stack_blocks(w, k):
     """Blocks checked for a stack: the first, the last, and the blocks holding
     the sparsest and the densest layer of the layer-adaptive allocation."""
