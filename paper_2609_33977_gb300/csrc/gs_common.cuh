@@ -42,6 +42,7 @@ struct gs_packed {
   int32_t* dec_cnt;   // [nblk64][4] arrival counters, then {unit ticket, finished CTAs} (self-resetting)
   // tcgen05 prefill: slab TMA descriptors over the tiles, box heights 16, 32, ..., 160 rows
   alignas(64) unsigned char wmaps[10][128];
+  alignas(64) unsigned char wmaps_full[10][128];   // same, box heights 16, 32, ..., 160 (whole slices)
   bool wmaps_valid;
 };
 

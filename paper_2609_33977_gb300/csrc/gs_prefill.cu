@@ -73,6 +73,16 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDrainLimitNs = 200000000ull;
 constexpr int kSmemBytes = kStages * kStageBytes + 2 * kMetaInts * 4 + kTblBytes + 1024;
 
+// Single-CTA tiles (T <= 128, where a pair tile would be half empty): each CTA
+// loads its tile's whole slice per stage and issues its own M = 128 MMAs.
+constexpr int kWStageBytesSingle = kSlabs * kNMax * kBK * 2;          // 40 KB: a whole slice
+constexpr int kStageBytesSingle = kXStageBytes + kWStageBytesSingle;  // 72 KB
+constexpr int kStagesSingle = 3;
+constexpr int kSmemBytesSingle = kStagesSingle * kStageBytesSingle + 2 * kMetaInts * 4 + kTblBytes + 1024;
+static_assert(kStagesSingle <= kStages, "barrier arrays are sized for the pair layout");
+static_assert(kStageBytesSingle % 1024 == 0, "stages must keep 1024-byte alignment");
+static_assert(kSmemBytesSingle <= 227 * 1024, "shared memory budget (single-CTA tiles)");
+
 static_assert(kZeroCol + 32 <= kTmemCols, "TMEM budget (scratch buffers + zero columns)");
 static_assert(kStageBytes % 1024 == 0 && kXSlabBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 static_assert(kFW % 32 == 0 && kRowsPerWarp % 8 == 0 && kNMax % 16 == 0, "tile shape");
@@ -84,7 +94,7 @@ static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 constexpr int kMaxLayers = 8;
 struct PrefillLayer {
   CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 2
-  CUtensorMap wmap[kNMaps];  // tiles as (64, kept, 4) slabs, box 64 x 8(i+1) x 2
+  CUtensorMap wmap[kNMaps];  // tiles as (64, kept, 4) slabs, box 64 x h(i+1) x 2: h = 8 (pair halves) or 16 (whole slices)
   const int32_t* win_off16;
   const uint16_t* kmask16;
   uint16_t* y;
@@ -195,7 +205,10 @@ __device__ __forceinline__ void gather_rows(const uint32_t* tbl, uint32_t* v) {
   }
 }
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
+template <bool kPair>
+__global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
+  constexpr int kStg = kPair ? kStages : kStagesSingle;
+  constexpr int kStgBytes = kPair ? kStageBytes : kStageBytesSingle;
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ __align__(8) uint64_t empty_bar[kStages];
@@ -207,17 +220,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs), 1: peer
-  int2* items = reinterpret_cast<int2*>(smem + kStages * kStageBytes) + (warp < 2 ? warp : 0) * kMaxG;
+  const uint32_t rank = kPair ? cluster_ctarank() : 0u;   // 0: leader (issues the pair's MMAs), 1: peer
+  int2* items = reinterpret_cast<int2*>(smem + kStg * kStgBytes) + (warp < 2 ? warp : 0) * kMaxG;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kStg; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
     for (int b = 0; b < kScrBufs; ++b) {
       mbar_init(&sfull_bar[b], 1);
-      mbar_init(&sempty_bar[b], 2 * kEpiWarps);   // the epilogue warps of both CTAs
+      mbar_init(&sempty_bar[b], (kPair ? 2 : 1) * kEpiWarps);   // the epilogue warps of the tile's CTAs
     }
     mbar_init(&drain_bar, 1);
     abort_s = 0;
@@ -228,16 +241,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     }
   }
   if (warp == 1) {
-    tmem_alloc_pair(&tmem_base_s, kTmemCols);
-    tmem_relinquish_pair();
+    if constexpr (kPair) {
+      tmem_alloc_pair(&tmem_base_s, kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&tmem_base_s, kTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  cluster_sync_all();
+  if constexpr (kPair) cluster_sync_all();
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   volatile int* abort_flag = &abort_s;
   const int n_tiles = P.n_tiles;
-  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  // tile owners: CTA pairs, or single CTAs
+  const int pair = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int n_pairs = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -254,24 +275,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
           const int2 e = items[it];
           const int c = e.x & 0xFFFF, nr = e.x >> 16, start = e.y;
           const int hn = nr >> 1;   // slice rows held by each CTA of the pair
-          const CUtensorMap* wm = &L.wmap[(hn >> 3) - 1];
+          const CUtensorMap* wm = kPair ? &L.wmap[(hn >> 3) - 1] : &L.wmap[(nr >> 4) - 1];
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kWaitLimitNs,
                                    kDevErrTimeout)) {
               ok = false;
               break;
             }
-            uint8_t* sx = smem + stage * kStageBytes;
-            // both CTAs' copies complete on the leader's full barrier, which
-            // expects the bytes of the two halves
-            if (rank == 0)
-              mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(2 * kXStageBytes + nr * kSlabs * kBK * 2));
-            const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
-            tma_load_3d_pair(sx, &L.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
-            tma_load_3d_pair(sx + kXStageBytes, wm, fb, 0, start + (int)rank * hn, ks * kSlabs);
+            uint8_t* sx = smem + stage * kStgBytes;
+            if constexpr (kPair) {
+              // both CTAs' copies complete on the leader's full barrier, which
+              // expects the bytes of the two halves
+              if (rank == 0)
+                mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(2 * kXStageBytes + nr * kSlabs * kBK * 2));
+              const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+              tma_load_3d_pair(sx, &L.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+              tma_load_3d_pair(sx + kXStageBytes, wm, fb, 0, start + (int)rank * hn, ks * kSlabs);
+            } else {
+              mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(kXStageBytes + nr * kSlabs * kBK * 2));
+              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+              tma_load_3d(sx + kXStageBytes, wm, &full_bar[stage], 0, start, ks * kSlabs);
+            }
             armed |= 1u << stage;
             armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
-            if (++stage == kStages) {
+            if (++stage == kStg) {
               stage = 0;
               phase ^= 1u;
             }
@@ -282,7 +309,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     }
     if (lane == 0 && !ok && rank == 0) {
       // let copies already in flight land before the CTA retires
-      for (int s = 0; s < kStages; ++s) {
+      for (int s = 0; s < kStg; ++s) {
         if (!((armed >> s) & 1u)) continue;
         const uint64_t t0 = globaltimer_ns();
         while (!mbar_try_wait(&full_bar[s], (armed_par >> s) & 1u))
@@ -303,39 +330,49 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
       if (lane == 0) {
         for (int it = 0; it < n_items && ok; ++it) {
           const int nr = items[it].x >> 16;
-          if (!mbar_wait_bounded_cluster(&sempty_bar[buf], ((se_ph >> buf) & 1u) ^ 1u, abort_flag, P.err,
-                                         kWaitLimitNs, kDevErrTimeout)) {
+          const bool freed =
+              kPair ? mbar_wait_bounded_cluster(&sempty_bar[buf], ((se_ph >> buf) & 1u) ^ 1u, abort_flag, P.err,
+                                                kWaitLimitNs, kDevErrTimeout)
+                    : mbar_wait_bounded(&sempty_bar[buf], ((se_ph >> buf) & 1u) ^ 1u, abort_flag, P.err, kWaitLimitNs,
+                                        kDevErrTimeout);
+          if (!freed) {
             ok = false;
             break;
           }
           se_ph ^= 1u << buf;
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(buf * kNMax);
-          const uint32_t idesc = idesc_bf16_f32(kPairM, nr);
+          const uint32_t idesc = idesc_bf16_f32(kPair ? kPairM : kBM, nr);
           for (int ks = 0; ks < kKSteps; ++ks) {
             if (!mbar_wait_bounded(&full_bar[stage], phase, abort_flag, P.err, kWaitLimitNs, kDevErrTimeout)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sx = smem_u32(smem + stage * kStageBytes);
+            const uint32_t sx = smem_u32(smem + stage * kStgBytes);
 #pragma unroll
             for (int j = 0; j < kSlabs; ++j) {
               const uint64_t ad = sdesc_sw128(sx + j * kXSlabBytes);
-              const uint64_t bd = sdesc_sw128(sx + kXStageBytes + j * (nr >> 1) * (kBK * 2));
+              const uint64_t bd = sdesc_sw128(sx + kXStageBytes + j * (kPair ? (nr >> 1) : nr) * (kBK * 2));
 #pragma unroll
-              for (int kk = 0; kk < kBK / 16; ++kk)
-                mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
-                                 (ks | j | kk) != 0 ? 1u : 0u);
+              for (int kk = 0; kk < kBK / 16; ++kk) {
+                if constexpr (kPair)
+                  mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
+                                   (ks | j | kk) != 0 ? 1u : 0u);
+                else
+                  mma_bf16_ss(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc, (ks | j | kk) != 0 ? 1u : 0u);
+              }
             }
-            mma_commit_pair_mc(&empty_bar[stage], 0x3);
-            if (++stage == kStages) {
+            if constexpr (kPair) mma_commit_pair_mc(&empty_bar[stage], 0x3);
+            else mma_commit(&empty_bar[stage]);
+            if (++stage == kStg) {
               stage = 0;
               phase ^= 1u;
             }
           }
           if (!ok) break;
-          mma_commit_pair_mc(&sfull_bar[buf], 0x3);
+          if constexpr (kPair) mma_commit_pair_mc(&sfull_bar[buf], 0x3);
+          else mma_commit(&sfull_bar[buf]);
           if (++buf == kScrBufs) buf = 0;
         }
       }
@@ -343,7 +380,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     }
     if (lane == 0) {
       // all MMAs issued by this thread have completed once drain_bar flips
-      mma_commit_pair(&drain_bar);
+      if constexpr (kPair) mma_commit_pair(&drain_bar);
+      else mma_commit(&drain_bar);
       mbar_wait_bounded(&drain_bar, 0u, nullptr, P.err, kWaitLimitNs, kDevErrTimeout);
     }
     __syncwarp();
@@ -358,7 +396,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     const uint32_t t_zero = t_scr + kZeroCol;
     tmem_st_x32_zero(t_zero);
     tmem_wait_st();
-    uint32_t* tbl = reinterpret_cast<uint32_t*>(smem + kStages * kStageBytes + 2 * kMetaInts * 4) + ew * 2 * kAcc;
+    uint32_t* tbl = reinterpret_cast<uint32_t*>(smem + kStg * kStgBytes + 2 * kMetaInts * 4) + ew * 2 * kAcc;
     int buf = 0;
     uint32_t sf_ph = 0u;   // bit b: parity of scratch buffer b's next fill
     bool ok = true;
@@ -429,7 +467,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
         reg_fence(v);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&sempty_bar[buf]), 0));
+        if (lane == 0) {
+          if constexpr (kPair) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&sempty_bar[buf]), 0));
+          else mbar_arrive(&sempty_bar[buf]);
+        }
         if (++buf == kScrBufs) buf = 0;
         build_table(t_next, bnd_n, wo_n, km_n);
         add_f32x2<kAcc>(acc, v);
@@ -443,7 +484,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
       }
       if (!ok) break;
       // accumulators -> bf16 y rows [r0, r0 + 40) of token tok
-      const int tok = m * kPairM + (int)rank * kBM + 32 * q + lane;
+      const int tok = (kPair ? m * kPairM + (int)rank * kBM : m * kBM) + 32 * q + lane;
       if (tok < P.T) {
         uint16_t* yrow = L.y + (int64_t)tok * L.out;
         const bool vec_ok = (L.out & 7) == 0;
@@ -473,12 +514,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) k_prefi
     while (globaltimer_ns() - t0 < 2000000ull) {
     }
   }
-  cluster_sync_all();
+  if constexpr (kPair) cluster_sync_all();
+  else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc_pair(tmem, kTmemCols);
+    if constexpr (kPair) tmem_dealloc_pair(tmem, kTmemCols);
+    else tmem_dealloc(tmem, kTmemCols);
   }
-  cluster_sync_all();
+  if constexpr (kPair) cluster_sync_all();
+  else __syncthreads();
 }
 
 // ------------------------------------------------------------------ host side
@@ -505,6 +549,9 @@ gs_status prefill_prepare_weight_maps(gs_packed* p) {
     if (!encode_tmap_slabs_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, (uint32_t)(8 * (h + 1)), kSlabs))
       return GS_ERR_CUDA;
     std::memcpy(p->wmaps[h], &m, sizeof(m));
+    if (!encode_tmap_slabs_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, (uint32_t)(16 * (h + 1)), kSlabs))
+      return GS_ERR_CUDA;
+    std::memcpy(p->wmaps_full[h], &m, sizeof(m));
   }
   p->wmaps_valid = true;
   return GS_OK;
@@ -518,9 +565,15 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, []() {
-    attr_err = cudaFuncSetAttribute(k_prefill, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    attr_err = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesSingle);
   });
   if (attr_err != cudaSuccess) return GS_ERR_CUDA;
+  // Up to 128 tokens a pair tile (256 tokens) would be half empty: each CTA
+  // then takes a 128-token tile of its own.
+  const bool pair = T > kBM;
+  const int64_t tile_m = pair ? kPairM : kBM;
   // Layers with no kept group produce zeros; the others share launches of up
   // to kMaxLayers, largest work per tile (kept groups per window) first, so
   // the last tiles the pairs pick up are the short ones.
@@ -553,14 +606,14 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
       const gs_packed* p = ps[i];
       PrefillLayer& L = P.L[k];
       if (!encode_tmap_slabs_bf16(&L.xmap, xs[i], (uint64_t)p->in, (uint64_t)T, kBM, kSlabs)) return GS_ERR_CUDA;
-      for (int h = 0; h < kNMaps; ++h) std::memcpy(&L.wmap[h], p->wmaps[h], sizeof(CUtensorMap));
+      for (int h = 0; h < kNMaps; ++h) std::memcpy(&L.wmap[h], pair ? p->wmaps[h] : p->wmaps_full[h], sizeof(CUtensorMap));
       L.win_off16 = p->win_off16;
       L.kmask16 = p->kmask16;
       L.y = static_cast<uint16_t*>(ys[i]);
       L.out = (int32_t)p->out;
       L.G = p->G;
       L.nw16 = p->nw16;
-      L.n_m = (int32_t)((T + kPairM - 1) / kPairM);
+      L.n_m = (int32_t)((T + tile_m - 1) / tile_m);
       L.n_w = (int32_t)((p->out + kFW - 1) / kFW);
       L.tile_begin = (int32_t)tiles;
       tiles += (int64_t)L.n_m * L.n_w;
@@ -570,10 +623,30 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
     P.T = (int32_t)T;
     P.n_tiles = (int32_t)tiles;
     P.err = err;
-    const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs (cluster dims 2)
-    k_prefill<<<grid, kThreads, kSmemBytes, s>>>(P);
+    cudaError_t e;
+    if (pair) {
+      const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs: clusters of two
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3((unsigned)grid);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = kSmemBytes;
+      cfg.stream = s;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      e = cudaLaunchKernelEx(&cfg, k_prefill<true>, P);
+    } else {
+      const int64_t max_ctas = sm_count();
+      const int grid = (int)(tiles < max_ctas ? tiles : max_ctas);
+      k_prefill<false><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
+      e = cudaGetLastError();
+    }
     note_launch();
-    if (cudaGetLastError() != cudaSuccess) return GS_ERR_CUDA;
+    if (e != cudaSuccess) return GS_ERR_CUDA;
   }
   return GS_OK;
 }
