@@ -103,9 +103,10 @@ gs_status gs_linear_ex(const void* x_dev, const gs_packed* p, int64_t T, void* y
  * gs_linear_batched - n independent layers, ys[i] = xs[i] W_hat_i^T for the
  * i-th handle, all with the same token count T.  In the decode regime all n
  * layers share one launch per 16 tokens (one grid streams every layer's kept
- * groups); in the prefill regime the layers run back to back.  Same per-layer
- * semantics and errors as gs_linear.  1 <= n <= 32 (n == 0 is a no-op); the
- * handles must be distinct.
+ * groups); in the prefill regime (T >= 33) up to 8 layers share one launch
+ * (one list of output tiles).  Results are those of gs_linear for each layer
+ * (prefill: bit for bit).  Same per-layer semantics and errors as gs_linear.
+ * 1 <= n <= 32 (n == 0 is a no-op); the handles must be distinct.
  */
 gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packed* const* ps,
                             int64_t T, void* const* ys_dev, void* stream);
