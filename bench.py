@@ -179,6 +179,7 @@ def oracle_sample_rate(layers, seconds: float, rows_per_call: int = 256):
     calls = 0
     i = 0
     t_end = time.perf_counter() + seconds
+    cpu0 = time.process_time()
     while time.perf_counter() < t_end or calls < len(layers):
         d = layers[i % len(layers)]
         L = d["L"]
@@ -193,15 +194,19 @@ def oracle_sample_rate(layers, seconds: float, rows_per_call: int = 256):
         i += 1
     sec_per_weight = t_used / done_weights
     tokens_per_s = 1.0 / (sec_per_weight * total_weights)
-    try:
-        from threadpoolctl import threadpool_info
-        cores = max((p.get("num_threads", 1) for p in threadpool_info()), default=1)
-    except Exception:
-        cores = os.cpu_count() or 1
-    return {"value": tokens_per_s, "unit": "tokens/s", "cores": int(cores), "kind": "oracle",
+    cores = _cores_used(time.process_time() - cpu0, t_used)
+    return {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
             "sample": f"{calls} oracle calls, each 1 token x {rows_per_call} output rows of one projection "
-                      f"(rotating over the 7), {t_used:.1f} s of CPU work; block tokens/s extrapolated by "
-                      f"weight count ({total_weights} weights per block)"}
+                      f"(rotating over the 7), {t_used:.1f} s wall; block tokens/s extrapolated by "
+                      f"weight count ({total_weights} weights per block); cores = process CPU time / wall "
+                      f"time over the calls"}
+
+
+def _cores_used(cpu_seconds: float, wall_seconds: float) -> int:
+    """Threads the oracle kept busy on average: process CPU time over wall time."""
+    if wall_seconds <= 0:
+        return 1
+    return max(1, int(round(cpu_seconds / wall_seconds)))
 
 
 # ----------------------------------------------------------------------------- reference arm
@@ -224,18 +229,21 @@ def run_reference(args):
     for i in range(args.warmup):
         one(i)
     t0 = time.perf_counter()
+    cpu0 = time.process_time()
     weights = 0
     for i in range(args.steps):
         weights += one(i)
     dt = time.perf_counter() - t0
+    cores = _cores_used(time.process_time() - cpu0, dt)
     tokens_per_s = weights / total_weights / dt
     sample = (f"each step: the fp64 oracle on 1 token x {rows_per_step} output rows of one projection "
-              f"(rotating over the 7); block tokens/s extrapolated by weight count")
+              f"(rotating over the 7); block tokens/s extrapolated by weight count; cores = process CPU time / "
+              f"wall time")
     line = {"impl": "reference", "metric": METRIC, "value": tokens_per_s, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / max(1, args.steps),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": "llama2-7b-block decode T=1 (sampled rows)", "layers": 7},
-            "cpu_baseline": {"value": tokens_per_s, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "cpu_baseline": {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": tokens_per_s, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
