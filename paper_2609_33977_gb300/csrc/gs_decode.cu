@@ -26,12 +26,13 @@
 // mma.sync A fragments from the slice, placing every kept row at its window
 // position (pruned rows stay zero), with the x chunk as the B fragment.  The
 // MMA row is the output row, so the fp32 accumulator stays in registers for
-// the whole unit: no scatter and no atomics on y.  At the unit's end the
-// odd-chunk warp hands its accumulator to the even-chunk warp through shared
-// memory, which adds it (a fixed order) and writes the result.
+// the whole unit: no scatter and no atomics on y.  At the unit's end one warp
+// of the pair hands its accumulator to the other through shared memory, which
+// adds it (one fp32 add per element) and writes the result; the writing role
+// alternates between the two warps from unit to unit.
 //
 // Reduction.  When a block's chunks are split over several units, the
-// even-chunk warp of each window writes its 16-row partial to the handle's
+// writing warp of each window writes its 16-row partial to the handle's
 // workspace and bumps the window's arrival counter; the last arriver adds the
 // partials in split order (so the result does not depend on arrival order),
 // writes y and resets the counter.
@@ -360,9 +361,9 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     asm volatile("griddepcontrol.wait;" ::: "memory");
     // Warp pair (win, win + kDW) owns the 16-row window win: the first warp
     // takes a unit's even chunks, the second its odd chunks, so two chunks are
-    // in the MMA pipeline per window.  At the unit's end the second warp hands
-    // its accumulator to the first through shared memory, which adds it (a
-    // fixed order) and writes the result.
+    // in the MMA pipeline per window.  At the unit's end one warp hands its
+    // accumulator to the other through shared memory (the taker alternates
+    // from unit to unit), which adds it and writes the result.
     const int win = warp & (kDW - 1), par = warp / kDW;
     const int g = lane >> 2, qd = lane & 3;
     const uint32_t lo_g = (1u << g) - 1u, lo_g8 = (1u << (g + 8)) - 1u;
@@ -438,9 +439,12 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[nt][i] += acc2[nt][i];
 
-      // ---- pair hand-off: the odd-chunk warp's accumulator joins the even one's
+      // ---- pair hand-off: one warp's accumulator joins the other's, which then
+      // writes the unit's result; the writing role alternates between the two
+      // warps from unit to unit, so the output path (and the split reduction's
+      // global round trips) is shared evenly
       const uint32_t hpar = (uint32_t)k & 1u;
-      if (par) {
+      if ((uint32_t)par != hpar) {
         if (!mbar_wait_bounded(&p_empty[win], hpar ^ 1u, abort_flag, P.err, kDecWaitLimitNs, kDevErrTimeout)) {
           ok = false;
           break;
