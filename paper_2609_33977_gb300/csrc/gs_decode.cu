@@ -122,6 +122,13 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
       : "memory");
 }
 
+// atomic add with acquire-release ordering at GPU scope; returns the old value
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int32_t* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -495,14 +502,18 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
             part[tok * kWin16 + g] = acc[nt][j];
             part[tok * kWin16 + g + 8] = acc[nt][2 + j];
           }
-        __threadfence();
+        // The lanes' partial stores are ordered before lane 0's counter update
+        // by the warp barrier; the update is an acquire-release RMW at GPU scope,
+        // so it publishes them (release is cumulative), and in the last arriver
+        // it acquires every other split's published partials, which the warp
+        // barrier after the broadcast extends to all lanes (their loads go to L2).
         __syncwarp();
         int last = 0;
         int32_t* cnt = L.cnt + U.blk * kDW + win;
-        if (lane == 0) last = (atomicAdd(cnt, 1) == L.nsplit - 1);
+        if (lane == 0) last = (atom_add_acq_rel_gpu(cnt, 1) == L.nsplit - 1);
         last = __shfl_sync(0xffffffffu, last, 0);
         if (last) {
-          __threadfence();
+          __syncwarp();
           const float* base_ws = L.ws + ((int64_t)U.blk * L.nsplit * kDW + win) * kPartFloats;
           const int Tl = T < NT * 8 ? T : NT * 8;
           for (int e = lane; e < Tl * kWin16; e += 32) {
