@@ -1,23 +1,30 @@
 // Prefill-regime group-sparse linear (many tokens, tensor-core bound):
 //   y[t, r] = sum over kept groups (r, c) of X_c[t, :] . W[r, 256c : 256c+256]   (Eq. 1)
 //
-// Tile = 128 tokens x 160 output rows (a "window").  For every chunk c the kept
-// rows of the window form one contiguous slice of the packed tiles (rows are
-// ascending inside a chunk), so the slice is a dense K-major operand that TMA
-// loads as-is.  Per chunk one tcgen05 MMA chain computes D[128 tok x n] =
-// X_c . W_slice^T (n <= 160 kept rows, rounded up to 16) into one of three
-// TMEM scratch buffers; the epilogue warps then add each window row's scratch
-// column (a zero column for rows pruned in chunk c) into the window
-// accumulator, which they hold in registers.  W (.) M
-// is never materialised and pruned groups cost neither bytes nor FLOPs.
+// Tiles.  A tile is a token range x 160 output rows (a "window").  For every
+// chunk c the kept rows of the window form one contiguous slice of the packed
+// tiles (rows are ascending inside a chunk), so the slice is a dense K-major
+// operand that TMA loads as-is.  Per chunk one tcgen05 MMA chain computes
+// D[tokens x n] = X_c . W_slice^T (n <= 160 kept rows, rounded up to 16) into
+// one of three TMEM scratch buffers; the epilogue warps then add each window
+// row's scratch column (a zero column for rows pruned in chunk c) into the
+// window accumulator, which they hold in registers.  W (.) M is never
+// materialised and pruned groups cost neither bytes nor FLOPs.
+//
+// Tile owners.  Normally a CTA pair (a cluster of two CTAs) owns a 256-token
+// tile: CTA r holds tokens 128r..128r+127 and half of each W slice, and the
+// leader's MMA thread issues M = 256 cta_group::2 MMAs whose D lands in both
+// CTAs' TMEM.  Up to 128 tokens (a pair tile would be half empty) each CTA
+// owns a 128-token tile, loads whole slices and issues its own M = 128 MMAs.
+// One launch walks the tiles of up to kMaxLayers layers that share T.
 //
 // Copies: a pipeline stage carries 128 of the chunk's 256 k as two 64-wide
 // slabs, fetched with one 3-D TMA box for X (128 rows x 2 slabs) and one for
-// the W slice (n rows x 2 slabs, from a descriptor whose box height is n).
+// the W slice (half or whole, from a descriptor with that box height).
 // TMA issue costs a fixed ~60-120 cycles per box whatever its size, so two
 // large boxes per stage keep the producer far below the copy time.
 //
-// Roles (one CTA per SM, persistent over tiles):
+// Roles (one CTA per SM, tile owners persistent over tiles):
 //   warp 0      TMA producer
 //   warp 1      TMEM allocator + single-thread MMA issuer
 //   warps 2..17 epilogue: warp (q, g) owns tokens 32q..32q+31 (its TMEM lane
