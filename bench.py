@@ -469,9 +469,11 @@ def run_ours(args):
     # ---- tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
     prefill = None
     prefill_sweep = None
+    decode_sweep = None
     if not args.no_prefill:
         prefill = measure_prefill(gs, torch, dev, stream, peaks)
         prefill_sweep = measure_prefill_sweep(gs, torch, dev, stream, peaks)
+        decode_sweep = measure_decode_sweep(gs, torch, dev, stream, peaks)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -505,6 +507,7 @@ def run_ours(args):
         "pack": {"seconds": pack_s, "layers": 7, "GB/s_incl_alloc_and_sync": pack_bytes / pack_s / 1e9},
         "prefill": prefill,
         "prefill_sweep": prefill_sweep,
+        "decode_sweep": decode_sweep,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -600,6 +603,48 @@ def measure_prefill_sweep(gs, torch, dev, stream, peaks):
                          "frac_of_attainable": tflops / attainable, "frac_of_tensor_peak": tflops / tpk})
             del xd, ys
         del ps
+        torch.cuda.empty_cache()
+    assert gs.device_status() == gs.GS_OK
+    return rows
+
+
+def measure_decode_sweep(gs, torch, dev, stream, peaks):
+    """Decode kernel on the first block of the 13B stack (T = 1, 16) and of the
+    Qwen stack (d = 0.5, T = 1): one batched launch per pass over the block's 7
+    projections, alternating between two packed copies (each larger than L2)."""
+    bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    rows = []
+    for cfg, d, Ts, name in ((4, 0.5, (1, 16), "llama2-13b block 0"),
+                             (5, 0.5, (1,), "qwen2.5-7b block 0, d=0.5")):
+        w = wl.workload(cfg, d, blocks=1)
+        k = wl.keep_counts(w)
+        Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
+        Md = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in range(7)]
+        copies = [[gs.pack(Wd[i], Md[i]) for i in range(7)] for _ in range(2)]
+        del Wd, Md
+        kept = sum(p.kept for p in copies[0])
+        for T in Ts:
+            xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
+            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
+            n = 50
+            with torch.cuda.stream(stream):
+                for i in range(4):
+                    gs.linear_batched_into(xd, copies[i % 2], ys, stream=stream)
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                for i in range(n):
+                    gs.linear_batched_into(xd, copies[i % 2], ys, stream=stream)
+                b.record(stream)
+                b.synchronize()
+            s_pass = a.elapsed_time(b) / 1e3 / n
+            nbytes = sum(512.0 * p.kept + 6.0 * (L.inp // 256) * ((L.out + 15) // 16) + 2.0 * T * (L.inp + L.out)
+                         for p, L in zip(copies[0], w.layers))
+            gbs = nbytes / s_pass / 1e9
+            rows.append({"workload": f"{name}, T={T}", "T": T, "kept_groups": kept, "us_per_block": s_pass * 1e6,
+                         "tokens/s": T / s_pass, "GB/s": gbs, "frac_of_measured_hbm": gbs / bw})
+            del xd, ys
+        del copies
         torch.cuda.empty_cache()
     assert gs.device_status() == gs.GS_OK
     return rows
