@@ -2,7 +2,7 @@
 //   y[t, r] = sum over kept groups (r, c) of sum_k x[t, 256c+k] W[r, 256c+k]   (Eq. 1)
 //
 // Work units.  A unit is (64-row block, range of chunks) of one layer: a
-// block's chunks are split into equal ranges of about 256 KB of kept weights
+// block's chunks are split into equal ranges of about 224 KB of kept weights
 // (a quarter of that when a launch has too few units to spread over the
 // CTAs).  Persistent CTA b starts on units b and
 // b + grid, then takes units from a shared ticket counter in list order
@@ -75,7 +75,7 @@ constexpr int kMaxCpu = 64;                   // chunks per unit
 constexpr int kMetaSlots = 2;
 constexpr int kDecSmemBytes = kRingBytes + kMetaSlots * kMaxCpu * 16 + 1024;
 constexpr int kPartFloats = kMaxT * kWin16;   // one warp's partial: 16 tokens x 16 rows
-constexpr int64_t kUnitBytes = 256 * 1024;    // target kept bytes per unit
+constexpr int64_t kUnitBytes = 224 * 1024;    // target kept bytes per unit
 // Ring allocation never waits forever: a chunk that does not fit before the
 // ring's end starts over at offset 0, which with every earlier chunk released
 // asks for (ring end - head) + need bytes; that stays within the ring for any
