@@ -17,17 +17,26 @@ float64 without rounding).  Each function follows one definition:
 * the packed layout (chunk-major kept-row lists, weight tiles, offsets), which
   the paper leaves unspecified; the layout is defined by the sequential loop in
   `pack` below.
+* selector export, Sec. 2.2 and App. F: with the Gumbel noise removed, a
+  selector logit l keeps its group when sigmoid(l) > 1/2; App. F applies the
+  same rule when the masks are exported, then reports each projection's
+  preserved rate (active / total weights), the Q/K/V rates averaged.
 
 Readings where the paper is silent (all listed in the design notes):
 * groups are 1 x 256 along the input dimension, aligned at multiples of 256;
 * M acts as a select, so a pruned weight is +0.0 (bit pattern 0x0000) even
   where W is negative;
-* a nonzero mask byte means "keep".
+* a nonzero mask byte means "keep";
+* the export threshold is 1/2 on sigmoid(l), strict (the paper names no
+  value): l = +0, l = -0 and NaN logits prune.
 
 Parity pins: every function here is pinned by the `-m "not gpu"` tests in
 tests/test_oracle_pins.py (exact integer cases, complement and disjoint-union
 identities, one-hot masks, permutation equivariance, hand-derived golden
-layouts, closed-form sparsities).
+layouts, closed-form sparsities; for the selector export: hand-derived
+threshold cases over the float32 special values, agreement with a library
+sigmoid at several temperatures, and the global preserved rate the paper
+prints for its LLaMA-2-7B allocation in Sec. 3.5).
 """
 from __future__ import annotations
 
@@ -219,3 +228,40 @@ def linear_packed(x_bits: np.ndarray, p: Packed) -> np.ndarray:
                     acc += xc[t, k] * tiles[j, k]
                 y[t, r] += acc
     return y
+
+
+# ---------------------------------------------------------------------------
+# Sec. 2.2 and App. F: selector export and preserved rates
+# ---------------------------------------------------------------------------
+
+def select_groups(logits: np.ndarray) -> np.ndarray:
+    """Evaluation-time selectors from float32 selector logits (Sec. 2.2; App. F).
+
+    The group is kept when sigmoid(l) > 1/2.  sigmoid is strictly increasing
+    with sigmoid(0) = 1/2, so that test is exactly l > 0 on the float32 value
+    (a float64 sigmoid would round to 1/2 for |l| below about 1e-16 and lose
+    the sign).  +0, -0 and NaN prune; +inf keeps.  Returns uint8 0/1 of the
+    logits' shape ([G_out, G_in] row-major for one layer).
+    """
+    lg = np.asarray(logits, dtype=np.float32).astype(np.float64)
+    B = np.zeros(lg.shape, dtype=np.uint8)
+    B[lg > 0.0] = 1
+    return B
+
+
+def kept_groups(B: np.ndarray) -> int:
+    """Number of retained groups, sum_uv B_uv (the numerator of Eq. 2)."""
+    return int((np.asarray(B) != 0).sum())
+
+
+def global_preserved_rate(Bs: Iterable[np.ndarray], shapes: Iterable[Tuple[int, int]]) -> float:
+    """Share of all target parameters kept: 1 - s with s from Eq. 2."""
+    return 1.0 - global_sparsity(Bs, shapes)
+
+
+def qkv_preserved_rate(B_q: np.ndarray, B_k: np.ndarray, B_v: np.ndarray,
+                       g_out: int = 1, g_in: int = G_IN) -> float:
+    """App. F: the Q, K and V projections are reported as the plain mean of their
+    three preserved rates."""
+    return (preserved_rate(B_q, g_out, g_in) + preserved_rate(B_k, g_out, g_in)
+            + preserved_rate(B_v, g_out, g_in)) / 3.0

@@ -17,7 +17,8 @@ are drawn at random and rescaled so the global kept-group count is exact.
 
 Seeding: every stream is a numpy PCG64 generator seeded with
 SeedSequence([cfg_id, variant, layer_id, stream_id, *extra]); stream ids are
-0 = W, 1 = per-layer ratios, 2 = group scores, 3 = x, 4 = outlier channels.
+0 = W, 1 = per-layer ratios, 2 = group scores, 3 = x, 4 = outlier channels,
+5 = selector logits.
 """
 from __future__ import annotations
 
@@ -29,7 +30,7 @@ import numpy as np
 
 GROUP_IN = 256          # g_in of the 1x256 group shape (Sec. 2.1)
 
-STREAM_W, STREAM_RATIOS, STREAM_SCORES, STREAM_X, STREAM_OUTLIERS = 0, 1, 2, 3, 4
+STREAM_W, STREAM_RATIOS, STREAM_SCORES, STREAM_X, STREAM_OUTLIERS, STREAM_LOGITS = 0, 1, 2, 3, 4, 5
 
 
 # --------------------------------------------------------------------------
@@ -275,6 +276,46 @@ def random_weight_bits(out: int, inp: int, seed: int, std: float = 0.02) -> np.n
 def random_activation_bits(T: int, inp: int, seed: int) -> np.ndarray:
     g = np.random.Generator(np.random.PCG64(np.random.SeedSequence([9003, seed])))
     return f32_to_bf16_bits(g.standard_normal((T, inp), dtype=np.float32))
+
+
+# --------------------------------------------------------------------------
+# selector logits (the float32 scores a trained mask generator exports)
+# --------------------------------------------------------------------------
+
+# float32 bit patterns placed among synthetic logits: +-0, the smallest
+# subnormals, the smallest normal, +-inf, quiet NaNs of both signs, +-max
+SPECIAL_LOGIT_BITS = (0x00000000, 0x80000000, 0x00000001, 0x80000001, 0x00800000,
+                      0x7F800000, 0xFF800000, 0x7FC00000, 0xFFC00000, 0x7F7FFFFF, 0xFF7FFFFF)
+
+
+def logit_mean(density: float) -> float:
+    """The mean mu of N(mu, 1) logits of which a fraction `density` is positive."""
+    from statistics import NormalDist
+    d = min(max(float(density), 1e-9), 1.0 - 1e-9)
+    return NormalDist().inv_cdf(d)
+
+
+def selector_logits(shape, density: float, seed: int, special_every: int = 0) -> np.ndarray:
+    """float32 logits ~ N(logit_mean(density), 1) of the given shape.  With
+    special_every = s > 0, about one entry in s (seeded positions) is replaced by
+    one of SPECIAL_LOGIT_BITS, cycling through the list."""
+    g = np.random.Generator(np.random.PCG64(np.random.SeedSequence([9004, STREAM_LOGITS, seed])))
+    lg = (g.standard_normal(shape, dtype=np.float32) + np.float32(logit_mean(density))).astype(np.float32)
+    if special_every > 0 and lg.size:
+        flat = lg.reshape(-1)
+        n = max(1, flat.size // special_every)
+        pos = g.choice(flat.size, size=min(n, flat.size), replace=False)
+        vals = np.array(SPECIAL_LOGIT_BITS, dtype=np.uint32).view(np.float32)
+        flat[pos] = vals[np.arange(pos.size) % vals.size]
+    return lg
+
+
+def selector_logits_device(n: int, density: float, seed: int, device="cuda"):
+    """`selector_logits` drawn on the device (torch Philox), no special values."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed_u64(9004, 0, 0, STREAM_LOGITS, seed))
+    return torch.randn((n,), generator=g, device=device, dtype=torch.float32) + logit_mean(density)
 
 
 # --------------------------------------------------------------------------

@@ -273,3 +273,68 @@ def test_bf16_rounding_helper():
     v = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, 1.0 + 2 ** -7, -2.5, 0.0], np.float32)
     assert wl.f32_to_bf16_bits(v).tolist() == [0x3F80, 0x3F80, 0x3F82, 0x3F81, 0xC020, 0x0000]
     assert np.array_equal(wl.bf16_bits_to_f32(np.array([0x3F80, 0xC020], np.uint16)), np.array([1.0, -2.5], np.float32))
+
+
+# --------------------------------------------------------------------- Sec. 2.2 / App. F: selector export
+
+def test_golden_selector_threshold():
+    g = json.loads((GOLDEN / "selector_threshold.json").read_text())
+    raw = np.array([int(h, 16) for h in g["logits_hex_f32"]], dtype=np.uint32).view(np.float32)
+    assert orc.select_groups(raw).tolist() == g["selector"]
+    assert orc.select_groups(raw).dtype == np.uint8
+
+
+@pytest.mark.parametrize("tau", [0.25, 1.0, 4.0])
+def test_selector_matches_sigmoid_away_from_zero(tau):
+    special = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(7)
+    lg = (rng.standard_normal((64, 37)) * 3.0).astype(np.float32)
+    lg[np.abs(lg) < 1e-6] = 1.0
+    # the noise-free Gumbel-Sigmoid relaxation at any temperature, thresholded at 1/2
+    ref = (special.expit(lg.astype(np.float64) / tau) > 0.5).astype(np.uint8)
+    assert np.array_equal(orc.select_groups(lg), ref)
+
+
+def test_selector_sign_symmetry_and_shape():
+    rng = np.random.default_rng(8)
+    lg = rng.standard_normal((5, 9)).astype(np.float32)
+    B = orc.select_groups(lg)
+    assert B.shape == (5, 9)
+    assert np.array_equal(orc.select_groups(-lg), 1 - B)          # no zeros among these logits
+    assert orc.kept_groups(B) == int(np.count_nonzero(lg > 0))
+
+
+def test_global_preserved_rate_reproduces_the_printed_allocation():
+    g = json.loads((GOLDEN / "llama2_7b_allocation.json").read_text())
+    Bs, shapes = [], []
+    for name, (d_out, d_in) in g["shapes"].items():
+        rate = g["attention_rate"] if name in ("q", "k", "v", "o") else g["mlp_rate"]
+        n = d_out * d_in // 256
+        B = np.zeros((d_out, d_in // 256), np.uint8)
+        B.reshape(-1)[: int(round(rate * n))] = 1
+        Bs.append(B)
+        shapes.append((d_out, d_in))
+    got = orc.global_preserved_rate(Bs, shapes)
+    tol = g["printed_rate_half_unit"] + g["global_half_unit"] + 1e-6
+    assert abs(got - g["global_preserved"]) <= tol
+    # an unweighted mean over the projections misses the printed figure by far
+    unweighted = float(np.mean([orc.preserved_rate(B) for B in Bs]))
+    assert abs(unweighted - g["global_preserved"]) > 10 * tol
+
+
+def test_global_preserved_rate_is_one_minus_golden_sparsity():
+    g = json.loads((GOLDEN / "global_sparsity.json").read_text())
+    Bs = [np.asarray(l["mask"]) for l in g["layers"]]
+    shapes = [(l["d_out"], l["d_in"]) for l in g["layers"]]
+    assert orc.global_preserved_rate(Bs, shapes) == 1.0 - g["s_global"]
+
+
+def test_qkv_rate_is_the_plain_mean():
+    # q keeps its only group, k keeps 2 of 8, v keeps none: (1 + 0.25 + 0) / 3
+    Bq = np.ones((1, 1), np.uint8)
+    Bk = np.zeros((4, 2), np.uint8)
+    Bk[0, 0] = Bk[3, 1] = 1
+    Bv = np.zeros((2, 1), np.uint8)
+    assert orc.qkv_preserved_rate(Bq, Bk, Bv) == pytest.approx(1.25 / 3, abs=1e-15)
+    # a parameter-weighted mean would give (256 + 512) / (256 + 2048 + 512)
+    assert abs(orc.qkv_preserved_rate(Bq, Bk, Bv) - 768 / 2816) > 0.1

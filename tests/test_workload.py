@@ -76,3 +76,15 @@ def test_outlier_channels():
     rest = np.abs(np.delete(x, ch, axis=1)).mean()
     assert 15 < big / rest < 25
     assert wl.outlier_channels(w, 6).size == 110   # down_proj: 1 % of 11008
+
+
+def test_selector_logits_density_and_specials():
+    lg = wl.selector_logits((400, 50), 0.3, seed=1)
+    assert lg.dtype == np.float32 and lg.shape == (400, 50)
+    assert abs(float((lg > 0).mean()) - 0.3) < 0.01
+    assert np.array_equal(lg, wl.selector_logits((400, 50), 0.3, seed=1))       # seeded
+    sp = wl.selector_logits((400, 50), 0.7, seed=2, special_every=50)
+    bits = sp.view(np.uint32).reshape(-1)
+    present = set(int(b) for b in bits) & set(wl.SPECIAL_LOGIT_BITS)
+    assert present == set(wl.SPECIAL_LOGIT_BITS)
+    assert np.isnan(sp).sum() >= 2
