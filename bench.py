@@ -475,6 +475,12 @@ def run_ours(args):
         prefill_sweep = measure_prefill_sweep(gs, torch, dev, stream, peaks)
         decode_sweep = measure_decode_sweep(gs, torch, dev, stream, peaks)
 
+    # ---- selector export (the step that produces the masks), measured last
+    try:
+        mask_export = measure_select(gs, torch, dev, stream, peaks)
+    except Exception as e:   # reported in the line, never hidden
+        mask_export = {"error": f"{type(e).__name__}: {e}"}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample_rate(layers, args.cpu_seconds)
@@ -508,6 +514,7 @@ def run_ours(args):
         "prefill": prefill,
         "prefill_sweep": prefill_sweep,
         "decode_sweep": decode_sweep,
+        "mask_export": mask_export,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -648,6 +655,37 @@ def measure_decode_sweep(gs, torch, dev, stream, peaks):
         torch.cuda.empty_cache()
     assert gs.device_status() == gs.GS_OK
     return rows
+
+
+def measure_select(gs, torch, dev, stream, peaks):
+    """Selector export (gs_select_groups) over all selectors of the 13B stack (40
+    blocks, 49,561,600 groups): float32 logits (198 MB) in, uint8 masks (50 MB) out,
+    together larger than L2.  Algorithmic bytes: 4 read + 1 written per selector."""
+    bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    w = wl.workload(4, 0.5)
+    n = w.total_groups
+    lg = wl.selector_logits_device(n, 0.5, seed=1, device=dev)
+    mask = torch.empty((n,), dtype=torch.uint8, device=dev)
+    kept = torch.empty((1,), dtype=torch.int64, device=dev)
+    reps = 50
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            gs.select_groups(lg, mask, kept, stream=stream)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            gs.select_groups(lg, mask, kept, stream=stream)
+        b.record(stream)
+        b.synchronize()
+    s_launch = a.elapsed_time(b) / 1e3 / reps
+    k = int(kept.cpu()[0])
+    del lg, mask, kept
+    torch.cuda.empty_cache()
+    gbs = 5.0 * n / s_launch / 1e9
+    return {"workload": "selectors of the llama2-13b stack (40 blocks), logits ~ N(0, 1)", "kernel": "k_select",
+            "selectors": n, "kept": k, "bytes_per_launch": 5 * n, "us_per_launch": s_launch * 1e6, "GB/s": gbs,
+            "frac_of_measured_hbm": gbs / bw}
 
 
 def run_layer(args):

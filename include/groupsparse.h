@@ -112,6 +112,31 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
                             int64_t T, void* const* ys_dev, void* stream);
 
 /*
+ * gs_select_groups - selector export (Sec. 2.2: at evaluation the Gumbel noise
+ * is dropped and the selectors are thresholded; App. F: the exported masks use
+ * the same rule).  B[i] = 1 when sigmoid(logits[i]) > 1/2, i.e. exactly when
+ * logits[i] > 0: +0, -0 and NaN prune, +inf keeps.  Also counts the kept
+ * groups, sum_uv B_uv of Eq. 2, from which the caller forms the preserved
+ * rates (kept / (G_out G_in) per layer, since every group holds g_out g_in
+ * weights).
+ *
+ * logits_dev  float32 [n], device, caller-owned, 16-byte aligned, read only.
+ *             For one layer with 1x256 groups: [out][in/256] row-major.
+ * n           number of selectors, 0 <= n < 2^36.
+ * mask_dev    uint8 [n], device, caller-owned, 16-byte aligned, fully
+ *             overwritten with 0 / 1: the mask layout gs_pack takes.  Must not
+ *             overlap logits_dev.
+ * kept_dev    int64, device, 8-byte aligned, overwritten with the number of
+ *             ones written; may be NULL.
+ * Results are exact (integer test on the float32 bit pattern).  n == 0
+ * writes kept = 0 and launches no kernel.  Asynchronous on `stream`.
+ * Errors: INVALID_ARG (n out of range, NULL or misaligned pointers, overlap),
+ * CUDA.
+ */
+gs_status gs_select_groups(const float* logits_dev, int64_t n, uint8_t* mask_dev, int64_t* kept_dev,
+                           void* stream);
+
+/*
  * gs_unpack - the check path: W_hat_dev[r][k] = W[r][k] where the group of
  * (r, k) is kept, +0.0 (0x0000) where it is pruned (M of Eq. 1 as a select).
  * W_hat_dev  bf16 [out][in], caller-owned, fully overwritten.

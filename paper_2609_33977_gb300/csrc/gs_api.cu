@@ -234,6 +234,18 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
   return GS_OK;
 }
 
+gs_status gs_select_groups(const float* logits_dev, int64_t n, uint8_t* mask_dev, int64_t* kept_dev,
+                           void* stream) {
+  if (n < 0 || n >= (int64_t(1) << 36)) return GS_ERR_INVALID_ARG;
+  if (kept_dev && (reinterpret_cast<uintptr_t>(kept_dev) & 7u) != 0) return GS_ERR_INVALID_ARG;
+  if (n > 0) {
+    if (!logits_dev || !mask_dev || !aligned16(logits_dev) || !aligned16(mask_dev)) return GS_ERR_INVALID_ARG;
+    const uintptr_t l0 = reinterpret_cast<uintptr_t>(logits_dev), m0 = reinterpret_cast<uintptr_t>(mask_dev);
+    if (l0 < m0 + (uintptr_t)n && m0 < l0 + 4 * (uintptr_t)n) return GS_ERR_INVALID_ARG;   // overlap
+  }
+  return launch_select(logits_dev, n, mask_dev, kept_dev, static_cast<cudaStream_t>(stream));
+}
+
 gs_status gs_unpack(const gs_packed* p, void* W_hat_dev, void* stream) {
   if (check_handle(p) != GS_OK || !W_hat_dev || !aligned16(W_hat_dev)) return GS_ERR_INVALID_ARG;
   return launch_unpack(p, W_hat_dev, static_cast<cudaStream_t>(stream));

@@ -68,6 +68,9 @@ gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t
 gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s);
 gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
 
+// select.cu
+gs_status launch_select(const float* logits, int64_t n, uint8_t* mask, int64_t* kept, cudaStream_t s);
+
 // decode.cu
 gs_status decode_prepare(gs_packed* p, cudaStream_t s);   // allocates + builds the decode metadata
 void decode_release(gs_packed* p);

@@ -35,6 +35,7 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib.gs_linear_ex.argtypes = [vp, vp, i64, vp, vp, ctypes.c_int]
     lib.gs_linear_batched.argtypes = [i32, ctypes.POINTER(vp), ctypes.POINTER(vp), i64, ctypes.POINTER(vp), vp]
     lib.gs_unpack.argtypes = [vp, vp, vp]
+    lib.gs_select_groups.argtypes = [vp, i64, vp, vp, vp]
     lib.gs_packed_info.argtypes = [vp, _c_i64p, _c_i64p, _c_i64p, ctypes.POINTER(ctypes.c_size_t)]
     lib.gs_packed_export.argtypes = [vp, _c_i64p, _c_i32p, _c_u16p, _c_i32p, _c_u16p]
     lib.gs_free.argtypes = [vp]
@@ -45,7 +46,7 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib.gs_launch_count.argtypes = []
     lib.gs_launch_count.restype = ctypes.c_int64
     for fn in (lib.gs_pack, lib.gs_linear, lib.gs_linear_ex, lib.gs_linear_batched, lib.gs_unpack,
-               lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status):
+               lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status, lib.gs_select_groups):
         fn.restype = ctypes.c_int
     return lib
 
@@ -191,6 +192,74 @@ def unpack(p: Packed, stream: Optional[torch.cuda.Stream] = None) -> torch.Tenso
     W = torch.empty((p.out, p.inp), dtype=torch.bfloat16, device="cuda")
     _check(lib.gs_unpack(p.handle, W.data_ptr(), _stream_ptr(stream)), "gs_unpack")
     return W
+
+
+def select_groups(logits: torch.Tensor, mask: Optional[torch.Tensor] = None,
+                  kept: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None):
+    """Selector export (Sec. 2.2; App. F): mask = [sigmoid(logits) > 1/2] as uint8 0/1 of
+    the logits' shape, and kept = the number of ones as an int64 [1] device tensor.
+    For one layer with 1x256 groups, logits are float32 [out, in/256]."""
+    _require_cuda(logits, torch.float32, "logits")
+    if mask is None:
+        mask = torch.empty(logits.shape, dtype=torch.uint8, device=logits.device)
+    else:
+        _require_cuda(mask, torch.uint8, "mask")
+        if mask.numel() != logits.numel():
+            raise ValueError("mask must hold one byte per logit")
+    if kept is None:
+        kept = torch.empty((1,), dtype=torch.int64, device=logits.device)
+    else:
+        _require_cuda(kept, torch.int64, "kept")
+        if kept.numel() < 1:
+            raise ValueError("kept must hold at least one int64")
+    _check(lib.gs_select_groups(logits.data_ptr(), logits.numel(), mask.data_ptr(), kept.data_ptr(),
+                                _stream_ptr(stream)), "gs_select_groups")
+    return mask, kept
+
+
+def pack_from_logits(W: torch.Tensor, logits: torch.Tensor,
+                     stream: Optional[torch.cuda.Stream] = None) -> Packed:
+    """Export a layer's selectors from its float32 logits [out, in/256] and pack W with them."""
+    mask, _ = select_groups(logits, stream=stream)
+    return pack(W, mask, stream)
+
+
+_QKV = {"q": "q", "k": "k", "v": "v", "q_proj": "q", "k_proj": "k", "v_proj": "v"}
+
+
+def preserved_report(kept: Sequence[int], shapes: Sequence[Sequence[int]],
+                     names: Optional[Sequence[str]] = None, group: int = 256) -> dict:
+    """Preserved rates of exported masks (App. F) from per-layer kept-group counts.
+
+    Each layer's rate is its active weights over its total weights, kept * group /
+    (d_out d_in); the global rate is 1 - s of Eq. 2 (all active weights over all
+    target weights).  With names, layers whose last dotted component is q, k and v
+    (or q_proj, k_proj, v_proj) under one prefix are also reported as the plain mean
+    of their three rates, keyed by that prefix."""
+    if len(kept) != len(shapes) or (names is not None and len(names) != len(kept)):
+        raise ValueError("kept, shapes (and names) must have the same length")
+    names = list(names) if names is not None else [str(i) for i in range(len(kept))]
+    rates = {}
+    active = total = 0
+    for n, k, (d_out, d_in) in zip(names, kept, shapes):
+        k, size = int(k), int(d_out) * int(d_in)
+        if k < 0 or k * group > size:
+            raise ValueError(f"{n}: {k} kept groups do not fit a {d_out} x {d_in} layer")
+        rates[n] = k * group / size
+        active += k * group
+        total += size
+    qkv = {}
+    for n in names:
+        prefix, _, last = n.rpartition(".")
+        if _QKV.get(last) == "q":
+            trio = {}
+            for m in names:
+                p2, _, l2 = m.rpartition(".")
+                if p2 == prefix and l2 in _QKV:
+                    trio[_QKV[l2]] = rates[m]
+            if len(trio) == 3:
+                qkv[prefix] = (trio["q"] + trio["k"] + trio["v"]) / 3.0
+    return {"layers": rates, "global": active / total if total else 0.0, "qkv": qkv}
 
 
 def device_status(stream: Optional[torch.cuda.Stream] = None) -> int:

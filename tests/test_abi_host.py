@@ -50,6 +50,7 @@ def test_host_side_validation(lib):
     lib.gs_linear_batched.argtypes = [i32, vp, vp, i64, vp, vp]
     lib.gs_packed_info.argtypes = [vp, vp, vp, vp, vp]
     lib.gs_packed_export.argtypes = [vp, vp, vp, vp, vp, vp]
+    lib.gs_select_groups.argtypes = [vp, i64, vp, vp, vp]
     lib.gs_free.argtypes = [vp]
     lib.gs_free.restype = None
     h = vp(12345)
@@ -71,4 +72,13 @@ def test_host_side_validation(lib):
     assert lib.gs_linear_batched(0, None, None, 1, None, None) == 0
     assert lib.gs_packed_info(None, None, None, None, None) == INVALID
     assert lib.gs_packed_export(None, None, None, None, None, None) == INVALID
+    assert lib.gs_select_groups(fake, -1, fake + 0x1000, None, None) == INVALID
+    assert lib.gs_select_groups(fake, 1 << 36, fake + 0x1000, None, None) == INVALID
+    assert lib.gs_select_groups(None, 8, fake, None, None) == INVALID
+    assert lib.gs_select_groups(fake, 8, None, None, None) == INVALID
+    assert lib.gs_select_groups(fake + 4, 8, fake + 0x1000, None, None) == INVALID   # misaligned logits
+    assert lib.gs_select_groups(fake, 8, fake + 0x1008, None, None) == INVALID       # misaligned mask
+    assert lib.gs_select_groups(fake, 8, fake + 0x1000, fake + 4, None) == INVALID   # misaligned count
+    assert lib.gs_select_groups(fake, 8, fake + 16, None, None) == INVALID           # mask overlaps logits
+    assert lib.gs_select_groups(None, 0, None, None, None) == 0                      # empty: nothing to do
     lib.gs_free(None)
