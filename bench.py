@@ -688,6 +688,20 @@ def measure_select(gs, torch, dev, stream, peaks):
             "frac_of_measured_hbm": gbs / bw}
 
 
+def run_mask_export(args):
+    """The selector export measurement alone; prints one JSON line."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+    peaks, _ = load_peaks()
+    stream = torch.cuda.Stream()
+    rec = measure_select(gs, torch, torch.device("cuda", 0), stream, peaks)
+    assert gs.device_status() == gs.GS_OK
+    print(json.dumps(rec), flush=True)
+    return 0
+
+
 def run_layer(args):
     """One synthetic layer (random mask of the given density), one kernel family,
     timed with CUDA events; prints one JSON line.  Used for sweeps and for the
@@ -781,6 +795,8 @@ def main():
     ap.add_argument("--tokens", type=int, default=16)
     ap.add_argument("--density", type=float, default=0.5)
     ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
+    ap.add_argument("--mask-export", action="store_true",
+                    help="time only the selector export kernel over the 13B stack's selectors")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -788,6 +804,8 @@ def main():
         return run_reference(args)
     if args.layer:
         return run_layer(args)
+    if args.mask_export:
+        return run_mask_export(args)
     return run_ours(args)
 
 
