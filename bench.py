@@ -616,23 +616,28 @@ def measure_prefill_sweep(gs, torch, dev, stream, peaks):
 
 
 def measure_decode_sweep(gs, torch, dev, stream, peaks):
-    """Decode kernel on the first block of the 13B stack (T = 1, 16) and of the
-    Qwen stack (d = 0.5, T = 1): one batched launch per pass over the block's 7
-    projections, alternating between two packed copies (each larger than L2)."""
+    """Decode kernel on the first block of the 13B stack (T = 1, 16), of the Qwen
+    stack (d = 0.5, T = 1), and on block 25 of the 7B stack under the paper-shaped
+    allocation (Q/K near 8 %, down above 53 %; T = 1): one batched launch per pass
+    over the block's 7 projections, alternating between two packed copies (each
+    larger than L2)."""
     bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
     rows = []
-    for cfg, d, Ts, name in ((4, 0.5, (1, 16), "llama2-13b block 0"),
-                             (5, 0.5, (1,), "qwen2.5-7b block 0, d=0.5")):
-        w = wl.workload(cfg, d, blocks=1)
+    for w, blk, Ts, name in ((wl.workload(4, 0.5, blocks=1), 0, (1, 16), "llama2-13b block 0"),
+                             (wl.workload(5, 0.5, blocks=1), 0, (1,), "qwen2.5-7b block 0, d=0.5"),
+                             (wl.workload(3, allocation="paper"), 25, (1,),
+                              "llama2-7b block 25, paper-shaped allocation")):
         k = wl.keep_counts(w)
-        Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
-        Md = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in range(7)]
-        copies = [[gs.pack(Wd[i], Md[i]) for i in range(7)] for _ in range(2)]
+        ids = list(range(7 * blk, 7 * blk + 7))
+        Wd = [wl.weight_device(w, i, device=dev) for i in ids]
+        Md = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in ids]
+        copies = [[gs.pack(Wd[j], Md[j]) for j in range(7)] for _ in range(2)]
         del Wd, Md
         kept = sum(p.kept for p in copies[0])
+        layers = [w.layers[i] for i in ids]
         for T in Ts:
-            xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
-            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
+            xd = [wl.activation_device(w, i, T, device=dev) for i in ids]
+            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in layers]
             n = 50
             with torch.cuda.stream(stream):
                 for i in range(4):
@@ -646,7 +651,7 @@ def measure_decode_sweep(gs, torch, dev, stream, peaks):
                 b.synchronize()
             s_pass = a.elapsed_time(b) / 1e3 / n
             nbytes = sum(512.0 * p.kept + 6.0 * (L.inp // 256) * ((L.out + 15) // 16) + 2.0 * T * (L.inp + L.out)
-                         for p, L in zip(copies[0], w.layers))
+                         for p, L in zip(copies[0], layers))
             gbs = nbytes / s_pass / 1e9
             rows.append({"workload": f"{name}, T={T}", "T": T, "kept_groups": kept, "us_per_block": s_pass * 1e6,
                          "tokens/s": T / s_pass, "GB/s": gbs, "frac_of_measured_hbm": gbs / bw})

@@ -113,6 +113,7 @@ class Workload:
     tokens: Tuple[int, ...]
     outlier_frac: float = 0.0           # fraction of input channels scaled x20
     variant: int = 0
+    allocation: str = "random"          # "random": U[a, b] ratios; "paper": paper_shaped_ratios
 
     @property
     def total_groups(self) -> int:
@@ -127,7 +128,8 @@ def _stack(block, nblocks: int) -> Tuple[Layer, ...]:
     return tuple(Layer(f"blk{b}.{n}", o, i) for b in range(nblocks) for (n, o, i) in block)
 
 
-def workload(cfg_id: int, density: float = 0.5, blocks: Optional[int] = None) -> Workload:
+def workload(cfg_id: int, density: float = 0.5, blocks: Optional[int] = None,
+             allocation: str = "random") -> Workload:
     """The five seeded workloads.
 
     1: one 1024x1024 layer, exactly half its 4096 groups kept, T = 8.
@@ -140,7 +142,17 @@ def workload(cfg_id: int, density: float = 0.5, blocks: Optional[int] = None) ->
     5: 28 Qwen2.5-7B blocks, global density d in {0.3, 0.5, 0.7} with per-layer
        U[d-0.2, d+0.2] rescaled to d, T in {1, 1024}.
     `blocks` truncates a stack to its first blocks (same seeds per layer index).
+    allocation="paper" (workload 3 only) replaces the random ratios by
+    paper_shaped_ratios, with their own seeds (variant 1).
     """
+    if allocation not in ("random", "paper"):
+        raise ValueError(f"unknown allocation {allocation!r}")
+    if allocation == "paper":
+        if cfg_id != 3:
+            raise ValueError("the paper-shaped allocation is defined for the LLaMA-2-7B stack (workload 3)")
+        n = 32 if blocks is None else blocks
+        return Workload(3, f"llama2-7b-stack{n}-paper-alloc", _stack(LLAMA2_7B_BLOCK, n), 0.5, None, (1, 16, 2048),
+                        outlier_frac=0.01, variant=1, allocation="paper")
     if cfg_id == 1:
         return Workload(1, "single-1024x1024", (Layer("linear", 1024, 1024),), 0.5, None, (8,))
     if cfg_id == 2:
@@ -211,9 +223,41 @@ def allocate_keep_counts(groups: Sequence[int], ratios: Sequence[float], budget:
     return k
 
 
+def paper_shaped_ratios(nblocks: int = 32) -> np.ndarray:
+    """Per-projection keep ratios [nblocks * 7] (q, k, v, o, gate, up, down per block)
+    shaped after the learned LLaMA-2-7B allocation the paper describes in Sec. 3.5
+    (only aggregate statistics are printed; the per-layer values are a figure):
+    attention about 36.6 % and MLP about 56.6 % of their parameters, the down
+    projection about 30.5 % of all preserved parameters, Q and K equal, V about 2.2x
+    Q, O the largest attention projection, attention comparable to MLP in blocks
+    3-17, and Q/K near 8 % with down above 53 % in blocks 22-31.  The depth profile
+    is defined on 32 blocks; a shorter stack takes its first blocks.
+    """
+    q = np.empty(32)
+    for b in range(32):
+        if b < 3:
+            q[b] = 0.20
+        elif b <= 17:
+            q[b] = 0.30
+        elif b <= 21:
+            q[b] = 0.25 - 0.05 * (b - 18)
+        else:
+            q[b] = 0.08
+    v = 2.2 * q
+    o = v + 0.14
+    gate = np.full(32, 0.50)
+    down = np.where(np.arange(32) >= 22, 0.81, 0.63)
+    R = np.stack([q, q, v, o, gate, gate, down], axis=1)
+    if not 1 <= nblocks <= 32:
+        raise ValueError("the paper-shaped profile covers 1..32 blocks")
+    return R[:nblocks].reshape(-1)
+
+
 def keep_counts(wl: Workload) -> np.ndarray:
     """Per-layer kept-group counts of a workload (exact global budget)."""
-    if wl.ratio_range is None:
+    if wl.allocation == "paper":
+        ratios = paper_shaped_ratios(len(wl.layers) // 7)
+    elif wl.ratio_range is None:
         ratios = np.full(len(wl.layers), wl.density)
     else:
         a, b = wl.ratio_range

@@ -228,7 +228,7 @@ _stack_cache = {}
 
 
 def stack_layer(gs, w, k, i):
-    key = (w.cfg_id, w.density, i)
+    key = (w.cfg_id, w.variant, w.density, i)
     if key not in _stack_cache:
         _stack_cache.clear()                  # one layer resident at a time (the stacks are GBs)
         Wb = wl.weight_bits(w, i)
@@ -262,6 +262,32 @@ def test_stack_shapes_sampled(gs, cfg, d, Ts):
                 assert_within_bound(y, xb, Wb, B, tokens=None if T <= 16 else sample_tokens(T, seed=i),
                                     what=f"cfg{cfg} d={d} {w.layers[i].name} T={T}")
     _stack_cache.clear()
+    assert gs.device_status() == gs.GS_OK
+
+
+def test_paper_allocation_blocks_batched(gs):
+    """The paper-shaped allocation of the full 7B stack (Sec. 3.5 statistics): all
+    seven projections of block 0 and of block 25 (Q/K near 8 %, down above 53 %) in
+    one batched call per token count: T = 1 and 16 (decode, every token) and
+    T = 2048 (prefill, token sample)."""
+    import torch
+    w = wl.workload(3, allocation="paper")
+    k = wl.keep_counts(w)
+    for b in (0, 25):
+        ids = list(range(7 * b, 7 * b + 7))
+        host = [(wl.weight_bits(w, i), wl.group_mask(w, i, int(k[i]))) for i in ids]
+        ps = [packed(gs, Wb, B) for Wb, B in host]
+        assert [p.kept for p in ps] == [int(k[i]) for i in ids]
+        for T in (1, 16, 2048):
+            xbs = [wl.activation_bits(w, i, T) for i in ids]
+            ys = [torch.empty((T, w.layers[i].out), dtype=torch.bfloat16, device="cuda") for i in ids]
+            gs.linear_batched_into([to_dev(xb) for xb in xbs], ps, ys)
+            for j, i in enumerate(ids):
+                Wb, B = host[j]
+                assert_within_bound(to_bits(ys[j]), xbs[j], Wb, B,
+                                    tokens=None if T <= 16 else sample_tokens(T, seed=i),
+                                    what=f"paper allocation {w.layers[i].name} T={T}")
+        del ps
     assert gs.device_status() == gs.GS_OK
 
 

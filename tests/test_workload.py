@@ -88,3 +88,28 @@ def test_selector_logits_density_and_specials():
     present = set(int(b) for b in bits) & set(wl.SPECIAL_LOGIT_BITS)
     assert present == set(wl.SPECIAL_LOGIT_BITS)
     assert np.isnan(sp).sum() >= 2
+
+
+def test_paper_shaped_allocation_matches_printed_statistics():
+    # Sec. 3.5 (LLaMA-2-7B, 50 % sparsity): attention 36.6 %, MLP 56.6 %, down 30.5 % of all
+    # preserved parameters, Q/K about 8 % of groups and down above 53 % in blocks 22-31
+    w = wl.workload(3, allocation="paper")
+    k = wl.keep_counts(w).reshape(32, 7)
+    N = np.array([L.groups for L in w.layers[:7]])
+    assert int(k.sum()) == w.budget == w.total_groups // 2
+    rate = k / N
+    attn = k[:, :4].sum() / (N[:4].sum() * 32)
+    mlp = k[:, 4:].sum() / (N[4:].sum() * 32)
+    assert abs(attn - 0.366) < 0.005 and abs(mlp - 0.566) < 0.005
+    assert abs(k[:, 6].sum() / k.sum() - 0.305) < 0.005
+    assert np.all(np.abs(rate[22:, 0] - 0.08) < 0.01) and np.all(rate[22:, 6] > 0.53)
+    assert np.all(np.abs(rate[:, 0] - rate[:, 1]) < 0.05) and np.all(np.abs(rate[:, 4] - rate[:, 5]) < 0.05)
+    assert abs(rate[:, 2].sum() / rate[:, 0].sum() - 2.2) < 0.1
+    assert np.all(rate[:, 3] >= rate[:, :3].max(axis=1))
+    mid = slice(3, 18)
+    assert abs(k[mid, :4].sum() / (N[:4].sum() * 15) - k[mid, 4:].sum() / (N[4:].sum() * 15)) < 0.1
+    # masks of the variant differ from the random-allocation stack's, and are reproducible
+    m = wl.group_mask(w, 0, int(k[0, 0]))
+    assert int(m.sum()) == int(k[0, 0]) and np.array_equal(m, wl.group_mask(w, 0, int(k[0, 0])))
+    with pytest.raises(ValueError):
+        wl.workload(4, allocation="paper")
