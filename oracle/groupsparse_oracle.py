@@ -17,6 +17,10 @@ float64 without rounding).  Each function follows one definition:
 * the packed layout (chunk-major kept-row lists, weight tiles, offsets), which
   the paper leaves unspecified; the layout is defined by the sequential loop in
   `pack` below.
+* other group shapes, Sec. 2.1 with g_out x g_in groups (1x128 and the square
+  16..128 shapes of the Sec. 3.5 ablation and App. E): `linear` takes the
+  shape, and `pack_groups` / `unpack_groups` / `linear_packed_groups` define a
+  column-major block layout that reduces to `pack`'s for 1x256;
 * selector export, Sec. 2.2 and App. F: with the Gumbel noise removed, a
   selector logit l keeps its group when sigmoid(l) > 1/2; App. F applies the
   same rule when the masks are exported, then reports each projection's
@@ -36,7 +40,10 @@ identities, one-hot masks, permutation equivariance, hand-derived golden
 layouts, closed-form sparsities; for the selector export: hand-derived
 threshold cases over the float32 special values, agreement with a library
 sigmoid at several temperatures, and the global preserved rate the paper
-prints for its LLaMA-2-7B allocation in Sec. 3.5).
+prints for its LLaMA-2-7B allocation in Sec. 3.5; for other group shapes:
+cell-by-cell one-hot orientation, brute force over every 16x16 mask of a
+32x32 weight against int64 loops, reduction of square and 1x128 masks to row
+masks, and the 1x256 layout identity).
 """
 from __future__ import annotations
 
@@ -84,14 +91,16 @@ def masked_weight_bits(W_bits: np.ndarray, B: np.ndarray, g_out: int = 1, g_in: 
 # the layer: y = x W_hat^T
 # ---------------------------------------------------------------------------
 
-def linear(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray) -> Tuple[np.ndarray, np.ndarray]:
+def linear(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray, g_out: int = 1,
+           g_in: int = G_IN) -> Tuple[np.ndarray, np.ndarray]:
     """y[t, r] = sum_k x[t, k] W_hat[r, k] in float64, and the magnitude sum
     A[t, r] = sum_k |x[t, k] W_hat[r, k]| that scales the acceptance bound.
 
-    x_bits: uint16 [T, in] bf16 bits; W_bits: uint16 [out, in]; B: [out, in/256].
+    x_bits: uint16 [T, in] bf16 bits; W_bits: uint16 [out, in];
+    B: [out/g_out, in/g_in] (default 1x256 groups: [out, in/256]).
     """
     x = _bf16_to_f64(x_bits)
-    What = masked_weight(W_bits, B)
+    What = masked_weight(W_bits, B, g_out, g_in)
     if x.ndim != 2 or x.shape[1] != What.shape[1]:
         raise ValueError("x must be [T, in]")
     y = x @ What.T
@@ -100,10 +109,10 @@ def linear(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray) -> Tuple[np.nd
 
 
 def linear_tokens(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray,
-                  tokens: Sequence[int]) -> Tuple[np.ndarray, np.ndarray]:
+                  tokens: Sequence[int], g_out: int = 1, g_in: int = G_IN) -> Tuple[np.ndarray, np.ndarray]:
     """`linear` restricted to the listed token rows of x."""
     idx = np.asarray(list(tokens), dtype=np.int64)
-    return linear(np.asarray(x_bits)[idx], W_bits, B)
+    return linear(np.asarray(x_bits)[idx], W_bits, B, g_out, g_in)
 
 
 # ---------------------------------------------------------------------------
@@ -265,3 +274,86 @@ def qkv_preserved_rate(B_q: np.ndarray, B_k: np.ndarray, B_v: np.ndarray,
     three preserved rates."""
     return (preserved_rate(B_q, g_out, g_in) + preserved_rate(B_k, g_out, g_in)
             + preserved_rate(B_v, g_out, g_in)) / 3.0
+
+
+# ---------------------------------------------------------------------------
+# other group shapes: Sec. 2.1 with general g_out x g_in groups; the shapes the
+# paper evaluates (Sec. 3.5 ablation, App. E)
+# ---------------------------------------------------------------------------
+
+GROUP_SHAPES = ((1, 128), (1, 256), (16, 16), (32, 32), (64, 64), (128, 128))
+
+
+def group_grid(out: int, inp: int, g_out: int, g_in: int) -> Tuple[int, int]:
+    """(G_out, G_in) = (d_out / g_out, d_in / g_in); the groups tile W exactly."""
+    if g_out <= 0 or g_in <= 0 or out % g_out or inp % g_in:
+        raise ValueError(f"a {out} x {inp} weight is not tiled by {g_out} x {g_in} groups")
+    return out // g_out, inp // g_in
+
+
+@dataclasses.dataclass
+class PackedGroups:
+    out: int
+    inp: int
+    g_out: int
+    g_in: int
+    offsets: np.ndarray     # int64 [G_in+1]; group column v owns packed groups [offsets[v], offsets[v+1])
+    block_row: np.ndarray   # int32 [K]; ascending kept group rows u of each group column
+    tiles: np.ndarray       # uint16 [K, g_out, g_in]; tiles[j] = W[g_out u : g_out (u+1), g_in v : g_in (v+1)]
+
+    @property
+    def kept(self) -> int:
+        return int(self.offsets[-1])
+
+
+def pack_groups(W_bits: np.ndarray, B: np.ndarray, g_out: int, g_in: int) -> PackedGroups:
+    """Column-major packing for any group shape: for group column v = 0..G_in-1, for
+    group row u = 0..G_out-1 in ascending order, if B[u, v] keeps the group, append u
+    and the g_out x g_in block of W it covers (bit copy).  With g_out = 1 this is the
+    chunk-major layout of `pack` (block_row = row_idx, tiles of one row)."""
+    W_bits = np.asarray(W_bits, dtype=np.uint16)
+    keep = np.asarray(B) != 0
+    out, inp = W_bits.shape
+    Go, Gi = group_grid(out, inp, g_out, g_in)
+    if keep.shape != (Go, Gi):
+        raise ValueError(f"mask must be [{Go}, {Gi}]")
+    rows: List[int] = []
+    tiles: List[np.ndarray] = []
+    offsets = [0]
+    for v in range(Gi):
+        for u in range(Go):
+            if keep[u, v]:
+                rows.append(u)
+                tiles.append(W_bits[g_out * u: g_out * (u + 1), g_in * v: g_in * (v + 1)])
+        offsets.append(len(rows))
+    return PackedGroups(out=out, inp=inp, g_out=g_out, g_in=g_in,
+                        offsets=np.asarray(offsets, dtype=np.int64),
+                        block_row=np.asarray(rows, dtype=np.int32),
+                        tiles=(np.stack(tiles) if tiles else np.zeros((0, g_out, g_in), np.uint16)).astype(np.uint16))
+
+
+def unpack_groups(p: PackedGroups) -> np.ndarray:
+    """Scatter the packed blocks back to a dense [out, in] bf16 matrix; pruned groups
+    stay +0.0 (0x0000)."""
+    W = np.zeros((p.out, p.inp), dtype=np.uint16)
+    Gi = p.inp // p.g_in
+    for v in range(Gi):
+        for j in range(int(p.offsets[v]), int(p.offsets[v + 1])):
+            u = int(p.block_row[j])
+            W[p.g_out * u: p.g_out * (u + 1), p.g_in * v: p.g_in * (v + 1)] = p.tiles[j]
+    return W
+
+
+def linear_packed_groups(x_bits: np.ndarray, p: PackedGroups) -> np.ndarray:
+    """y from the packed blocks: for every kept group (u, v), y[:, rows of u] +=
+    x[:, columns of v] . block^T in float64, groups visited in packed order."""
+    x = _bf16_to_f64(x_bits)
+    y = np.zeros((x.shape[0], p.out), dtype=np.float64)
+    tiles = _bf16_to_f64(p.tiles.reshape(-1)).reshape(p.tiles.shape)
+    Gi = p.inp // p.g_in
+    for v in range(Gi):
+        xv = x[:, p.g_in * v: p.g_in * (v + 1)]
+        for j in range(int(p.offsets[v]), int(p.offsets[v + 1])):
+            u = int(p.block_row[j])
+            y[:, p.g_out * u: p.g_out * (u + 1)] += xv @ tiles[j].T
+    return y

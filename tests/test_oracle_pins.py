@@ -338,3 +338,91 @@ def test_qkv_rate_is_the_plain_mean():
     assert orc.qkv_preserved_rate(Bq, Bk, Bv) == pytest.approx(1.25 / 3, abs=1e-15)
     # a parameter-weighted mean would give (256 + 512) / (256 + 2048 + 512)
     assert abs(orc.qkv_preserved_rate(Bq, Bk, Bv) - 768 / 2816) > 0.1
+
+
+# --------------------------------------------------------------------- other group shapes (Sec. 2.1, Sec. 3.5, App. E)
+
+@pytest.mark.parametrize("g", [16, 32])
+def test_one_hot_square_group_orientation(g):
+    # a single kept g x g group (u, v) of a 2g x 3g weight keeps exactly rows g*u..g*u+g-1
+    # and columns g*v..g*v+g-1 (checked cell by cell, no Kronecker product)
+    vals = np.arange(1, 2 * g * 3 * g + 1, dtype=np.float32).reshape(2 * g, 3 * g) % 200 + 1
+    Wb = bits_of(vals)
+    for u in range(2):
+        for v in range(3):
+            B = np.zeros((2, 3), np.uint8)
+            B[u, v] = 1
+            got = orc.masked_weight_bits(Wb, B, g, g)
+            for r in range(2 * g):
+                for k in range(3 * g):
+                    inside = (g * u <= r < g * u + g) and (g * v <= k < g * v + g)
+                    assert got[r, k] == (Wb[r, k] if inside else 0)
+
+
+def test_brute_force_every_square_mask_tiny():
+    # 32 x 32 weight, 16 x 16 groups: all 16 masks; y by int64 loops where group
+    # membership is the integer division B[r // 16, k // 16]
+    rng = np.random.default_rng(11)
+    Wb, Wi = int_bits(rng, (32, 32))
+    xb, xi = int_bits(rng, (3, 32))
+    for bits in range(16):
+        B = np.array([[(bits >> 0) & 1, (bits >> 1) & 1], [(bits >> 2) & 1, (bits >> 3) & 1]], np.uint8)
+        ref = np.zeros((3, 32), np.int64)
+        for t in range(3):
+            for r in range(32):
+                ref[t, r] = sum(int(xi[t, k]) * int(Wi[r, k]) for k in range(32) if B[r // 16, k // 16])
+        y, _ = orc.linear(xb, Wb, B, 16, 16)
+        assert np.array_equal(y, ref.astype(np.float64)), bits
+        assert np.array_equal(orc.linear_packed_groups(xb, orc.pack_groups(Wb, B, 16, 16)), ref.astype(np.float64))
+
+
+def test_square_and_narrow_masks_reduce_to_row_masks():
+    rng = np.random.default_rng(12)
+    Wb = wl.random_weight_bits(128, 512, seed=12)
+    xb = wl.random_activation_bits(4, 512, seed=13)
+    # a 32 x 32 mask is the 1 x 32 mask with each group row repeated 32 times
+    Bsq = (rng.random((4, 16)) < 0.5).astype(np.uint8)
+    Brow = np.repeat(Bsq, 32, axis=0)
+    assert np.array_equal(orc.masked_weight_bits(Wb, Bsq, 32, 32), orc.masked_weight_bits(Wb, Brow, 1, 32))
+    y1, _ = orc.linear(xb, Wb, Bsq, 32, 32)
+    y2, _ = orc.linear(xb, Wb, Brow, 1, 32)
+    assert np.array_equal(y1, y2)
+    # a 1 x 128 mask whose column pairs agree is the 1 x 256 mask
+    B256 = (rng.random((128, 2)) < 0.5).astype(np.uint8)
+    B128 = np.repeat(B256, 2, axis=1)
+    assert np.array_equal(orc.masked_weight_bits(Wb, B128, 1, 128), orc.masked_weight_bits(Wb, B256))
+
+
+def test_pack_groups_reduces_to_the_1x256_layout():
+    Wb = wl.random_weight_bits(40, 768, seed=14)
+    B = wl.random_mask(40, 3, 0.5, seed=15)
+    pg, p = orc.pack_groups(Wb, B, 1, 256), orc.pack(Wb, B)
+    assert np.array_equal(pg.offsets, p.offsets) and np.array_equal(pg.block_row, p.row_idx)
+    assert np.array_equal(pg.tiles.reshape(-1, 256), p.tiles)
+
+
+@pytest.mark.parametrize("g_out,g_in", orc.GROUP_SHAPES)
+def test_pack_groups_roundtrip_counts_and_route(g_out, g_in):
+    out, inp = 256, 512
+    Wb = wl.random_weight_bits(out, inp, seed=16)
+    xb = wl.random_activation_bits(3, inp, seed=17)
+    Go, Gi = orc.group_grid(out, inp, g_out, g_in)
+    B = (np.random.default_rng(g_out * 1000 + g_in).random((Go, Gi)) < 0.45).astype(np.uint8)
+    p = orc.pack_groups(Wb, B, g_out, g_in)
+    assert p.kept == int(B.sum()) and p.tiles.shape == (p.kept, g_out, g_in)
+    assert np.all(np.diff(p.offsets) >= 0)
+    for v in range(Gi):
+        rows = p.block_row[p.offsets[v]:p.offsets[v + 1]]
+        assert rows.tolist() == [u for u in range(Go) if B[u, v]]
+    assert np.array_equal(orc.unpack_groups(p), orc.masked_weight_bits(Wb, B, g_out, g_in))
+    y, A = orc.linear(xb, Wb, B, g_out, g_in)
+    assert np.all(np.abs(orc.linear_packed_groups(xb, p) - y) <= 1e-13 * A + 1e-300)
+    assert orc.preserved_rate(B, g_out, g_in) == p.kept * g_out * g_in / (out * inp)
+
+
+def test_group_grid_rejects_untiled_shapes():
+    assert orc.group_grid(11008, 4096, 128, 128) == (86, 32)
+    with pytest.raises(ValueError):
+        orc.group_grid(100, 256, 16, 16)
+    with pytest.raises(ValueError):
+        orc.group_grid(128, 200, 1, 128)

@@ -113,3 +113,11 @@ def test_paper_shaped_allocation_matches_printed_statistics():
     assert int(m.sum()) == int(k[0, 0]) and np.array_equal(m, wl.group_mask(w, 0, int(k[0, 0])))
     with pytest.raises(ValueError):
         wl.workload(4, allocation="paper")
+
+
+def test_every_config_shape_is_tiled_by_every_group_shape():
+    for cfg, d in ((1, 0.5), (2, 0.5), (3, 0.5), (4, 0.5), (5, 0.5)):
+        for L in wl.workload(cfg, d).layers[:7]:
+            for g_out, g_in in orc.GROUP_SHAPES:
+                Go, Gi = orc.group_grid(L.out, L.inp, g_out, g_in)
+                assert Go * g_out == L.out and Gi * g_in == L.inp
