@@ -20,6 +20,9 @@
  *     touches no device memory.
  *   - The caller owns W, mask, x, y and W_hat.  The library owns the handle's
  *     device buffers until gs_free.
+ *   - One process drives one CUDA device: the kernels' shared-memory limits
+ *     and the SM count that sizes their grids are configured on the first
+ *     device that launches them and reused for every later call.
  *   - Kernels bound every wait they perform.  A wait that runs out records
  *     GS_ERR_DEVICE_TIMEOUT in a library-owned device flag and the kernel
  *     returns; gs_device_status reads (and clears) that flag.
