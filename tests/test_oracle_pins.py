@@ -426,3 +426,18 @@ def test_group_grid_rejects_untiled_shapes():
         orc.group_grid(100, 256, 16, 16)
     with pytest.raises(ValueError):
         orc.group_grid(128, 200, 1, 128)
+
+
+def test_golden_square_layout():
+    g = json.loads((GOLDEN / "square_layout.json").read_text())
+    W = bits_of(np.asarray(g["W"], np.float32))
+    B = np.asarray(g["mask"], np.uint8)
+    x = bits_of(np.asarray(g["x"], np.float32))
+    e = g["expected"]
+    p = orc.pack_groups(W, B, g["g"], g["g"])
+    assert p.offsets.tolist() == e["offsets"] and p.block_row.tolist() == e["block_row"]
+    assert np.array_equal(p.tiles, bits_of(np.asarray(e["tiles"], np.float32)))
+    y, _ = orc.linear(x, W, B, g["g"], g["g"])
+    assert np.array_equal(y, np.asarray(e["y"], np.float64))
+    assert np.array_equal(orc.linear_packed_groups(x, p), np.asarray(e["y"], np.float64))
+    assert orc.preserved_rate(B, g["g"], g["g"]) == e["preserved_rate"]
