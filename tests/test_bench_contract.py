@@ -40,3 +40,20 @@ def test_reference_arm_other_ranks_are_silent():
     r = _run({"RANK": "1", "WORLD_SIZE": "2"})
     assert r.returncode == 0, r.stderr[-2000:]
     assert r.stdout.strip() == ""
+
+
+def test_bench_helpers():
+    sys.path.insert(0, str(ROOT))
+    import bench
+    # the recorded DRAM traffic is reported only for the kernel source it was measured on
+    rec = json.loads((ROOT / "profiles" / "traffic.json").read_text())["k_decode"]["llama2-7b-block"]
+    got = bench.recorded_traffic("k_decode", "gs_decode.cu", "llama2-7b-block")
+    if rec["source_sha256_16"] == bench.kernel_source_hash("gs_decode.cu"):
+        assert got == rec["dram_bytes_per_launch"]
+    else:
+        assert got is None
+    assert bench.recorded_traffic("k_decode", "gs_decode.cu", "no-such-workload") is None
+    assert bench.recorded_traffic("no_such_kernel", "gs_decode.cu", "llama2-7b-block") is None
+    # threads kept busy = process CPU time / wall time, at least one
+    assert bench._cores_used(30.0, 10.0) == 3 and bench._cores_used(0.2, 10.0) == 1
+    assert bench._cores_used(5.0, 0.0) == 1
