@@ -466,20 +466,24 @@ def run_ours(args):
             del Wd_rot
     torch.cuda.empty_cache()
 
-    # ---- tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
+    # ---- per-GPU characterisations (N = 1 only: at N > 1 every rank would repeat them
+    # while all GPUs are held, and they are not part of the scaled metric)
+    # tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
     prefill = None
     prefill_sweep = None
     decode_sweep = None
-    if not args.no_prefill:
+    mask_export = None
+    if not args.no_prefill and world == 1:
         prefill = measure_prefill(gs, torch, dev, stream, peaks)
         prefill_sweep = measure_prefill_sweep(gs, torch, dev, stream, peaks)
         decode_sweep = measure_decode_sweep(gs, torch, dev, stream, peaks)
 
-    # ---- selector export (the step that produces the masks), measured last
-    try:
-        mask_export = measure_select(gs, torch, dev, stream, peaks)
-    except Exception as e:   # reported in the line, never hidden
-        mask_export = {"error": f"{type(e).__name__}: {e}"}
+    # selector export (the step that produces the masks), measured last
+    if world == 1:
+        try:
+            mask_export = measure_select(gs, torch, dev, stream, peaks)
+        except Exception as e:   # reported in the line, never hidden
+            mask_export = {"error": f"{type(e).__name__}: {e}"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
