@@ -82,3 +82,19 @@ def test_host_side_validation(lib):
     assert lib.gs_select_groups(fake, 8, fake + 16, None, None) == INVALID           # mask overlaps logits
     assert lib.gs_select_groups(None, 0, None, None, None) == 0                      # empty: nothing to do
     lib.gs_free(None)
+
+
+def test_header_is_plain_c(tmp_path):
+    # the boundary is a C ABI: the header compiles as strict C99 (no C++ or torch types) and as C++
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "use_header.c"
+    src.write_text('#include "groupsparse.h"\n'
+                   "int main(void) { gs_packed* p = 0; (void)p; return gs_status_string(GS_OK)[0] == 0; }\n")
+    for cmd in ([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror"],
+                [gcc, "-x", "c++", "-std=c++17", "-Wall", "-Wextra", "-Werror"]):
+        r = subprocess.run(cmd + [f"-I{ROOT / 'include'}", "-fsyntax-only", str(src)], capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
