@@ -202,6 +202,24 @@ def oracle_sample_rate(layers, seconds: float, rows_per_call: int = 256):
                       f"time over the calls"}
 
 
+def oracle_single_thread_rate(seconds: float):
+    """The same bounded oracle sample in a child process whose BLAS and OpenMP
+    pools are limited to one thread (the variables must be set before numpy
+    loads, hence the child).  The child generates its own copy of the seeded
+    block inputs and touches no GPU."""
+    env = dict(os.environ)
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+        env[k] = "1"
+    env.pop("RANK", None)
+    env.pop("WORLD_SIZE", None)
+    r = subprocess.run([sys.executable, str(Path(__file__).resolve()), "--oracle-single-thread", "--warmup", "3",
+                        "--cpu-seconds", str(seconds)], env=env, capture_output=True, text=True, timeout=600)
+    if r.returncode != 0:
+        return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}"}
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": d["value"], "unit": d["unit"], "cores": d["cores"], "sample": d["sample"]}
+
+
 def _cores_used(cpu_seconds: float, wall_seconds: float) -> int:
     """Threads the oracle kept busy on average: process CPU time over wall time."""
     if wall_seconds <= 0:
@@ -488,6 +506,7 @@ def run_ours(args):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample_rate(layers, args.cpu_seconds)
+        cpu["single_thread"] = oracle_single_thread_rate(args.cpu_seconds / 2)
 
     hbm_peak = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
     traffic = recorded_traffic("k_decode", "gs_decode.cu", "llama2-7b-block")
@@ -798,6 +817,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--rotate", type=int, default=0, help="rotated packed copies (0 = enough to exceed 3x L2)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--oracle-single-thread", action="store_true",
+                    help="internal: time the oracle sample only and print it (run with one BLAS thread)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--layer", default=None, help="single-layer mode: OUTxIN (random mask of --density)")
@@ -809,6 +830,10 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.oracle_single_thread:
+        _, layers = block_inputs()
+        print(json.dumps(oracle_sample_rate(layers, args.cpu_seconds)), flush=True)
+        return 0
     if args.impl == "reference":
         return run_reference(args)
     if args.layer:

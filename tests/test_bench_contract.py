@@ -57,3 +57,11 @@ def test_bench_helpers():
     # threads kept busy = process CPU time / wall time, at least one
     assert bench._cores_used(30.0, 10.0) == 3 and bench._cores_used(0.2, 10.0) == 1
     assert bench._cores_used(5.0, 0.0) == 1
+
+
+def test_single_thread_oracle_baseline():
+    sys.path.insert(0, str(ROOT))
+    import bench
+    d = bench.oracle_single_thread_rate(0.5)
+    assert "error" not in d, d
+    assert d["cores"] == 1 and d["value"] > 0 and d["unit"] == "tokens/s" and d["sample"]
