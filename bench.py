@@ -212,12 +212,15 @@ def oracle_single_thread_rate(seconds: float):
         env[k] = "1"
     env.pop("RANK", None)
     env.pop("WORLD_SIZE", None)
-    r = subprocess.run([sys.executable, str(Path(__file__).resolve()), "--oracle-single-thread", "--warmup", "3",
-                        "--cpu-seconds", str(seconds)], env=env, capture_output=True, text=True, timeout=600)
-    if r.returncode != 0:
-        return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}"}
-    d = json.loads(r.stdout.strip().splitlines()[-1])
-    return {"value": d["value"], "unit": d["unit"], "cores": d["cores"], "sample": d["sample"]}
+    try:
+        r = subprocess.run([sys.executable, str(Path(__file__).resolve()), "--oracle-single-thread", "--warmup", "3",
+                            "--cpu-seconds", str(seconds)], env=env, capture_output=True, text=True, timeout=600)
+        if r.returncode != 0:
+            return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}"}
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+        return {"value": d["value"], "unit": d["unit"], "cores": d["cores"], "sample": d["sample"]}
+    except Exception as e:   # reported in the line, never hidden; the GPU figures stand without it
+        return {"error": f"{type(e).__name__}: {e}"}
 
 
 def _cores_used(cpu_seconds: float, wall_seconds: float) -> int:
