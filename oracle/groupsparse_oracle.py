@@ -43,7 +43,10 @@ sigmoid at several temperatures, and the global preserved rate the paper
 prints for its LLaMA-2-7B allocation in Sec. 3.5; for other group shapes:
 cell-by-cell one-hot orientation, brute force over every 16x16 mask of a
 32x32 weight against int64 loops, reduction of square and 1x128 masks to row
-masks, and the 1x256 layout identity).
+masks, and the 1x256 layout identity; for token subsets: a hand-derived golden
+case whose token list is out of order and repeats a row, and int64 loops per
+listed token; for the kept count: hand-written masks with keep bytes other
+than 1, and the exact per-layer budget of the seeded generator).
 """
 from __future__ import annotations
 

@@ -441,3 +441,59 @@ def test_golden_square_layout():
     assert np.array_equal(y, np.asarray(e["y"], np.float64))
     assert np.array_equal(orc.linear_packed_groups(x, p), np.asarray(e["y"], np.float64))
     assert orc.preserved_rate(B, g["g"], g["g"]) == e["preserved_rate"]
+
+
+# --------------------------------------------------------------------- token subsets and kept counts
+
+def test_golden_token_rows():
+    # linear_tokens returns the listed rows, in the listed order, repeats included
+    g = json.loads((GOLDEN / "token_rows.json").read_text())
+    B = np.asarray(g["mask"], dtype=np.uint8)
+    W = const_groups(g["W_const"])
+    x = const_groups(g["x_const"])
+    y, A = orc.linear_tokens(x, W, B, g["tokens"])
+    e = g["expected"]
+    assert np.array_equal(y, np.asarray(e["y"]))
+    assert np.array_equal(A, np.asarray(e["A"]))
+    assert orc.kept_groups(B) == e["kept_groups"]
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_token_rows_against_integer_loops(seed):
+    # every listed token row equals the exact int64 layer output of that token;
+    # the list is unsorted and repeats entries (a sorted or deduplicated result fails)
+    rng = np.random.default_rng(100 + seed)
+    out, inp, T = 7, 1024, 6
+    xb, xi = int_bits(rng, (T, inp))
+    Wb, Wi = int_bits(rng, (out, inp))
+    B = (rng.random((out, inp // 256)) < 0.5).astype(np.uint8)
+    tokens = [5, 1, 1, 3, 0, 5]
+    y, A = orc.linear_tokens(xb, Wb, B, tokens)
+    assert y.shape == (len(tokens), out)
+    for i, t in enumerate(tokens):
+        assert np.array_equal(y[i], int_reference(xi[t:t + 1], Wi, B)[0].astype(np.float64))
+        assert np.array_equal(A[i], int_reference(np.abs(xi[t:t + 1]), np.abs(Wi), B)[0].astype(np.float64))
+
+
+def test_kept_groups_counts_nonzero_bytes_as_keep():
+    # mask bytes are keep-if-nonzero: 3, 255 and 1 all keep; the count is the
+    # numerator of Eq. 2, here written out by hand
+    B = np.array([[0, 3, 0, 0], [255, 0, 0, 1], [1, 1, 0, 0]], dtype=np.uint8)
+    assert orc.kept_groups(B) == 5
+    assert orc.kept_groups(np.zeros((9, 4), np.uint8)) == 0
+    assert orc.kept_groups(np.ones((9, 4), np.uint8)) == 36
+    assert orc.kept_groups(B.astype(bool)) == 5
+
+
+def test_kept_groups_matches_the_allocated_budget():
+    # the seeded generator places exactly k_l groups per layer (its own top-k
+    # recipe, no oracle code); the oracle's count must return each k_l and the sum
+    from paper_2609_33977_gb300 import workload as wl_mod
+    w = wl_mod.workload(2)
+    ks = wl_mod.keep_counts(w)
+    total = 0
+    for i in (0, 4, 6):
+        B = wl_mod.group_mask(w, i, int(ks[i]))
+        assert orc.kept_groups(B) == int(ks[i])
+        total += orc.kept_groups(B)
+    assert total == int(ks[0] + ks[4] + ks[6])
