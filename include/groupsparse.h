@@ -175,9 +175,12 @@ gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* r
  *
  * mask_dev       uint8 [out][in/256] row-major; nonzero = keep.  Read only.
  * out, in        out >= 1; in >= 256 and a multiple of 256.
- * offsets_dev    int64 [in/256 + 1], caller-owned, overwritten.
- * win_off16_dev  int32 [in/256][ceil(out/16) + 1], caller-owned, overwritten.
- * kmask16_dev    uint16 [in/256][ceil(out/16)], caller-owned, overwritten.
+ * offsets_dev    int64 [in/256 + 1], caller-owned, 8-byte aligned, overwritten.
+ * win_off16_dev  int32 [in/256][ceil(out/16) + 1], caller-owned, 4-byte
+ *                aligned, overwritten.
+ * kmask16_dev    uint16 [in/256][ceil(out/16)], caller-owned, 2-byte aligned,
+ *                overwritten.
+ * The three outputs must not overlap each other or the mask.
  * Temporary counts live in one fixed array in the library's device memory
  * (2^20 entries of int32, held by every GPU that loads the library until the
  * process exits); (in/256) * ceil(out/16) above 2^20 returns
@@ -188,7 +191,8 @@ gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* r
  * The first call on a device looks up the array's device address (with that
  * device current) and caches it; make that first call before any stream
  * capture.  Asynchronous on `stream`.
- * Errors: INVALID_ARG (nulls, sizes), UNSUPPORTED (beyond the fixed array), CUDA.
+ * Errors: INVALID_ARG (nulls, sizes, misaligned or overlapping buffers),
+ * UNSUPPORTED (beyond the fixed array), CUDA.
  */
 gs_status gs_pack_index_noalloc(const uint8_t* mask_dev, int64_t out, int64_t in, int64_t* offsets_dev,
                                 int32_t* win_off16_dev, uint16_t* kmask16_dev, void* stream);

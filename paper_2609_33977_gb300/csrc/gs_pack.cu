@@ -262,9 +262,23 @@ extern "C" gs_status gs_pack_index_noalloc(const uint8_t* mask_dev, int64_t out,
   using namespace gs;
   if (!mask_dev || !offsets_dev || !win_off16_dev || !kmask16_dev) return GS_ERR_INVALID_ARG;
   if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX || in % kGroupIn != 0) return GS_ERR_INVALID_ARG;
+  // element alignment of each output (int64, int32, uint16)
+  if ((reinterpret_cast<uintptr_t>(offsets_dev) & 7u) != 0 || (reinterpret_cast<uintptr_t>(win_off16_dev) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(kmask16_dev) & 1u) != 0)
+    return GS_ERR_INVALID_ARG;
   const int64_t G = in / kGroupIn;
   const int64_t nw16 = (out + kWin16 - 1) / kWin16;
   if (G * nw16 > kNoAllocMaxEntries) return GS_ERR_UNSUPPORTED;   // beyond the fixed scratch array
+  {
+    // the outputs must not overlap each other or the mask they are computed from
+    const uintptr_t lo[4] = {reinterpret_cast<uintptr_t>(mask_dev), reinterpret_cast<uintptr_t>(offsets_dev),
+                             reinterpret_cast<uintptr_t>(win_off16_dev), reinterpret_cast<uintptr_t>(kmask16_dev)};
+    const uintptr_t len[4] = {(uintptr_t)(out * G), (uintptr_t)(8 * (G + 1)), (uintptr_t)(4 * G * (nw16 + 1)),
+                              (uintptr_t)(2 * G * nw16)};
+    for (int a = 0; a < 4; ++a)
+      for (int b = a + 1; b < 4; ++b)
+        if (lo[a] < lo[b] + len[b] && lo[b] < lo[a] + len[a]) return GS_ERR_INVALID_ARG;
+  }
   int32_t* counts = nullptr;
   const gs_status st = noalloc_counts_address(&counts);
   if (st != GS_OK) return st;

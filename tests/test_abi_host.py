@@ -81,6 +81,15 @@ def test_host_side_validation(lib):
     assert lib.gs_select_groups(fake, 8, fake + 0x1000, fake + 4, None) == INVALID   # misaligned count
     assert lib.gs_select_groups(fake, 8, fake + 16, None, None) == INVALID           # mask overlaps logits
     assert lib.gs_select_groups(None, 0, None, None, None) == 0                      # empty: nothing to do
+    lib.gs_pack_index_noalloc.argtypes = [vp, i64, i64, vp, vp, vp, vp]
+    m, o, w, k = 0x100000, 0x200000, 0x300000, 0x400000   # mask, offsets, window offsets, window masks
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o + 4, w, k, None) == INVALID     # int64 offsets at 4 B
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w + 2, k, None) == INVALID     # int32 offsets at 2 B
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w, k + 1, None) == INVALID     # uint16 masks at 1 B
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, o + 16, k, None) == INVALID    # outputs overlap
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w, m + 16, None) == INVALID    # output overlaps the mask
+    assert lib.gs_pack_index_noalloc(None, 16, 512, o, w, k, None) == INVALID
+    assert lib.gs_pack_index_noalloc(m, 16, 300, o, w, k, None) == INVALID
     lib.gs_free(None)
 
 

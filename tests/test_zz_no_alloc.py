@@ -9,14 +9,17 @@ offsets and window kept-masks as gs_pack into buffers the caller provides; its
 temporary per-window counts live in a fixed array inside the library.
 
 Each case calls the entry point twice in a row (the shared array keeps the
-previous call's contents) and compares both results bit for bit with the
-layout gs_pack produces for the same mask.
+previous call's contents) and compares both results bit for bit with the CPU
+oracle's packed layout for the same mask, and with what gs_pack produces.  One
+case packs a large layer and then a smaller one with a different mask, so a
+result that read counts left behind by the earlier call would differ.
 """
 import ctypes
 
 import numpy as np
 import pytest
 
+from oracle import groupsparse_oracle as orc
 from paper_2609_33977_gb300 import workload as wl
 
 pytestmark = pytest.mark.gpu
@@ -59,12 +62,31 @@ def test_matches_gs_pack_on_two_calls(ctx, out, inp, d, seed):
     Wb = wl.random_weight_bits(out, inp, seed=seed)
     mask = torch.from_numpy(B).cuda()
     W = torch.from_numpy(Wb.view(np.int16)).view(torch.bfloat16).cuda()
-    ref = gs.pack(W, mask).export()
+    ref = orc.pack(Wb, B)
+    lib_ref = gs.pack(W, mask).export()
     for _ in range(2):
         offsets, win, km = run_noalloc(torch, lib, mask, out, inp)
-        assert np.array_equal(offsets, ref["offsets"])
-        assert np.array_equal(win, ref["win_off16"])
-        assert np.array_equal(km, ref["kmask16"])
+        assert np.array_equal(offsets, ref.offsets)
+        assert np.array_equal(win, ref.win_off16)
+        assert np.array_equal(km, ref.kmask16)
+        assert np.array_equal(offsets, lib_ref["offsets"])
+        assert np.array_equal(win, lib_ref["win_off16"])
+        assert np.array_equal(km, lib_ref["kmask16"])
+
+
+def test_large_then_small_layer_with_another_mask(ctx):
+    # the shared array still holds the large layer's counts when the small one
+    # is packed; every entry the small call reads must be its own
+    torch, gs, lib = ctx
+    shapes = [(13824, 5120, 0.7, 11), (300, 1024, 0.3, 12), (13824, 5120, 0.2, 13), (48, 512, 0.9, 14)]
+    for out, inp, d, seed in shapes:
+        B = wl.random_mask(out, inp // 256, d, seed=seed)
+        Wb = np.zeros((out, inp), np.uint16)
+        ref = orc.pack(Wb, B)
+        offsets, win, km = run_noalloc(torch, lib, torch.from_numpy(B).cuda(), out, inp)
+        assert np.array_equal(offsets, ref.offsets), (out, inp)
+        assert np.array_equal(win, ref.win_off16), (out, inp)
+        assert np.array_equal(km, ref.kmask16), (out, inp)
 
 
 def test_rejects_sizes_beyond_the_fixed_array(ctx):
@@ -75,3 +97,10 @@ def test_rejects_sizes_beyond_the_fixed_array(ctx):
     assert lib.gs_pack_index_noalloc(fake, out, 256 * G, fake, fake, fake, None) == GS_ERR_UNSUPPORTED
     assert lib.gs_pack_index_noalloc(None, 16, 256, fake, fake, fake, None) == GS_ERR_INVALID_ARG
     assert lib.gs_pack_index_noalloc(fake, 16, 300, fake, fake, fake, None) == GS_ERR_INVALID_ARG
+    # misaligned outputs and overlapping buffers are refused before any launch
+    m, o, w, k = 0x100000, 0x200000, 0x300000, 0x400000
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o + 4, w, k, None) == GS_ERR_INVALID_ARG
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w + 2, k, None) == GS_ERR_INVALID_ARG
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w, k + 1, None) == GS_ERR_INVALID_ARG
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, o + 16, k, None) == GS_ERR_INVALID_ARG
+    assert lib.gs_pack_index_noalloc(m, 16, 512, o, w, m + 16, None) == GS_ERR_INVALID_ARG
