@@ -87,14 +87,20 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
  * projection, no bias), fp32 accumulation, bf16 output rounded to nearest even.
  *
  * x_dev  bf16 [T][in] row-major, caller-owned, read only.
- * p      packed handle from gs_pack.  The handle also owns the decode kernel's
- *        split-reduction scratch, so gs_linear / gs_linear_ex /
- *        gs_linear_batched calls that share a handle must be ordered with
- *        respect to each other (same stream, or synchronized streams).
+ * p      packed handle from gs_pack; read only, so one handle may serve
+ *        gs_linear / gs_linear_ex / gs_linear_batched calls on several streams
+ *        at once.  The decode kernel's split-reduction scratch is kept per
+ *        (handle, stream): the scratch of gs_pack's stream is made by gs_pack,
+ *        and the first decode-regime call on any other stream allocates that
+ *        stream's (so make it before capturing that stream into a CUDA graph).
+ *        Up to 8 streams per handle.  Calls on one stream are ordered by the
+ *        stream; a CUDA graph keeps the scratch of the stream it was captured
+ *        from, so its replays must be ordered with other work on that stream.
  * T      number of tokens; T == 0 is a no-op, T < 0 is INVALID_ARG.
  * y_dev  bf16 [T][out] row-major, caller-owned; fully overwritten (rows of
  *        outputs with no kept group are written as +0.0).
- * Errors: INVALID_ARG, CUDA.  Asynchronous on `stream`.
+ * Errors: INVALID_ARG, UNSUPPORTED (a ninth stream on one handle), OOM (a new
+ * stream's scratch), CUDA.  Asynchronous on `stream`.
  */
 gs_status gs_linear(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream);
 
@@ -157,7 +163,10 @@ gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t*
 
 /*
  * gs_packed_export - synchronous copy of the packed layout to host buffers
- * (for bit-exact checks).  Sizes: offsets int64[G+1], row_idx int32[K],
+ * (for bit-exact checks).  The layout holds exactly the kept groups of Eq. 1
+ * (Sec. 2.1: B selects whole 1 x 256 groups of W) and where each one sits in
+ * W; the paper prints no layout, and the one here is the chunk-major layout
+ * that gs_pack describes.  Sizes: offsets int64[G+1], row_idx int32[K],
  * tiles uint16[K*256], win_off16 int32[G*(ceil(out/16)+1)],
  * kmask16 uint16[G*ceil(out/16)], with K = kept_groups.  Any pointer may be NULL.
  */
@@ -207,9 +216,59 @@ const char* gs_status_string(gs_status s);
  * gs_device_status - synchronizes `stream`, then reads and clears the device
  * error flag of the current device: GS_OK or GS_ERR_DEVICE_TIMEOUT (a bounded
  * wait in some earlier kernel ran out).  GS_ERR_CUDA if the stream itself
- * reports an error.
+ * reports an error.  After a timeout, the outputs of the call that timed out
+ * (and of calls issued before this status was read) are undefined.  Reading
+ * the timeout also marks every decode split scratch for re-zeroing, which
+ * happens on the stream of its next use, so later calls are correct again.
  */
 gs_status gs_device_status(void* stream);
+
+/*
+ * gs_preserved_rates - the preserved rates of App. F from kept-group counts:
+ * a projection's active weights over its total weights after the binary mask
+ * is applied, and the global rate over all target projections, which is
+ * 1 - s of Eq. 2 (the parameter-weighted mean).  Every group holds
+ * group_weights = g_out * g_in weights (256 for 1 x 256 groups).
+ *
+ * n               number of layers, n >= 0.
+ * kept_host       int64 [n] kept groups per layer (e.g. gs_packed_info, or the
+ *                 count gs_select_groups writes).
+ * d_out_host,
+ * d_in_host       int64 [n] layer shapes.
+ * rates_host      double [n] or NULL: kept_i * group_weights / (d_out_i d_in_i).
+ * global_host     double or NULL: sum_i kept_i group_weights / sum_i d_out_i d_in_i
+ *                 (0 when n == 0).
+ * n_qkv, qkv_host int32 [n_qkv][3] layer indices (q, k, v); App. F reports the
+ *                 three attention input projections as the plain mean of their
+ *                 rates: qkv_rates_host[j] = (r_q + r_k + r_v) / 3.
+ * Host only (no device work).  Errors: INVALID_ARG (negative sizes or counts,
+ * more kept weights than a layer holds, an index out of range, totals at or
+ * above 2^62, NULL arrays with nonzero counts).
+ */
+gs_status gs_preserved_rates(int32_t n, const int64_t* kept_host, const int64_t* d_out_host,
+                             const int64_t* d_in_host, int64_t group_weights, double* rates_host,
+                             double* global_host, int32_t n_qkv, const int32_t* qkv_host,
+                             double* qkv_rates_host);
+
+/*
+ * Test hooks for the failure paths (the paper has no counterpart; they exist
+ * so that the error handling can be exercised without faulting a GPU).
+ *
+ * gs_debug_fail_alloc(nth) - the nth device allocation the library makes from
+ * now on fails as if the device were out of memory (nth = 1: the next one;
+ * 0 disarms).  gs_pack then returns GS_ERR_OOM and frees what it had
+ * allocated.
+ *
+ * gs_debug_inject_wait(family, limit_ns) - the next launch of that kernel
+ * family (GS_ALGO_DECODE or GS_ALGO_PREFILL) makes its first CTA (the first
+ * CTA pair for prefill) wait, before issuing any copy or tensor-core work, on
+ * a library word that nothing ever sets, for at most limit_ns (<= 1 s).  The
+ * wait runs out, the kernel records GS_ERR_DEVICE_TIMEOUT and that CTA skips
+ * its work; the other CTAs finish theirs.  One-shot; limit_ns = 0 disarms.
+ * Errors: INVALID_ARG (negative count, unknown family, limit above 1 s).
+ */
+gs_status gs_debug_fail_alloc(int64_t nth);
+gs_status gs_debug_inject_wait(gs_algo family, uint64_t limit_ns);
 
 /* Number of kernel launches the library issued since the process started (all
  * families; used to report launch counts). */

@@ -3,11 +3,15 @@
 Each translation unit is compiled in parallel to an object under
 `paper_2609_33977_gb300/_build/`, then linked into
 `paper_2609_33977_gb300/libgroupsparse.so` against the shared CUDA runtime.
-A rebuild happens only when a source or header is newer than the library.
+Beside the library a stamp file records a hash of every source, header, this
+script, the compiler flags and the nvcc version; the library is rebuilt unless
+the stamp matches, so a prebuilt library from another tree or another set of
+flags is never reused.
 """
 from __future__ import annotations
 
 import concurrent.futures as cf
+import hashlib
 import os
 import shutil
 import subprocess
@@ -44,20 +48,39 @@ def _headers():
     return sorted(CSRC.glob("*.cuh")) + sorted(INCLUDE.glob("*.h"))
 
 
-def needs_build() -> bool:
-    if not LIB.exists():
+STAMP = LIB.with_suffix(".so.stamp")
+FLAGS = ["-std=c++17", "-O3", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
+
+
+def _nvcc_version(nvcc: str) -> str:
+    r = subprocess.run([nvcc, "--version"], capture_output=True, text=True)
+    return r.stdout.strip()
+
+
+def build_stamp(extra_flags=None) -> str:
+    """Hash of everything the library is built from."""
+    h = hashlib.sha256()
+    for p in list(sources()) + _headers() + [Path(__file__)]:
+        h.update(p.name.encode())
+        h.update(p.read_bytes())
+    h.update(" ".join(FLAGS + list(extra_flags or [])).encode())
+    h.update(_nvcc_version(_nvcc()).encode())
+    return h.hexdigest()
+
+
+def needs_build(extra_flags=None) -> bool:
+    if not LIB.exists() or not STAMP.exists():
         return True
-    t = LIB.stat().st_mtime
-    return any(p.stat().st_mtime > t for p in list(sources()) + _headers() + [Path(__file__)])
+    return STAMP.read_text().strip() != build_stamp(extra_flags)
 
 
 def build_library(force: bool = False, verbose: bool = False, extra_flags=None) -> Path:
-    if not force and not needs_build():
+    if not force and not needs_build(extra_flags):
         return LIB
     nvcc = _nvcc()
+    stamp = build_stamp(extra_flags)
     BUILD.mkdir(exist_ok=True)
-    common = [nvcc, "-std=c++17", "-O3", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC", f"-I{INCLUDE}",
-              "--expt-relaxed-constexpr", *(extra_flags or [])]
+    common = [nvcc, *FLAGS, f"-I{INCLUDE}", *(extra_flags or [])]
 
     def compile_one(src: Path):
         obj = BUILD / (src.stem + ".o")
@@ -80,6 +103,7 @@ def build_library(force: bool = False, verbose: bool = False, extra_flags=None) 
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
+    STAMP.write_text(stamp + "\n")
     return LIB
 
 

@@ -16,6 +16,10 @@ constexpr int kMaxDevices = 64;
 std::mutex g_flag_mu;
 int* g_flags[kMaxDevices] = {nullptr};
 std::atomic<int64_t> g_launches{0};
+std::atomic<uint64_t> g_timeout_epoch{0};
+// test hooks: countdown to a failing allocation (0 = off), injected wait limits
+std::atomic<int64_t> g_fail_alloc_in{0};
+std::atomic<uint64_t> g_inject_ns[3] = {{0}, {0}, {0}};
 
 // Token count at and above which gs_linear uses the tensor-core kernel.
 constexpr int64_t kPrefillMinTokens = 33;
@@ -44,14 +48,9 @@ void free_buffers(gs_packed* p) {
 gs_status dev_alloc(void** ptr, size_t bytes, size_t* total) {
   *ptr = nullptr;
   if (bytes == 0) return GS_OK;
-  const cudaError_t e = cudaMalloc(ptr, bytes);
-  if (e == cudaErrorMemoryAllocation) {
-    cudaGetLastError();
-    return GS_ERR_OOM;
-  }
-  if (e != cudaSuccess) return GS_ERR_CUDA;
-  *total += bytes;
-  return GS_OK;
+  const gs_status st = lib_malloc(ptr, bytes);
+  if (st == GS_OK) *total += bytes;
+  return st;
 }
 
 gs_status check_handle(const gs_packed* p) {
@@ -69,8 +68,8 @@ int* device_error_flag() {
   std::lock_guard<std::mutex> lk(g_flag_mu);
   if (!g_flags[dev]) {
     int* f = nullptr;
-    if (cudaMalloc(&f, sizeof(int)) != cudaSuccess) return nullptr;
-    if (cudaMemset(f, 0, sizeof(int)) != cudaSuccess) {
+    if (cudaMalloc(&f, 2 * sizeof(int)) != cudaSuccess) return nullptr;
+    if (cudaMemset(f, 0, 2 * sizeof(int)) != cudaSuccess) {
       cudaFree(f);
       return nullptr;
     }
@@ -80,6 +79,32 @@ int* device_error_flag() {
 }
 
 void note_launch(int64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+uint64_t timeout_epoch() { return g_timeout_epoch.load(std::memory_order_acquire); }
+
+gs_status lib_malloc(void** ptr, size_t bytes) {
+  *ptr = nullptr;
+  int64_t n = g_fail_alloc_in.load(std::memory_order_relaxed);
+  while (n > 0 && !g_fail_alloc_in.compare_exchange_weak(n, n - 1)) {
+  }
+  if (n == 1) return GS_ERR_OOM;   // the armed allocation fails as if the device were full
+  const cudaError_t e = cudaMalloc(ptr, bytes);
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    *ptr = nullptr;
+    return GS_ERR_OOM;
+  }
+  if (e != cudaSuccess) {
+    *ptr = nullptr;
+    return GS_ERR_CUDA;
+  }
+  return GS_OK;
+}
+
+uint64_t take_injected_wait(int family) {
+  if (family < 1 || family > 2) return 0;
+  return g_inject_ns[family].exchange(0);
+}
 
 }  // namespace gs
 
@@ -306,8 +331,56 @@ gs_status gs_device_status(void* stream) {
   if (cudaMemcpy(&v, f, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return GS_ERR_CUDA;
   if (v != 0) {
     cudaMemset(f, 0, sizeof(int));
+    // a kernel that gave up may have left split counters half counted: every
+    // decode scratch slot is re-zeroed before its next use
+    g_timeout_epoch.fetch_add(1, std::memory_order_acq_rel);
     return GS_ERR_DEVICE_TIMEOUT;
   }
+  return GS_OK;
+}
+
+gs_status gs_preserved_rates(int32_t n, const int64_t* kept_host, const int64_t* d_out_host, const int64_t* d_in_host,
+                             int64_t group_weights, double* rates_host, double* global_host, int32_t n_qkv,
+                             const int32_t* qkv_host, double* qkv_rates_host) {
+  if (n < 0 || n_qkv < 0 || group_weights <= 0) return GS_ERR_INVALID_ARG;
+  if (n > 0 && (!kept_host || !d_out_host || !d_in_host)) return GS_ERR_INVALID_ARG;
+  if (n_qkv > 0 && (!qkv_host || !qkv_rates_host)) return GS_ERR_INVALID_ARG;
+  // exact integer totals: every count and size below 2^62
+  constexpr int64_t kLim = int64_t(1) << 62;
+  int64_t active = 0, total = 0;
+  for (int32_t i = 0; i < n; ++i) {
+    const int64_t k = kept_host[i], a = d_out_host[i], b = d_in_host[i];
+    if (a <= 0 || b <= 0 || k < 0 || a > kLim / b) return GS_ERR_INVALID_ARG;
+    const int64_t size = a * b;
+    if (k > size / group_weights) return GS_ERR_INVALID_ARG;   // more kept weights than the layer has
+    if (active > kLim - k * group_weights || total > kLim - size) return GS_ERR_INVALID_ARG;
+    active += k * group_weights;
+    total += size;
+  }
+  for (int32_t j = 0; j < n_qkv; ++j)
+    for (int t = 0; t < 3; ++t)
+      if (qkv_host[3 * j + t] < 0 || qkv_host[3 * j + t] >= n) return GS_ERR_INVALID_ARG;
+  auto rate = [&](int32_t i) {
+    return (double)(kept_host[i] * group_weights) / (double)(d_out_host[i] * d_in_host[i]);
+  };
+  if (rates_host)
+    for (int32_t i = 0; i < n; ++i) rates_host[i] = rate(i);
+  if (global_host) *global_host = total > 0 ? (double)active / (double)total : 0.0;
+  for (int32_t j = 0; j < n_qkv; ++j)
+    qkv_rates_host[j] = (rate(qkv_host[3 * j]) + rate(qkv_host[3 * j + 1]) + rate(qkv_host[3 * j + 2])) / 3.0;
+  return GS_OK;
+}
+
+gs_status gs_debug_fail_alloc(int64_t nth) {
+  if (nth < 0) return GS_ERR_INVALID_ARG;
+  g_fail_alloc_in.store(nth, std::memory_order_relaxed);
+  return GS_OK;
+}
+
+gs_status gs_debug_inject_wait(gs_algo family, uint64_t limit_ns) {
+  if (family != GS_ALGO_DECODE && family != GS_ALGO_PREFILL) return GS_ERR_INVALID_ARG;
+  if (limit_ns > 1000000000ull) return GS_ERR_INVALID_ARG;
+  g_inject_ns[family].store(limit_ns);
   return GS_OK;
 }
 

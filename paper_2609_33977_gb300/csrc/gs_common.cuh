@@ -17,6 +17,17 @@ constexpr int kTileBytes = kGroupIn * 2;   // one packed group: 256 bf16 = 512 B
 // Device-error codes written into the library's device flag.
 constexpr int kDevErrTimeout = 1;
 
+// Decode split-reduction scratch of one handle for one stream: gs_linear calls
+// on different streams use different slots, so one handle can serve several
+// streams at once.
+constexpr int kDecSlots = 8;
+struct DecSlot {
+  void* stream;       // cudaStream_t the slot belongs to
+  float* ws;          // [nblk64][dec_nsplit_max][4][16 tokens][16 rows] partial sums
+  int32_t* cnt;       // [nblk64][4] arrival counters, then {unit ticket, finished CTAs} (self-resetting)
+  uint64_t epoch;     // timeout epoch at which the counters were last known clean
+};
+
 }  // namespace gs
 
 // Library-owned packed weight.  All arrays live on `device`.
@@ -38,8 +49,8 @@ struct gs_packed {
   int32_t dec_cpu_fine;   // chunks per unit when the layer is scheduled last (a quarter of that)
   int32_t dec_nsplit_max; // ceil(G / dec_cpu_fine): splits the workspace is sized for
   int4* dmeta;        // [nblk64][G]: {first packed row of the block's slice, kept masks of its 4 windows, 0}
-  float* dec_ws;      // [nblk64][dec_nsplit_max][4][16 tokens][16 rows] partial sums
-  int32_t* dec_cnt;   // [nblk64][4] arrival counters, then {unit ticket, finished CTAs} (self-resetting)
+  gs::DecSlot dec_slot[gs::kDecSlots];   // per-stream split scratch; slot 0 is made for gs_pack's stream
+  int32_t dec_nslots;
   // tcgen05 prefill: slab TMA descriptors over the tiles, box heights 16, 32, ..., 160 rows
   alignas(64) unsigned char wmaps[10][128];
   alignas(64) unsigned char wmaps_full[10][128];   // same, box heights 16, 32, ..., 160 (whole slices)
@@ -59,9 +70,20 @@ bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t o
 bool encode_tmap_slabs_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows, uint32_t box_rows,
                             uint32_t box_slabs);
 
-// library-owned per-device error flag (allocated on first use)
+// library-owned per-device flags (allocated on first use): [0] the error flag
+// gs_device_status reads, [1] a word nothing ever sets (test-injected waits)
 int* device_error_flag();
 void note_launch(int64_t n = 1);
+// Incremented each time gs_device_status reports a timeout: scratch whose
+// arrival counters were last cleaned at an older epoch is re-zeroed first.
+uint64_t timeout_epoch();
+// Every device allocation of the library goes through here (so that a test can
+// make the n-th one fail); OOM on cudaErrorMemoryAllocation, else CUDA.
+gs_status lib_malloc(void** ptr, size_t bytes);
+// Test hook: limit of a wait on the never-set word to inject into the next
+// launch of a kernel family (GS_ALGO_DECODE / GS_ALGO_PREFILL); 0 = none.
+// Reading it disarms it.
+uint64_t take_injected_wait(int family);
 
 // pack.cu
 gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t s, int32_t* cnt_tmp);
@@ -74,6 +96,8 @@ gs_status launch_select(const float* logits, int64_t n, uint8_t* mask, int64_t* 
 // decode.cu
 gs_status decode_prepare(gs_packed* p, cudaStream_t s);   // allocates + builds the decode metadata
 void decode_release(gs_packed* p);
+// split scratch of handle p for stream s (made on first use; re-zeroed after a timeout)
+gs_status decode_slot(const gs_packed* p, cudaStream_t s, const DecSlot** slot);
 gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void* const* ys, int n, int T,
                         cudaStream_t s);
 int decode_max_tokens();

@@ -109,6 +109,7 @@ struct DecParams {
   int32_t n_units;
   int32_t* sched;        // {next unit ticket, finished CTAs}: zero between launches
   int* err;
+  uint64_t inject_ns;    // test hook: CTA 0 first waits this long on a word nothing sets (0 = off)
 };
 
 // Weight slices are read once per launch: the evict-first L2 policy keeps
@@ -208,7 +209,23 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
     lay[threadIdx.x] = make_int4(L.unit_begin, L.nsplit, L.cpu, L.G);
     lay_dmeta[threadIdx.x] = L.dmeta;
   }
+  if (P.inject_ns != 0 && blockIdx.x == 0 && threadIdx.x == 0) {
+    // test hook: a bounded wait on a word that nothing sets (the flag word
+    // after the error flag) runs out before this CTA issues anything; the CTA
+    // then records the timeout and skips all its units
+    const volatile int* never = P.err + 1;
+    const uint64_t t0 = globaltimer_ns();
+    while (*never == 0) {
+      if (globaltimer_ns() - t0 > P.inject_ns) {
+        atomicExch(P.err, kDevErrTimeout);
+        abort_s = 1;
+        break;
+      }
+      __nanosleep(1000);
+    }
+  }
   __syncthreads();
+  const bool injected_abort = abort_s != 0;
   // Programmatic dependent launch: the next launch in the stream may become
   // resident as soon as SM slots free up.  Before touching anything the grid
   // before it may write (x may be its y; the ticket counter and split
@@ -220,7 +237,9 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
   volatile int* abort_flag = &abort_s;
   const int T = P.T;
 
-  if (warp == kCW) {
+  if (injected_abort) {
+    // nothing was issued: fall through to the end of the launch
+  } else if (warp == kCW) {
     // ------------------------------------------------------------ producer warp
     uint32_t q = 0;              // chunks issued so far (ring sequence number)
     uint32_t oldest = 0;         // oldest chunk not yet known to be released
@@ -562,6 +581,8 @@ __global__ void k_pack_decode_meta(const int32_t* __restrict__ win_off16, const 
                        (int)(km[2] | (km[3] << 16)), 0);
 }
 
+std::mutex g_slot_mu;
+
 int sm_count_dec() {
   static int n = 0;
   if (n == 0) {
@@ -613,14 +634,16 @@ gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
   p->dec_cpu_fine = std::max(1, cpu / 4);
   p->dec_nsplit_max = (p->G + p->dec_cpu_fine - 1) / p->dec_cpu_fine;
   const size_t nmeta = (size_t)p->nblk64 * (size_t)p->G;
-  if (cudaMalloc(&p->dmeta, nmeta * sizeof(int4)) != cudaSuccess) return GS_ERR_OOM;
+  {
+    const gs_status am = lib_malloc(reinterpret_cast<void**>(&p->dmeta), nmeta * sizeof(int4));
+    if (am != GS_OK) return am;
+  }
   p->device_bytes += nmeta * sizeof(int4);
-  const size_t nws = (size_t)p->nblk64 * p->dec_nsplit_max * kDW * kPartFloats;
-  const size_t ncnt = (size_t)p->nblk64 * kDW + 2;   // + {unit ticket, finished CTAs}
-  if (cudaMalloc(&p->dec_ws, nws * sizeof(float)) != cudaSuccess) return GS_ERR_OOM;
-  if (cudaMalloc(&p->dec_cnt, ncnt * sizeof(int32_t)) != cudaSuccess) return GS_ERR_OOM;
-  if (cudaMemsetAsync(p->dec_cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) return GS_ERR_CUDA;
-  p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
+  // the split scratch of gs_pack's stream is made now (gs_linear on that
+  // stream then never allocates); other streams get theirs on first use
+  const DecSlot* slot = nullptr;
+  const gs_status st = decode_slot(p, s, &slot);
+  if (st != GS_OK) return st;
   const int64_t n = (int64_t)nmeta;
   k_pack_decode_meta<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p->win_off16, p->kmask16, p->G, p->nw16, p->nblk64,
                                                            p->dmeta);
@@ -630,11 +653,48 @@ gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
 
 void decode_release(gs_packed* p) {
   if (p->dmeta) cudaFree(p->dmeta);
-  if (p->dec_ws) cudaFree(p->dec_ws);
-  if (p->dec_cnt) cudaFree(p->dec_cnt);
   p->dmeta = nullptr;
-  p->dec_ws = nullptr;
-  p->dec_cnt = nullptr;
+  std::lock_guard<std::mutex> lk(g_slot_mu);
+  for (int i = 0; i < p->dec_nslots; ++i) {
+    if (p->dec_slot[i].ws) cudaFree(p->dec_slot[i].ws);
+    if (p->dec_slot[i].cnt) cudaFree(p->dec_slot[i].cnt);
+    p->dec_slot[i] = DecSlot{};
+  }
+  p->dec_nslots = 0;
+}
+
+gs_status decode_slot(const gs_packed* pc, cudaStream_t s, const DecSlot** out) {
+  gs_packed* p = const_cast<gs_packed*>(pc);   // the slot table is the only mutable part of a handle
+  const size_t nws = (size_t)p->nblk64 * p->dec_nsplit_max * kDW * kPartFloats;
+  const size_t ncnt = (size_t)p->nblk64 * kDW + 2;   // + {unit ticket, finished CTAs}
+  const uint64_t epoch = timeout_epoch();
+  std::lock_guard<std::mutex> lk(g_slot_mu);
+  DecSlot* slot = nullptr;
+  for (int i = 0; i < p->dec_nslots; ++i)
+    if (p->dec_slot[i].stream == static_cast<void*>(s)) slot = &p->dec_slot[i];
+  if (!slot) {
+    if (p->dec_nslots >= kDecSlots) return GS_ERR_UNSUPPORTED;
+    DecSlot n{};
+    n.stream = static_cast<void*>(s);
+    gs_status st = lib_malloc(reinterpret_cast<void**>(&n.ws), nws * sizeof(float));
+    if (st == GS_OK) st = lib_malloc(reinterpret_cast<void**>(&n.cnt), ncnt * sizeof(int32_t));
+    if (st == GS_OK && cudaMemsetAsync(n.cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) st = GS_ERR_CUDA;
+    if (st != GS_OK) {
+      if (n.ws) cudaFree(n.ws);
+      if (n.cnt) cudaFree(n.cnt);
+      return st;
+    }
+    n.epoch = epoch;
+    p->dec_slot[p->dec_nslots] = n;
+    slot = &p->dec_slot[p->dec_nslots++];
+    p->device_bytes += nws * sizeof(float) + ncnt * sizeof(int32_t);
+  } else if (slot->epoch != epoch) {
+    // a timed-out launch may have left arrival counters or the ticket half counted
+    if (cudaMemsetAsync(slot->cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) return GS_ERR_CUDA;
+    slot->epoch = epoch;
+  }
+  *out = slot;
+  return GS_OK;
 }
 
 gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void* const* ys, int n, int T,
@@ -666,17 +726,22 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
   P.err = device_error_flag();
   if (!P.err) return GS_ERR_CUDA;
   int64_t units = 0;
+  const DecSlot* first_slot = nullptr;
   for (int k = 0; k < n; ++k) {
     const gs_packed* p = ps[order[k]];
     DecLayer& L = P.L[k];
+    const DecSlot* slot = nullptr;
+    const gs_status st = decode_slot(p, s, &slot);
+    if (st != GS_OK) return st;
+    if (order[k] == 0) first_slot = slot;
     L.x = static_cast<const uint16_t*>(xs[order[k]]);
     if (!encode_tmap_slabs_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)T, (uint32_t)(kGroupIn / 64)))
       return GS_ERR_CUDA;
     L.tiles = p->tiles;
     L.dmeta = p->dmeta;
     L.y = static_cast<uint16_t*>(ys[order[k]]);
-    L.ws = p->dec_ws;
-    L.cnt = p->dec_cnt;
+    L.ws = slot->ws;
+    L.cnt = slot->cnt;
     L.out = (int32_t)p->out;
     L.in = (int32_t)p->in;
     L.G = p->G;
@@ -688,7 +753,8 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
   }
   if (units > INT32_MAX) return GS_ERR_UNSUPPORTED;
   P.n_units = (int32_t)units;
-  P.sched = ps[0]->dec_cnt + (size_t)ps[0]->nblk64 * kDW;
+  P.sched = first_slot->cnt + (size_t)ps[0]->nblk64 * kDW;
+  P.inject_ns = take_injected_wait(GS_ALGO_DECODE);
   const int grid = (int)std::min<int64_t>(units, max_grid);
   cudaError_t e;
   if (n <= kSmallBatch) {
@@ -699,6 +765,7 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     Q.n_units = P.n_units;
     Q.sched = P.sched;
     Q.err = P.err;
+    Q.inject_ns = P.inject_ns;
     e = T <= 8 ? launch_nt<1>(Q, grid, s) : launch_nt<2>(Q, grid, s);
   } else {
     e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);

@@ -113,6 +113,7 @@ struct PrefillParams {
   PrefillLayer L[kMaxLayers];
   int32_t n_layers, T, n_tiles;
   int* err;
+  uint64_t inject_ns;        // test hook: tile owner 0 first waits this long on a word nothing sets (0 = off)
 };
 
 // layer of global tile t
@@ -267,7 +268,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
   const int pair = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
   const int n_pairs = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
-  if (warp == 0) {
+  if (P.inject_ns != 0 && pair == 0) {
+    // test hook: before any copy or MMA is issued, a bounded wait on a word
+    // that nothing sets runs out in each CTA of tile owner 0; the owner then
+    // records the timeout and skips its tiles (every role, both CTAs)
+    if (threadIdx.x == 0) {
+      const volatile int* never = P.err + 1;
+      const uint64_t t0 = globaltimer_ns();
+      while (*never == 0) {
+        if (globaltimer_ns() - t0 > P.inject_ns) {
+          atomicExch(P.err, kDevErrTimeout);
+          abort_s = 1;
+          break;
+        }
+        __nanosleep(1000);
+      }
+    }
+    __syncthreads();
+  }
+  const bool injected_abort = pair == 0 && abort_s != 0;
+
+  if (injected_abort) {
+    // nothing was issued: go straight to the TMEM release
+  } else if (warp == 0) {
     // ------------------------------------------------------------ producer
     uint32_t stage = 0, phase = 0;
     uint32_t armed = 0u, armed_par = 0u;   // per stage: a copy was issued / the phase it completes
@@ -630,6 +653,7 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
     P.T = (int32_t)T;
     P.n_tiles = (int32_t)tiles;
     P.err = err;
+    P.inject_ns = b0 == 0 ? take_injected_wait(GS_ALGO_PREFILL) : 0;
     cudaError_t e;
     if (pair) {
       const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs: clusters of two

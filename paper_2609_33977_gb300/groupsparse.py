@@ -45,8 +45,12 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib.gs_device_status.argtypes = [vp]
     lib.gs_launch_count.argtypes = []
     lib.gs_launch_count.restype = ctypes.c_int64
+    lib.gs_preserved_rates.argtypes = [i32, vp, vp, vp, i64, vp, vp, i32, vp, vp]
+    lib.gs_debug_fail_alloc.argtypes = [i64]
+    lib.gs_debug_inject_wait.argtypes = [ctypes.c_int, ctypes.c_uint64]
     for fn in (lib.gs_pack, lib.gs_linear, lib.gs_linear_ex, lib.gs_linear_batched, lib.gs_unpack,
-               lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status, lib.gs_select_groups):
+               lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status, lib.gs_select_groups,
+               lib.gs_preserved_rates, lib.gs_debug_fail_alloc, lib.gs_debug_inject_wait):
         fn.restype = ctypes.c_int
     return lib
 
@@ -229,37 +233,52 @@ _QKV = {"q": "q", "k": "k", "v": "v", "q_proj": "q", "k_proj": "k", "v_proj": "v
 
 def preserved_report(kept: Sequence[int], shapes: Sequence[Sequence[int]],
                      names: Optional[Sequence[str]] = None, group: int = 256) -> dict:
-    """Preserved rates of exported masks (App. F) from per-layer kept-group counts.
-
-    Each layer's rate is its active weights over its total weights, kept * group /
-    (d_out d_in); the global rate is 1 - s of Eq. 2 (all active weights over all
-    target weights).  With names, layers whose last dotted component is q, k and v
-    (or q_proj, k_proj, v_proj) under one prefix are also reported as the plain mean
-    of their three rates, keyed by that prefix."""
+    """Preserved rates of exported masks (App. F) from per-layer kept-group counts,
+    computed by gs_preserved_rates: each layer's active over total weights, the
+    global rate (1 - s of Eq. 2) and, for layers named q, k and v (or q_proj,
+    k_proj, v_proj) under one dotted prefix, the mean of the three, keyed by
+    that prefix.  This function only arranges the arguments."""
     if len(kept) != len(shapes) or (names is not None and len(names) != len(kept)):
         raise ValueError("kept, shapes (and names) must have the same length")
     names = list(names) if names is not None else [str(i) for i in range(len(kept))]
-    rates = {}
-    active = total = 0
-    for n, k, (d_out, d_in) in zip(names, kept, shapes):
-        k, size = int(k), int(d_out) * int(d_in)
-        if k < 0 or k * group > size:
-            raise ValueError(f"{n}: {k} kept groups do not fit a {d_out} x {d_in} layer")
-        rates[n] = k * group / size
-        active += k * group
-        total += size
-    qkv = {}
-    for n in names:
-        prefix, _, last = n.rpartition(".")
-        if _QKV.get(last) == "q":
-            trio = {}
-            for m in names:
-                p2, _, l2 = m.rpartition(".")
-                if p2 == prefix and l2 in _QKV:
-                    trio[_QKV[l2]] = rates[m]
-            if len(trio) == 3:
-                qkv[prefix] = (trio["q"] + trio["k"] + trio["v"]) / 3.0
-    return {"layers": rates, "global": active / total if total else 0.0, "qkv": qkv}
+    n = len(kept)
+    k_arr = np.ascontiguousarray(kept, dtype=np.int64)
+    sh = np.asarray(shapes, dtype=np.int64).reshape(n, 2)
+    d_out = np.ascontiguousarray(sh[:, 0])
+    d_in = np.ascontiguousarray(sh[:, 1])
+    index = {m: i for i, m in enumerate(names)}
+    prefixes, triples = [], []
+    for m in names:
+        prefix, _, last = m.rpartition(".")
+        if _QKV.get(last) != "q":
+            continue
+        trio = {}
+        for m2 in names:
+            p2, _, l2 = m2.rpartition(".")
+            if p2 == prefix and l2 in _QKV:
+                trio[_QKV[l2]] = index[m2]
+        if len(trio) == 3:
+            prefixes.append(prefix)
+            triples.append((trio["q"], trio["k"], trio["v"]))
+    qkv_idx = np.ascontiguousarray(np.asarray(triples, dtype=np.int32).reshape(-1, 3))
+    rates = np.zeros(max(n, 1), np.float64)
+    qkv_rates = np.zeros(max(len(triples), 1), np.float64)
+    glob = ctypes.c_double()
+    _check(lib.gs_preserved_rates(n, k_arr.ctypes.data, d_out.ctypes.data, d_in.ctypes.data, int(group),
+                                  rates.ctypes.data, ctypes.byref(glob), len(triples), qkv_idx.ctypes.data,
+                                  qkv_rates.ctypes.data), "gs_preserved_rates")
+    return {"layers": {m: float(rates[i]) for i, m in enumerate(names)}, "global": glob.value,
+            "qkv": {pf: float(qkv_rates[j]) for j, pf in enumerate(prefixes)}}
+
+
+def debug_fail_alloc(nth: int) -> None:
+    """Test hook: the nth device allocation the library makes from now on fails (0 disarms)."""
+    _check(lib.gs_debug_fail_alloc(int(nth)), "gs_debug_fail_alloc")
+
+
+def debug_inject_wait(algo: int, limit_ns: int) -> None:
+    """Test hook: the next launch of that kernel family times out on a word nothing sets."""
+    _check(lib.gs_debug_inject_wait(int(algo), int(limit_ns)), "gs_debug_inject_wait")
 
 
 def device_status(stream: Optional[torch.cuda.Stream] = None) -> int:

@@ -107,3 +107,52 @@ def test_header_is_plain_c(tmp_path):
                 [gcc, "-x", "c++", "-std=c++17", "-Wall", "-Wextra", "-Werror"]):
         r = subprocess.run(cmd + [f"-I{ROOT / 'include'}", "-fsyntax-only", str(src)], capture_output=True, text=True)
         assert r.returncode == 0, r.stderr
+
+
+def test_preserved_rates_call(lib):
+    # App. F arithmetic lives in the library (host only, no device work):
+    # exact per-layer rates, the Eq. 2 global rate and the Q/K/V plain mean
+    import numpy as np
+    from oracle import groupsparse_oracle as orc
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    lib.gs_preserved_rates.argtypes = [i32, vp, vp, vp, i64, vp, vp, i32, vp, vp]
+    rng = np.random.default_rng(11)
+    shapes = [(48, 512), (16, 512), (16, 512), (32, 768), (64, 1024)]
+    Bs = [(rng.random((o, i // 256)) < 0.45).astype(np.uint8) for o, i in shapes]
+    kept = np.array([int(B.sum()) for B in Bs], np.int64)
+    d_out = np.array([s[0] for s in shapes], np.int64)
+    d_in = np.array([s[1] for s in shapes], np.int64)
+    qkv = np.array([[0, 1, 2], [2, 1, 0]], np.int32)
+    rates = np.zeros(5)
+    qrates = np.zeros(2)
+    glob = ctypes.c_double()
+    assert lib.gs_preserved_rates(5, kept.ctypes.data, d_out.ctypes.data, d_in.ctypes.data, 256, rates.ctypes.data,
+                                  ctypes.byref(glob), 2, qkv.ctypes.data, qrates.ctypes.data) == 0
+    for i, B in enumerate(Bs):
+        assert rates[i] == orc.preserved_rate(B)
+    assert glob.value == pytest.approx(orc.global_preserved_rate(Bs, shapes), abs=1e-15)
+    assert qrates[0] == pytest.approx(orc.qkv_preserved_rate(Bs[0], Bs[1], Bs[2]), abs=1e-15)
+    assert qrates[1] == pytest.approx(orc.qkv_preserved_rate(Bs[2], Bs[1], Bs[0]), abs=1e-15)
+    INVALID = 1
+    bad = kept.copy()
+    bad[3] = 32 * 3 + 1                      # more kept groups than the layer holds
+    assert lib.gs_preserved_rates(5, bad.ctypes.data, d_out.ctypes.data, d_in.ctypes.data, 256, None, None, 0,
+                                  None, None) == INVALID
+    neg = np.array([[0, 1, 5]], np.int32)    # index out of range
+    assert lib.gs_preserved_rates(5, kept.ctypes.data, d_out.ctypes.data, d_in.ctypes.data, 256, None, None, 1,
+                                  neg.ctypes.data, qrates.ctypes.data) == INVALID
+    assert lib.gs_preserved_rates(1, None, d_out.ctypes.data, d_in.ctypes.data, 256, None, None, 0, None,
+                                  None) == INVALID
+    assert lib.gs_preserved_rates(0, None, None, None, 256, None, ctypes.byref(glob), 0, None, None) == 0
+    assert glob.value == 0.0
+
+
+def test_debug_hooks_validate_arguments(lib):
+    lib.gs_debug_fail_alloc.argtypes = [ctypes.c_int64]
+    lib.gs_debug_inject_wait.argtypes = [ctypes.c_int, ctypes.c_uint64]
+    INVALID = 1
+    assert lib.gs_debug_fail_alloc(-1) == INVALID
+    assert lib.gs_debug_fail_alloc(0) == 0
+    assert lib.gs_debug_inject_wait(0, 1000) == INVALID          # AUTO is not a kernel family
+    assert lib.gs_debug_inject_wait(1, 2_000_000_000) == INVALID  # above 1 s
+    assert lib.gs_debug_inject_wait(1, 0) == 0 and lib.gs_debug_inject_wait(2, 0) == 0

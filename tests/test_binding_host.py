@@ -67,5 +67,6 @@ def test_preserved_report_against_oracle():
     assert rep["qkv"] == {"b1": pytest.approx(orc.qkv_preserved_rate(*Bs[:3]), abs=1e-15)}
     # no complete q/k/v trio, no QKV entry; a count that cannot fit is refused
     assert gs.preserved_report([1], [(1, 256)], ["x.q"])["qkv"] == {}
-    with pytest.raises(ValueError, match="fit"):
+    with pytest.raises(gs.GroupSparseError) as e:
         gs.preserved_report([3], [(2, 256)])
+    assert e.value.status == gs.GS_ERR_INVALID_ARG
