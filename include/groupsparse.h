@@ -91,11 +91,12 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
  *        gs_linear / gs_linear_ex / gs_linear_batched calls on several streams
  *        at once.  The decode kernel's split-reduction scratch is kept per
  *        (handle, stream): the scratch of gs_pack's stream is made by gs_pack,
- *        and the first decode-regime call on any other stream allocates that
- *        stream's (so make it before capturing that stream into a CUDA graph).
- *        Up to 8 streams per handle.  Calls on one stream are ordered by the
- *        stream; a CUDA graph keeps the scratch of the stream it was captured
- *        from, so its replays must be ordered with other work on that stream.
+ *        and the first decode-regime call on any other stream allocates and
+ *        zeroes that stream's, synchronously and outside any graph capture
+ *        in progress on it.  Up to 8 streams per handle.  Calls on one stream
+ *        are ordered by the stream; a CUDA graph keeps the scratch of the
+ *        stream it was captured from, so its replays must be ordered with
+ *        other work on that stream.
  * T      number of tokens; T == 0 is a no-op, T < 0 is INVALID_ARG.
  * y_dev  bf16 [T][out] row-major, caller-owned; fully overwritten (rows of
  *        outputs with no kept group are written as +0.0).

@@ -676,9 +676,22 @@ gs_status decode_slot(const gs_packed* pc, cudaStream_t s, const DecSlot** out) 
     if (p->dec_nslots >= kDecSlots) return GS_ERR_UNSUPPORTED;
     DecSlot n{};
     n.stream = static_cast<void*>(s);
+    // The stream may be capturing a CUDA graph (e.g. a capture side stream that
+    // has not run a decode call before).  The slot is made outside the capture:
+    // this thread's capture mode is relaxed while the buffers are allocated and
+    // zeroed on a private non-blocking stream, then restored.
+    cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
+    if (cudaThreadExchangeStreamCaptureMode(&mode) != cudaSuccess) return GS_ERR_CUDA;
     gs_status st = lib_malloc(reinterpret_cast<void**>(&n.ws), nws * sizeof(float));
     if (st == GS_OK) st = lib_malloc(reinterpret_cast<void**>(&n.cnt), ncnt * sizeof(int32_t));
-    if (st == GS_OK && cudaMemsetAsync(n.cnt, 0, ncnt * sizeof(int32_t), s) != cudaSuccess) st = GS_ERR_CUDA;
+    if (st == GS_OK) {
+      cudaStream_t zs = nullptr;
+      if (cudaStreamCreateWithFlags(&zs, cudaStreamNonBlocking) != cudaSuccess ||
+          cudaMemsetAsync(n.cnt, 0, ncnt * sizeof(int32_t), zs) != cudaSuccess || cudaStreamSynchronize(zs) != cudaSuccess)
+        st = GS_ERR_CUDA;
+      if (zs) cudaStreamDestroy(zs);
+    }
+    cudaThreadExchangeStreamCaptureMode(&mode);
     if (st != GS_OK) {
       if (n.ws) cudaFree(n.ws);
       if (n.cnt) cudaFree(n.cnt);
