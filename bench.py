@@ -1,17 +1,29 @@
 #!/usr/bin/env python
 """Throughput benchmark of the group-sparse linear layer y = x (W (.) M)^T.
 
-Workload: one LLaMA-2-7B-shaped decoder block (q/k/v/o 4096x4096, gate/up
-11008x4096, down 4096x11008), bf16 weights ~ N(0, 0.02^2), 1x256 groups along
-the input dimension, per-module keep ratios U[0.3, 0.7] rescaled so the block
-keeps exactly 50 % of its 790,528 groups, decode batches of 1, 4 and 16 tokens.
+Headline workload: the full LLaMA-2-13B-shaped linear stack (40 blocks of
+q/k/v/o 5120x5120, gate/up 13824x5120, down 5120x13824; 280 layers, bf16
+weights ~ N(0, 0.02^2), 1x256 groups along the input dimension, per-layer keep
+ratios U[0.2, 0.8] rescaled so the stack keeps exactly 50 % of its 49,561,600
+groups: 12.69 GB of kept weights).  This is the largest configuration of the
+five; it fits one GB300.
 
-One step = the seven projections at T = 1, 4 and 16 (three batched launches of
-the decode kernel, 21 tokens through the block), on one of R rotated packed
-copies so that the weights streamed per step never sit in L2.  Packing is a
-one-time transform of frozen weights and is timed separately ("pack").  The
-tensor-core prefill kernel is measured on the first block of the 7B stack at
-T = 2048 with activation outliers ("prefill").
+One step = one decode pass over the whole stack at T = 1 and one at T = 16
+(17 tokens): per pass one gs_linear_batched call per block (the block's 7
+projections share one launch), captured as one CUDA graph per step.  The
+stack's kept weights (12.7 GB) are far larger than L2, so every pass streams
+them from HBM.  tokens/s = tokens per step / step time, which is T / (sum of
+the layer times) per pass.  Packing is a one-time transform of frozen weights
+and is timed separately ("pack").
+
+Extra keys (N = 1 only): per-T decode passes, the same passes with one call per
+layer, the tensor-core prefill over the whole 13B stack at T = 128, 512 and
+2048, the whole LLaMA-2-7B stack at T = 2048 with activation outliers, the
+whole Qwen2.5-7B stack at densities 0.3 / 0.5 / 0.7 (decode T = 1, prefill
+T = 1024), the single 1024x1024 layer at T = 8 (a graph over 256 rotated
+packed copies), one LLaMA-2-7B block at T = 1, 4, 16, the selector export,
+dense bf16 torch matmuls on unpruned weights as reference points, and the CPU
+oracle on a bounded sample.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -39,7 +51,11 @@ sys.path.insert(0, str(ROOT))
 from paper_2609_33977_gb300 import workload as wl  # noqa: E402
 
 METRIC = "group-sparse linear tokens/s; decode HBM GB/s and prefill TFLOP/s vs GB300 peak"
-DECODE_T = (1, 4, 16)
+HEADLINE_CFG = 4            # the LLaMA-2-13B-shaped stack, 40 blocks
+DECODE_T = (1, 16)          # decode token counts of the headline step
+PREFILL_T = (128, 512, 2048)
+BLOCK_T = (1, 4, 16)        # the single LLaMA-2-7B block (second configuration)
+NOMINAL_HBM_GBS = 8000.0    # the ~8 TB/s nominal HBM3e bandwidth the target is stated against
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -144,81 +160,205 @@ def recorded_traffic(kernel: str, source: str, workload: str):
     return None
 
 
-# ----------------------------------------------------------------------------- workload
-def block_inputs():
-    w = wl.workload(2)
-    k = wl.keep_counts(w)
-    layers = []
-    for i, L in enumerate(w.layers):
-        layers.append({"L": L, "k": int(k[i]), "W": wl.weight_bits(w, i), "B": wl.group_mask(w, i, int(k[i])),
-                       "x": {T: wl.activation_bits(w, i, T) for T in DECODE_T}})
-    return w, layers
+
+# ----------------------------------------------------------------------------- algorithmic work
+def layer_decode_bytes(L, k: int, T: int) -> int:
+    """Bytes one decode pass moves for one layer: kept weights, the index metadata
+    the kernel reads (16-bit window mask + 32-bit offset per chunk x 16-row window),
+    x and y."""
+    return 512 * int(k) + 6 * L.G * ((L.out + 15) // 16) + 2 * T * (L.inp + L.out)
 
 
-def decode_bytes(layers, T):
-    """Algorithmic bytes of one decode launch over the block: kept weights + the index
-    metadata the kernel reads (16-bit window mask + 32-bit offset per chunk x 16-row
-    window) + x + y."""
-    b = 0
-    for d in layers:
-        L = d["L"]
-        nw16 = (L.out + 15) // 16
-        b += 512 * d["k"] + 6 * L.G * nw16 + 2 * T * L.inp + 2 * T * L.out
-    return b
+def stack_decode_bytes(layers, ks, T: int) -> int:
+    return sum(layer_decode_bytes(L, k, T) for L, k in zip(layers, ks))
+
+
+def kept_flops(ks, T: int) -> float:
+    """Kept FLOPs of a pass: 2 T 256 per kept group (pruned groups cost nothing)."""
+    return 2.0 * T * 256 * float(sum(int(k) for k in ks))
+
+
+# ----------------------------------------------------------------------------- packed stacks
+class Stack:
+    """Every layer of a workload packed on the device.  Weights are drawn on the
+    device (torch Philox seeded from the workload's SeedSequence), masks on the host
+    (numpy top-k of seeded scores, several layers at once in a thread pool); each
+    dense weight is freed once packed."""
+
+    def __init__(self, gs, torch, dev, w, pool, blocks_of: int = 7):
+        self.w = w
+        self.layers = list(w.layers)
+        ks = wl.keep_counts(w)
+        futs = [pool.submit(wl.group_mask, w, i, int(ks[i])) for i in range(len(self.layers))]
+        self.packs = []
+        pack_s = 0.0
+        for i in range(len(self.layers)):
+            W = wl.weight_device(w, i, device=dev)
+            M = torch.from_numpy(futs[i].result()).to(dev)
+            torch.cuda.synchronize(dev)
+            t0 = time.perf_counter()
+            self.packs.append(gs.pack(W, M))
+            torch.cuda.synchronize(dev)
+            pack_s += time.perf_counter() - t0
+            del W, M
+        self.kept = [p.kept for p in self.packs]
+        assert sum(self.kept) == w.budget, (sum(self.kept), w.budget)
+        assert self.kept == [int(k) for k in ks]
+        self.pack_s = pack_s
+        n = len(self.layers)
+        self.blocks = [list(range(b, min(n, b + blocks_of))) for b in range(0, n, blocks_of)]
+        torch.cuda.empty_cache()
+
+    @property
+    def kept_groups(self) -> int:
+        return int(sum(self.kept))
+
+    def pack_bytes(self) -> int:
+        """HBM bytes of packing: kept W read + tiles written + mask + metadata + row indices."""
+        return sum(1024 * k + L.groups + 6 * L.G * ((L.out + 15) // 16) + 4 * k for L, k in zip(self.layers, self.kept))
+
+    def free(self):
+        for p in self.packs:
+            p.free()
+        self.packs = []
+
+
+def stack_inputs(torch, w, dev, T: int):
+    xs = [wl.activation_device(w, i, T, device=dev) for i in range(len(w.layers))]
+    ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
+    return xs, ys
+
+
+def stack_pass(gs, S, xs, ys, stream, per_layer: bool = False):
+    """One pass over the stack: one batched call per block (or one call per layer)."""
+    if per_layer:
+        for i, p in enumerate(S.packs):
+            gs.linear_into(xs[i], p, ys[i], stream=stream)
+        return
+    for blk in S.blocks:
+        gs.linear_batched_into([xs[i] for i in blk], [S.packs[i] for i in blk], [ys[i] for i in blk], stream=stream)
+
+
+def capture(torch, stream, fn):
+    """A CUDA graph of fn() (launches on `stream`); fn runs once first, outside capture."""
+    with torch.cuda.stream(stream):
+        fn()
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    stream.synchronize()
+    return g
+
+
+def time_replays(torch, stream, graphs, reps: int, warm: int = 3) -> float:
+    """Seconds per graph replay (CUDA events on `stream`, replays cycling over `graphs`)."""
+    with torch.cuda.stream(stream):
+        for i in range(warm):
+            graphs[i % len(graphs)].replay()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(reps):
+            graphs[i % len(graphs)].replay()
+        b.record(stream)
+        b.synchronize()
+    return a.elapsed_time(b) / 1e3 / reps
+
+
+def time_calls(torch, stream, fn, reps: int, warm: int = 1) -> float:
+    """Seconds per fn() (launches on `stream`, no graph)."""
+    with torch.cuda.stream(stream):
+        for _ in range(warm):
+            fn()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        b.synchronize()
+    return a.elapsed_time(b) / 1e3 / reps
+
+
+def dense_block_seconds(torch, w, dev, stream, T: int, reps: int = 10, block: int = 0) -> float:
+    """Seconds per pass of dense bf16 torch.matmul over one block's unpruned weights
+    (the reference point; a block's dense weights are larger than L2)."""
+    ids = list(range(7 * block, 7 * block + 7))
+    Wd = [wl.weight_device(w, i, device=dev) for i in ids]
+    xd = [wl.activation_device(w, i, T, device=dev) for i in ids]
+
+    def run():
+        for W, x in zip(Wd, xd):
+            torch.matmul(x, W.t())
+    s = time_calls(torch, stream, run, reps, warm=2)
+    del Wd, xd
+    torch.cuda.empty_cache()
+    return s
 
 
 # ----------------------------------------------------------------------------- CPU oracle timing
-def oracle_sample_rate(layers, seconds: float, rows_per_call: int = 256):
+def oracle_block_inputs(cfg: int = HEADLINE_CFG):
+    """Host (numpy) copies of block 0 of a stack: the sample the CPU oracle is timed on."""
+    w = wl.workload(cfg)
+    ks = wl.keep_counts(w)
+    layers = []
+    for i in range(7):
+        layers.append({"L": w.layers[i], "W": wl.weight_bits(w, i), "B": wl.group_mask(w, i, int(ks[i])),
+                       "x1": wl.activation_bits(w, i, 1)})
+    return w, layers
+
+
+def oracle_sample_rate(w, layers, seconds: float, rows_per_call: int = 256):
     """Times the fp64 oracle on bounded samples: one token through `rows_per_call`
-    output rows of one projection per call, rotating over the projections, for
-    about `seconds`.  Returns block tokens/s extrapolated by weight count."""
+    output rows of one projection of block 0 per call, rotating over its 7
+    projections, for about `seconds`.  Returns stack tokens/s extrapolated by
+    weight count (every block has the same shapes)."""
     from oracle import groupsparse_oracle as orc
-    total_weights = sum(d["L"].out * d["L"].inp for d in layers)
+    total_weights = sum(L.out * L.inp for L in w.layers)
     done_weights = 0
     t_used = 0.0
     calls = 0
-    i = 0
     t_end = time.perf_counter() + seconds
     cpu0 = time.process_time()
     while time.perf_counter() < t_end or calls < len(layers):
-        d = layers[i % len(layers)]
+        d = layers[calls % len(layers)]
         L = d["L"]
         r0 = (calls * 977) % max(1, L.out - rows_per_call)
         rows = slice(r0, r0 + rows_per_call)
-        x1 = d["x"][1]
         t0 = time.perf_counter()
-        orc.linear(x1, d["W"][rows], d["B"][rows])
+        orc.linear(d["x1"], d["W"][rows], d["B"][rows])
         t_used += time.perf_counter() - t0
         done_weights += rows_per_call * L.inp
         calls += 1
-        i += 1
-    sec_per_weight = t_used / done_weights
-    tokens_per_s = 1.0 / (sec_per_weight * total_weights)
+    tokens_per_s = done_weights / t_used / total_weights
     cores = _cores_used(time.process_time() - cpu0, t_used)
-    return {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"{calls} oracle calls, each 1 token x {rows_per_call} output rows of one projection "
-                      f"(rotating over the 7), {t_used:.1f} s wall; block tokens/s extrapolated by "
-                      f"weight count ({total_weights} weights per block); cores = process CPU time / wall "
-                      f"time over the calls"}
+    return {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "host_cpus": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"{calls} oracle calls, each 1 token x {rows_per_call} output rows of one projection of "
+                      f"block 0 (rotating over its 7), {t_used:.1f} s wall; stack tokens/s extrapolated by weight "
+                      f"count ({total_weights} weights in the {len(w.layers)} layers); cores = process CPU time / "
+                      f"wall time over the calls; host_cpus = os.cpu_count()"}
 
 
 def oracle_single_thread_rate(seconds: float):
     """The same bounded oracle sample in a child process whose BLAS and OpenMP
     pools are limited to one thread (the variables must be set before numpy
     loads, hence the child).  The child generates its own copy of the seeded
-    block inputs and touches no GPU."""
+    inputs and touches no GPU."""
     env = dict(os.environ)
     for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
         env[k] = "1"
-    env.pop("RANK", None)
-    env.pop("WORLD_SIZE", None)
+    for k in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
+        env.pop(k, None)
     try:
         r = subprocess.run([sys.executable, str(Path(__file__).resolve()), "--oracle-single-thread", "--warmup", "3",
                             "--cpu-seconds", str(seconds)], env=env, capture_output=True, text=True, timeout=600)
         if r.returncode != 0:
             return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}"}
         d = json.loads(r.stdout.strip().splitlines()[-1])
-        return {"value": d["value"], "unit": d["unit"], "cores": d["cores"], "sample": d["sample"]}
+        return {"value": d["value"], "unit": d["unit"], "cores": d["cores"],
+                "sample": "the same sample in a child process with one BLAS / OpenMP thread"}
     except Exception as e:   # reported in the line, never hidden; the GPU figures stand without it
         return {"error": f"{type(e).__name__}: {e}"}
 
@@ -232,19 +372,22 @@ def _cores_used(cpu_seconds: float, wall_seconds: float) -> int:
 
 # ----------------------------------------------------------------------------- reference arm
 def run_reference(args):
+    """The CPU oracle, as it stands, on the headline workload: each step times the
+    fp64 oracle on one token through a bounded sample of output rows of block 0's
+    projections, extrapolated to the stack by weight count."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    _, layers = block_inputs()
+    w, layers = oracle_block_inputs()
     from oracle import groupsparse_oracle as orc
-    total_weights = sum(d["L"].out * d["L"].inp for d in layers)
+    total_weights = sum(L.out * L.inp for L in w.layers)
     rows_per_step = 64
 
     def one(i):
         d = layers[i % len(layers)]
         L = d["L"]
         r0 = (i * 977) % max(1, L.out - rows_per_step)
-        orc.linear(d["x"][1], d["W"][r0:r0 + rows_per_step], d["B"][r0:r0 + rows_per_step])
+        orc.linear(d["x1"], d["W"][r0:r0 + rows_per_step], d["B"][r0:r0 + rows_per_step])
         return rows_per_step * L.inp
 
     for i in range(args.warmup):
@@ -257,15 +400,15 @@ def run_reference(args):
     dt = time.perf_counter() - t0
     cores = _cores_used(time.process_time() - cpu0, dt)
     tokens_per_s = weights / total_weights / dt
-    sample = (f"each step: the fp64 oracle on 1 token x {rows_per_step} output rows of one projection "
-              f"(rotating over the 7); block tokens/s extrapolated by weight count; cores = process CPU time / "
-              f"wall time")
+    sample = (f"each step: the fp64 oracle on 1 token x {rows_per_step} output rows of one projection of block 0 "
+              f"(rotating over its 7); stack tokens/s extrapolated by weight count; cores = process CPU time / "
+              f"wall time; host_cpus = os.cpu_count()")
     line = {"impl": "reference", "metric": METRIC, "value": tokens_per_s, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / max(1, args.steps),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "llama2-7b-block decode T=1 (sampled rows)", "layers": 7},
-            "cpu_baseline": {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                             "sample": sample},
+            "config": {"workload": f"{w.name} decode, T=1 (sampled rows of block 0)", "layers": len(w.layers)},
+            "cpu_baseline": {"value": tokens_per_s, "unit": "tokens/s", "cores": cores, "host_cpus": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": tokens_per_s, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
@@ -273,6 +416,7 @@ def run_reference(args):
 
 # ----------------------------------------------------------------------------- our arm
 def run_ours(args):
+    import concurrent.futures as cf
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -289,50 +433,29 @@ def run_ours(args):
     from paper_2609_33977_gb300 import groupsparse as gs
 
     peaks, peaks_src = load_peaks()
-    t_gen = time.perf_counter()
-    w, layers = block_inputs()
-    log(f"[bench] inputs generated in {time.perf_counter() - t_gen:.1f}s")
-
-    def dev_bits(a):
-        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
-
-    Wd = [dev_bits(d["W"]) for d in layers]
-    Md = [torch.from_numpy(d["B"]).to(dev) for d in layers]
-
-    # ---- pack (one-time transform), timed on its own
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    packs0 = [gs.pack(Wd[i], Md[i]) for i in range(len(layers))]
-    torch.cuda.synchronize()
-    pack_s = time.perf_counter() - t0
-    kept = sum(p.kept for p in packs0)
-    assert kept == w.budget, (kept, w.budget)
-    pack_bytes = sum(512 * d["k"] * 2 + d["L"].groups + 6 * d["L"].G * ((d["L"].out + 15) // 16) + 4 * d["k"]
-                     for d in layers)
-
-    # ---- rotated copies so each step streams weights that are not L2-resident
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    kept_bytes = 512 * kept
-    R = max(2, int(math.ceil(3 * l2 / kept_bytes)) + 1) if args.rotate <= 0 else args.rotate
-    packs = [packs0] + [[gs.pack(Wd[i], Md[i]) for i in range(len(layers))] for _ in range(R - 1)]
-    xs = {T: [dev_bits(d["x"][T]) for d in layers] for T in DECODE_T}
-    ys = {T: [torch.empty((T, d["L"].out), dtype=torch.bfloat16, device=dev) for d in layers] for T in DECODE_T}
-
+    hbm_peak = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    tpk = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
+    tpk_sus = float(peaks.get("bf16_tflops_sustained", PEAKS_FALLBACK["bf16_tflops_sustained"]))
+    pool = cf.ThreadPoolExecutor(max_workers=8)
     stream = torch.cuda.Stream(device=dev)
-    graphs = []
-    with torch.cuda.stream(stream):
-        for c in range(R):                       # warm-up launches outside capture
-            for T in DECODE_T:
-                gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
-        stream.synchronize()
-        for c in range(R):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                for T in DECODE_T:
-                    gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
-            graphs.append(g)
-    stream.synchronize()
-    launches_per_step = len(DECODE_T)
+
+    # ---- the headline stack, packed once (one-time transform of frozen weights)
+    t_gen = time.perf_counter()
+    w4 = wl.workload(HEADLINE_CFG)
+    S = Stack(gs, torch, dev, w4, pool)
+    log(f"[bench] {w4.name}: {len(S.layers)} layers packed in {time.perf_counter() - t_gen:.1f}s "
+        f"({S.kept_groups} kept groups)")
+    xs = {}
+    ys = {}
+    for T in DECODE_T:
+        xs[T], ys[T] = stack_inputs(torch, w4, dev, T)
+
+    def step():
+        for T in DECODE_T:
+            stack_pass(gs, S, xs[T], ys[T], stream)
+
+    g_step = capture(torch, stream, step)
+    launches_per_step = len(DECODE_T) * len(S.blocks)
 
     def barrier():
         if dist is not None:
@@ -340,8 +463,8 @@ def run_ours(args):
 
     # ---- warm-up, then exactly K timed steps
     with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            graphs[i % R].replay()
+        for _ in range(args.warmup):
+            g_step.replay()
     stream.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
@@ -352,196 +475,99 @@ def run_ours(args):
     n0 = gs.launch_count()
     with torch.cuda.stream(stream):
         ev0.record(stream)
-        for i in range(args.steps):
-            graphs[i % R].replay()
+        for _ in range(args.steps):
+            g_step.replay()
         ev1.record(stream)
     ev1.synchronize()
     torch.cuda.synchronize(dev)
     barrier()
     clock_rec = clocks.stop()
-    # graph replays do not go through the library's launch counter: count the
-    # kernels they contain (one decode launch per token batch per step)
+    # graph replays bypass the library's launch counter: count the kernels they hold
     launches = args.steps * launches_per_step + (gs.launch_count() - n0)
     elapsed = max_over_ranks(ev0.elapsed_time(ev1) / 1e3, dist, dev)
     tokens_per_step = sum(DECODE_T)
     value = whole_job_rate(tokens_per_step, args.steps, elapsed, world)
-    bytes_per_step = sum(decode_bytes(layers, T) for T in DECODE_T)
+    bytes_per_step = sum(stack_decode_bytes(S.layers, S.kept, T) for T in DECODE_T)
     achieved_gbs = bytes_per_step * args.steps / elapsed / 1e9
+    assert gs.device_status() == gs.GS_OK
 
-    # ---- per-T kernel timing (decode alone, one graph per T) for the breakdown
+    # ---- each decode pass alone, per-block batched calls and per-layer calls
     per_T = {}
-    with torch.cuda.stream(stream):
-        for T in DECODE_T:
-            gT = []
-            for c in range(R):
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g, stream=stream):
-                    gs.linear_batched_into(xs[T], packs[c], ys[T], stream=stream)
-                gT.append(g)
-            n = max(50, min(2000, args.steps))
-            for i in range(10):
-                gT[i % R].replay()
-            a = torch.cuda.Event(enable_timing=True)
-            b = torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            for i in range(n):
-                gT[i % R].replay()
-            b.record(stream)
-            b.synchronize()
-            us = a.elapsed_time(b) * 1e3 / n
-            per_T[str(T)] = {"us_per_launch": us, "GB/s": decode_bytes(layers, T) / us / 1e3,
-                             "tokens/s": T / us * 1e6}
-
-    # ---- end to end through the public API with host buffers
-    # One pinned host buffer per direction holds a step's inputs (x of every
-    # projection for T = 1, 4, 16, back to back) and its results.  The device
-    # side alternates between two copies of each, so a step's copies overlap
-    # the neighbouring steps' launches; events order every buffer's reuse.
-    y_len = {T: sum(T * d["L"].out for d in layers) for T in DECODE_T}
-    xh_all = torch.cat([torch.cat([xx.reshape(-1) for xx in xs[T]]) for T in DECODE_T]).cpu().pin_memory()
-    yh_all = torch.empty(sum(y_len.values()), dtype=torch.bfloat16).pin_memory()
-    xd_all = [torch.empty_like(xh_all, device=dev) for _ in range(2)]
-    yd_all = [torch.empty_like(yh_all, device=dev) for _ in range(2)]
-
-    def layer_views(buf, dim):
-        out, off = {}, 0
-        for T in DECODE_T:
-            views = []
-            for d in layers:
-                n = T * getattr(d["L"], dim)
-                views.append(buf[off:off + n].view(T, getattr(d["L"], dim)))
-                off += n
-            out[T] = views
-        return out
-
-    xv = [layer_views(xd_all[k], "inp") for k in range(2)]
-    yv = [layer_views(yd_all[k], "out") for k in range(2)]
-    h2d = xh_all.numel() * 2
-    d2h = yh_all.numel() * 2
-    e2e_steps = max(20, min(args.steps, 2000))
-    h2d_stream = torch.cuda.Stream(device=dev)
-    d2h_stream = torch.cuda.Stream(device=dev)
-    x_ready = [torch.cuda.Event() for _ in range(2)]
-    k_done = [torch.cuda.Event() for _ in range(2)]
-    y_read = [torch.cuda.Event() for _ in range(2)]
-    used = [False, False]
-
-    def e2e_step(i):
-        c, k = i % R, i % 2
-        if used[k]:
-            h2d_stream.wait_event(k_done[k])    # the launches two steps back have read this x buffer
-        with torch.cuda.stream(h2d_stream):
-            xd_all[k].copy_(xh_all, non_blocking=True)
-            x_ready[k].record(h2d_stream)
-        stream.wait_event(x_ready[k])
-        if used[k]:
-            stream.wait_event(y_read[k])        # the copy two steps back has read this y buffer
-        with torch.cuda.stream(stream):
-            for T in DECODE_T:
-                gs.linear_batched_into(xv[k][T], packs[c], yv[k][T], stream=stream)
-            k_done[k].record(stream)
-        d2h_stream.wait_event(k_done[k])
-        with torch.cuda.stream(d2h_stream):
-            yh_all.copy_(yd_all[k], non_blocking=True)
-            y_read[k].record(d2h_stream)
-        used[k] = True
-
-    for i in range(5):
-        e2e_step(i)
-    torch.cuda.synchronize(dev)
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    h2d_stream.wait_event(a)
-    for i in range(e2e_steps):
-        e2e_step(i)
-    stream.wait_event(y_read[(e2e_steps - 1) % 2])    # the last step's results are on the host
-    b.record(stream)
-    b.synchronize()
-    torch.cuda.synchronize(dev)
-    e2e_s = a.elapsed_time(b) / 1e3
-    e2e_value = world * tokens_per_step * e2e_steps / e2e_s
-    # results of the e2e path equal the device-resident path
-    y_dev = torch.cat([torch.cat([yy.reshape(-1) for yy in ys[T]]) for T in DECODE_T])
-    assert torch.equal(yh_all.to(dev), y_dev), "e2e result mismatch"
-
-    # ---- dense bf16 torch matmul on the unpruned weights (reference point)
-    dense = {}
-    with torch.cuda.stream(stream):
-        for T in DECODE_T:
-            Wd_rot = [Wd] + [[wt.clone() for wt in Wd] for _ in range(1)]
-            for i in range(5):
-                for j, d in enumerate(layers):
-                    torch.matmul(xs[T][j], Wd_rot[i % 2][j].t())
-            a = torch.cuda.Event(enable_timing=True)
-            b = torch.cuda.Event(enable_timing=True)
-            n = 50
-            a.record(stream)
-            for i in range(n):
-                for j, d in enumerate(layers):
-                    torch.matmul(xs[T][j], Wd_rot[i % 2][j].t())
-            b.record(stream)
-            b.synchronize()
-            us = a.elapsed_time(b) * 1e3 / n
-            dense[str(T)] = {"us_per_block": us, "tokens/s": T / us * 1e6}
-            del Wd_rot
+    for T in DECODE_T:
+        nb = stack_decode_bytes(S.layers, S.kept, T)
+        s_b = time_replays(torch, stream, [capture(torch, stream, lambda: stack_pass(gs, S, xs[T], ys[T], stream))],
+                           reps=20)
+        s_l = time_replays(torch, stream, [capture(torch, stream,
+                                                   lambda: stack_pass(gs, S, xs[T], ys[T], stream, per_layer=True))],
+                           reps=20)
+        per_T[str(T)] = {"ms_per_pass": s_b * 1e3, "tokens/s": T / s_b, "GB/s": nb / s_b / 1e9,
+                         "frac_of_measured_hbm": nb / s_b / 1e9 / hbm_peak,
+                         "frac_of_8TBs_nominal": nb / s_b / 1e9 / NOMINAL_HBM_GBS,
+                         "launches_per_pass": len(S.blocks),
+                         "per_layer_calls": {"ms_per_pass": s_l * 1e3, "GB/s": nb / s_l / 1e9,
+                                             "launches_per_pass": len(S.layers)}}
     torch.cuda.empty_cache()
+
+    # ---- end to end through the public API with host buffers (no graph)
+    e2e = measure_e2e(gs, torch, dev, stream, S, xs, ys, tokens_per_step, world, args)
 
     # ---- per-GPU characterisations (N = 1 only: at N > 1 every rank would repeat them
     # while all GPUs are held, and they are not part of the scaled metric)
-    # tensor-core prefill on the first block of the 7B stack, T = 2048 (outliers)
-    prefill = None
-    prefill_sweep = None
-    decode_sweep = None
-    mask_export = None
-    if not args.no_prefill and world == 1:
-        prefill = measure_prefill(gs, torch, dev, stream, peaks)
-        prefill_sweep = measure_prefill_sweep(gs, torch, dev, stream, peaks)
-        decode_sweep = measure_decode_sweep(gs, torch, dev, stream, peaks)
-
-    # selector export (the step that produces the masks), measured last
-    if world == 1:
+    extras = {}
+    if world == 1 and not args.headline_only:
+        dense = {}
+        for T in DECODE_T:
+            s = dense_block_seconds(torch, w4, dev, stream, T) * len(S.blocks)
+            dense[str(T)] = {"ms_per_stack_pass": s * 1e3, "tokens/s": T / s,
+                             "how": "dense bf16 torch.matmul on block 0's unpruned weights, x 40 blocks"}
+        extras["dense_torch_bf16"] = dense
+        del xs, ys
+        torch.cuda.empty_cache()
+        extras["prefill_stack"] = measure_prefill_stack(gs, torch, dev, stream, S, PREFILL_T, tpk, tpk_sus,
+                                                        hbm_peak, dense_ref=True)
+        extras["pack"] = {"workload": w4.name, "seconds": S.pack_s, "layers": len(S.layers),
+                          "GB/s_incl_alloc_and_sync": S.pack_bytes() / S.pack_s / 1e9}
+        S.free()
+        del S
+        torch.cuda.empty_cache()
+        extras["stack_7b"] = measure_stack_7b(gs, torch, dev, stream, pool, tpk, tpk_sus, hbm_peak)
+        extras["stack_qwen"] = measure_stack_qwen(gs, torch, dev, stream, pool, tpk, tpk_sus, hbm_peak)
+        extras["single_layer"] = measure_single_layer(gs, torch, dev, stream, hbm_peak)
+        extras["block_7b"] = measure_block_7b(gs, torch, dev, stream, pool, hbm_peak)
         try:
-            mask_export = measure_select(gs, torch, dev, stream, peaks)
+            extras["mask_export"] = measure_select(gs, torch, dev, stream, peaks)
         except Exception as e:   # reported in the line, never hidden
-            mask_export = {"error": f"{type(e).__name__}: {e}"}
+            extras["mask_export"] = {"error": f"{type(e).__name__}: {e}"}
+        assert gs.device_status() == gs.GS_OK
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = oracle_sample_rate(layers, args.cpu_seconds)
+        w_o, layers_o = oracle_block_inputs()
+        cpu = oracle_sample_rate(w_o, layers_o, args.cpu_seconds)
         cpu["single_thread"] = oracle_single_thread_rate(args.cpu_seconds / 2)
 
-    hbm_peak = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
-    traffic = recorded_traffic("k_decode", "gs_decode.cu", "llama2-7b-block")
+    traffic = recorded_traffic("k_decode", "gs_decode.cu", "llama2-13b-block")
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "llama2-7b-block decode: 7 projections x T=1,4,16 (21 tokens per step)",
-                   "layers": 7, "kept_groups": kept, "total_groups": w.total_groups, "density": kept / w.total_groups,
-                   "kept_weight_bytes": kept_bytes,
-                   "l2": f"inputs larger than L2: {R} rotated packed copies ({R * kept_bytes / 1e6:.0f} MB) vs "
-                         f"L2 {l2 / 1e6:.0f} MB", "parallelism": f"replicas x{world}", "graph": "one CUDA graph per step"},
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "gpu_launches": launches,
+        "config": {"workload": f"{w4.name} decode: {len(w4.layers)} layers x T=1,16 (17 tokens per step)",
+                   "layers": len(w4.layers), "kept_groups": w4.budget, "total_groups": w4.total_groups,
+                   "density": w4.budget / w4.total_groups, "kept_weight_bytes": 512 * w4.budget,
+                   "l2": f"inputs larger than L2: {512 * w4.budget / 1e9:.2f} GB of kept weights per pass",
+                   "parallelism": f"replicas x{world}",
+                   "graph": f"one CUDA graph per step: {launches_per_step} batched decode launches "
+                            f"(one per block per T)"},
         "roofline": {"kernel": "k_decode", "bound": "hbm", "achieved": achieved_gbs, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved_gbs / hbm_peak, "peak_source": f"{peaks_src} hbm_gbs",
                      "bytes_per_step": bytes_per_step, "traffic": traffic,
-                     "frac_of_8TBs_nominal": achieved_gbs / 8000.0},
+                     "frac_of_8TBs_nominal": achieved_gbs / NOMINAL_HBM_GBS},
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "steps": e2e_steps, "how": "per step: one pinned host -> device copy of every x (T = 1, 4, 16), three "
-                                         "gs_linear_batched calls through the Python binding (no graph), one device -> "
-                                         "pinned host copy of every y; copies on their own streams, device buffers "
-                                         "alternating between steps so copies overlap neighbouring launches"},
-        "gpu_launches": launches,
+        "e2e": e2e,
         "clocks": clock_rec,
         "per_T": per_T,
-        "dense_torch_bf16": dense,
-        "pack": {"seconds": pack_s, "layers": 7, "GB/s_incl_alloc_and_sync": pack_bytes / pack_s / 1e9},
-        "prefill": prefill,
-        "prefill_sweep": prefill_sweep,
-        "decode_sweep": decode_sweep,
-        "mask_export": mask_export,
     }
+    line.update(extras)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
@@ -549,143 +575,208 @@ def run_ours(args):
     return 0
 
 
-def _time_block(gs, torch, stream, xd, ps, ys, algo, n=10):
-    """Seconds per pass over one block's 7 projections (CUDA events, after warm-up);
-    one batched call per pass (T >= 33 takes the tensor-core prefill kernel)."""
-    assert algo == gs.ALGO_PREFILL and xd[0].shape[0] >= 33
-    with torch.cuda.stream(stream):
-        for _ in range(3):
-            gs.linear_batched_into(xd, ps, ys, stream=stream)
+def measure_e2e(gs, torch, dev, stream, S, xs, ys, tokens_per_step, world, args):
+    """The headline step through the public API (gs_linear_batched via the Python
+    binding, no graph) with host buffers: every step copies all x of both passes
+    from pinned host memory and all y back.  Two schedules: `value` overlaps a
+    step's copies with the neighbouring steps' launches (copies on their own
+    streams, device buffers alternating between steps); `serialised` runs copy,
+    launches and copy back in order on one stream."""
+    layers = S.layers
+    xh = torch.cat([torch.cat([x.reshape(-1) for x in xs[T]]) for T in DECODE_T]).cpu().pin_memory()
+    yh = torch.empty(sum(T * L.out for T in DECODE_T for L in layers), dtype=torch.bfloat16).pin_memory()
+    xd = [torch.empty_like(xh, device=dev) for _ in range(2)]
+    yd = [torch.empty_like(yh, device=dev) for _ in range(2)]
+
+    def views(buf, dim):
+        out, off = {}, 0
+        for T in DECODE_T:
+            v = []
+            for L in layers:
+                n = T * getattr(L, dim)
+                v.append(buf[off:off + n].view(T, getattr(L, dim)))
+                off += n
+            out[T] = v
+        return out
+
+    xv = [views(xd[k], "inp") for k in range(2)]
+    yv = [views(yd[k], "out") for k in range(2)]
+    h2d = xh.numel() * 2
+    d2h = yh.numel() * 2
+    n_steps = max(10, min(args.steps, 200))
+    h2d_stream = torch.cuda.Stream(device=dev)
+    d2h_stream = torch.cuda.Stream(device=dev)
+    x_ready = [torch.cuda.Event() for _ in range(2)]
+    k_done = [torch.cuda.Event() for _ in range(2)]
+    y_read = [torch.cuda.Event() for _ in range(2)]
+    used = [False, False]
+
+    def overlapped(i):
+        k = i % 2
+        if used[k]:
+            h2d_stream.wait_event(k_done[k])   # the launches two steps back have read this x buffer
+        with torch.cuda.stream(h2d_stream):
+            xd[k].copy_(xh, non_blocking=True)
+            x_ready[k].record(h2d_stream)
+        stream.wait_event(x_ready[k])
+        if used[k]:
+            stream.wait_event(y_read[k])       # the copy two steps back has read this y buffer
+        for T in DECODE_T:
+            stack_pass(gs, S, xv[k][T], yv[k][T], stream)
+        k_done[k].record(stream)
+        d2h_stream.wait_event(k_done[k])
+        with torch.cuda.stream(d2h_stream):
+            yh.copy_(yd[k], non_blocking=True)
+            y_read[k].record(d2h_stream)
+        used[k] = True
+
+    def serialised(i):
+        with torch.cuda.stream(stream):
+            xd[0].copy_(xh, non_blocking=True)
+            for T in DECODE_T:
+                stack_pass(gs, S, xv[0][T], yv[0][T], stream)
+            yh.copy_(yd[0], non_blocking=True)
+
+    out = {}
+    for name, fn in (("overlapped", overlapped), ("serialised", serialised)):
+        for i in range(3):
+            fn(i)
+        torch.cuda.synchronize(dev)
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for _ in range(n):
-            gs.linear_batched_into(xd, ps, ys, stream=stream)
+        h2d_stream.wait_event(a)
+        for i in range(n_steps):
+            fn(i)
+        if name == "overlapped":
+            stream.wait_event(y_read[(n_steps - 1) % 2])   # the last step's results are on the host
         b.record(stream)
         b.synchronize()
-    return a.elapsed_time(b) / 1e3 / n
+        torch.cuda.synchronize(dev)
+        out[name] = world * tokens_per_step * n_steps / (a.elapsed_time(b) / 1e3)
+        # the host copy of the results equals the device-resident path's results
+        y_ref = torch.cat([torch.cat([y.reshape(-1) for y in ys[T]]) for T in DECODE_T])
+        assert torch.equal(yh.to(dev), y_ref), f"e2e ({name}) result mismatch"
+    return {"value": out["overlapped"], "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": n_steps, "serialised": out["serialised"],
+            "how": "per step: one pinned host -> device copy of every layer's x (T = 1 and 16), one "
+                   "gs_linear_batched call per block and T through the Python binding (no graph), one device -> "
+                   "pinned host copy of every y.  value: copies on their own streams, device buffers alternating "
+                   "between steps; serialised: copy, launches, copy back in order on one stream"}
 
 
-def measure_prefill(gs, torch, dev, stream, peaks):
-    w = wl.workload(3, blocks=1)
-    k = wl.keep_counts(w)
-    T = 2048
-    # device-side draws of the same distributions (numpy draws of 7 full layers are slow)
-    Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
-    Bd = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in range(7)]
-    xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
-    ps = [gs.pack(Wd[i], Bd[i]) for i in range(7)]
-    ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
-    kept = sum(p.kept for p in ps)
-    flops = 2.0 * T * 256 * kept
-    s_block = _time_block(gs, torch, stream, xd, ps, ys, gs.ALGO_PREFILL)
-    n = 10
-    with torch.cuda.stream(stream):
-        # dense bf16 reference point on the unpruned weights
-        for i in range(7):
-            torch.matmul(xd[i], Wd[i].t())
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(n):
-            for i in range(7):
-                torch.matmul(xd[i], Wd[i].t())
-        b.record(stream)
-        b.synchronize()
-        s_dense = a.elapsed_time(b) / 1e3 / n
-    tflops = flops / s_block / 1e12
-    peak = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
-    dense_flops = 2.0 * T * sum(L.out * L.inp for L in w.layers)
+def measure_prefill_stack(gs, torch, dev, stream, S, Ts, tpk, tpk_sus, hbm_peak, dense_ref=False):
+    """Tensor-core prefill over a whole packed stack: one batched call per block
+    (7 layers per launch).  tokens/s = T / pass time; kept TFLOP/s against the
+    measured dense bf16 peak (burst, and sustained: a pass is a long step); at
+    small T the attainable rate is min(tensor peak, kept FLOPs / time to stream
+    the pass's bytes at the measured HBM bandwidth)."""
+    rows = []
+    w = S.w
+    for T in Ts:
+        xs, ys = stack_inputs(torch, w, dev, T)
+        reps = 3 if T >= 1024 else 5
+        s = time_calls(torch, stream, lambda: stack_pass(gs, S, xs, ys, stream), reps, warm=1)
+        flops = kept_flops(S.kept, T)
+        nbytes = 512.0 * S.kept_groups + sum(2.0 * T * (L.inp + L.out) for L in S.layers)
+        attainable = min(tpk, flops / (nbytes / (hbm_peak * 1e9)) / 1e12)
+        tf = flops / s / 1e12
+        row = {"workload": f"{w.name}, T={T}", "T": T, "kept_groups": S.kept_groups, "ms_per_pass": s * 1e3,
+               "tokens/s": T / s, "kept_TFLOP/s": tf, "frac_of_burst_peak": tf / tpk,
+               "frac_of_sustained_peak": tf / tpk_sus, "attainable_TFLOP/s": attainable,
+               "frac_of_attainable": tf / attainable, "launches_per_pass": len(S.blocks)}
+        del xs, ys
+        torch.cuda.empty_cache()
+        if dense_ref:
+            sd = dense_block_seconds(torch, w, dev, stream, T, reps=3) * len(S.blocks)
+            row["dense_torch_ms_per_pass"] = sd * 1e3
+            row["speedup_vs_dense"] = sd / s
+            row["dense_how"] = "dense bf16 torch.matmul on block 0's unpruned weights, x blocks"
+        rows.append(row)
     assert gs.device_status() == gs.GS_OK
-    out = {"workload": "llama2-7b block 0 (7 projections), T=2048, 1% outlier channels x20, layer-adaptive 50%",
-           "kept_groups": kept, "kept_tflop_per_block": flops / 1e12, "ms_per_block": s_block * 1e3,
-           "tokens/s": T / s_block, "TFLOP/s": tflops, "peak_TFLOP/s": peak, "frac": tflops / peak,
-           "peak_source": "measured bf16_tflops (burst)",
-           "dense_torch_ms_per_block": s_dense * 1e3,
-           "dense_torch_TFLOP/s": dense_flops / s_dense / 1e12, "speedup_vs_dense": s_dense / s_block}
-    del Wd, Bd, xd, ps, ys
+    return rows
+
+
+def measure_stack_7b(gs, torch, dev, stream, pool, tpk, tpk_sus, hbm_peak):
+    """The whole LLaMA-2-7B stack (32 blocks, 224 layers) at T = 2048 with 1 % of
+    input channels scaled x20 (the third configuration)."""
+    w = wl.workload(3)
+    S = Stack(gs, torch, dev, w, pool)
+    rows = measure_prefill_stack(gs, torch, dev, stream, S, (2048,), tpk, tpk_sus, hbm_peak, dense_ref=True)
+    S.free()
+    torch.cuda.empty_cache()
+    return rows[0]
+
+
+def measure_stack_qwen(gs, torch, dev, stream, pool, tpk, tpk_sus, hbm_peak):
+    """The whole Qwen2.5-7B stack (28 blocks, 196 layers) at global densities 0.3,
+    0.5 and 0.7: a decode pass at T = 1 (graph of one batched call per block) and a
+    prefill pass at T = 1024 (the fifth configuration)."""
+    out = []
+    for d in (0.3, 0.5, 0.7):
+        w = wl.workload(5, d)
+        S = Stack(gs, torch, dev, w, pool)
+        xs, ys = stack_inputs(torch, w, dev, 1)
+        s = time_replays(torch, stream, [capture(torch, stream, lambda: stack_pass(gs, S, xs, ys, stream))], reps=30)
+        nb = stack_decode_bytes(S.layers, S.kept, 1)
+        row = {"workload": w.name, "density": d, "kept_groups": S.kept_groups,
+               "decode_T1": {"ms_per_pass": s * 1e3, "tokens/s": 1 / s, "GB/s": nb / s / 1e9,
+                             "frac_of_measured_hbm": nb / s / 1e9 / hbm_peak,
+                             "frac_of_8TBs_nominal": nb / s / 1e9 / NOMINAL_HBM_GBS}}
+        del xs, ys
+        row["prefill_T1024"] = measure_prefill_stack(gs, torch, dev, stream, S, (1024,), tpk, tpk_sus, hbm_peak)[0]
+        S.free()
+        torch.cuda.empty_cache()
+        out.append(row)
+    return out
+
+
+def measure_single_layer(gs, torch, dev, stream, hbm_peak, copies: int = 256):
+    """The single 1024x1024 layer (first configuration: exactly half of its 4096
+    groups kept, T = 8): one graph of `copies` calls, each on its own packed copy
+    (256 MiB of kept weights in all, larger than L2)."""
+    w = wl.workload(1)
+    ks = wl.keep_counts(w)
+    W = wl.weight_device(w, 0, device=dev)
+    M = torch.from_numpy(wl.group_mask(w, 0, int(ks[0]))).to(dev)
+    ps = [gs.pack(W, M) for _ in range(copies)]
+    x = wl.activation_device(w, 0, 8, device=dev)
+    ys = [torch.empty((8, 1024), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
+
+    def run():
+        for p, y in zip(ps, ys):
+            gs.linear_into(x, p, y, stream=stream)
+    s = time_replays(torch, stream, [capture(torch, stream, run)], reps=20) / copies
+    nb = layer_decode_bytes(w.layers[0], ks[0], 8)
+    out = {"workload": "single 1024x1024 layer, 2048 of 4096 groups kept, T=8", "us_per_call": s * 1e6,
+           "tokens/s": 8 / s, "GB/s": nb / s / 1e9, "frac_of_measured_hbm": nb / s / 1e9 / hbm_peak,
+           "how": f"one CUDA graph of {copies} gs_linear calls, each on its own packed copy"}
+    for p in ps:
+        p.free()
+    del ps, W, M
     torch.cuda.empty_cache()
     return out
 
 
-def measure_prefill_sweep(gs, torch, dev, stream, peaks):
-    """Prefill kernel over the token counts of the 13B and Qwen stacks (first block
-    of each).  The attainable rate at a token count is min(tensor peak, kept FLOPs
-    over the time to stream the block's bytes at the measured HBM bandwidth)."""
-    tpk = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
-    bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"])) * 1e9
+def measure_block_7b(gs, torch, dev, stream, pool, hbm_peak, copies: int = 4):
+    """One LLaMA-2-7B block (second configuration: per-module keep U[0.3, 0.7]
+    rescaled to 50 %) at T = 1, 4 and 16: one batched call per T, graphs cycling
+    over `copies` packed copies (together larger than L2)."""
+    w = wl.workload(2)
+    Ss = [Stack(gs, torch, dev, w, pool) for _ in range(copies)]
     rows = []
-    for cfg, d, Ts, name in ((4, 0.5, (128, 512, 2048), "llama2-13b block 0"),
-                             (5, 0.5, (1024,), "qwen2.5-7b block 0, d=0.5")):
-        w = wl.workload(cfg, d, blocks=1)
-        k = wl.keep_counts(w)
-        Wd = [wl.weight_device(w, i, device=dev) for i in range(7)]
-        ps = [gs.pack(Wd[i], torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev)) for i in range(7)]
-        del Wd
-        kept = sum(p.kept for p in ps)
-        for T in Ts:
-            xd = [wl.activation_device(w, i, T, device=dev) for i in range(7)]
-            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in w.layers]
-            s_block = _time_block(gs, torch, stream, xd, ps, ys, gs.ALGO_PREFILL)
-            flops = 2.0 * T * 256 * kept
-            nbytes = 512.0 * kept + sum(2.0 * T * (L.inp + L.out) for L in w.layers)
-            attainable = min(tpk, flops / (nbytes / bw) / 1e12)
-            tflops = flops / s_block / 1e12
-            rows.append({"workload": f"{name}, T={T}", "T": T, "kept_groups": kept, "ms_per_block": s_block * 1e3,
-                         "tokens/s": T / s_block, "TFLOP/s": tflops, "attainable_TFLOP/s": attainable,
-                         "frac_of_attainable": tflops / attainable, "frac_of_tensor_peak": tflops / tpk})
-            del xd, ys
-        del ps
-        torch.cuda.empty_cache()
-    assert gs.device_status() == gs.GS_OK
-    return rows
-
-
-def measure_decode_sweep(gs, torch, dev, stream, peaks):
-    """Decode kernel on the first block of the 13B stack (T = 1, 16), of the Qwen
-    stack (d = 0.5, T = 1), and on block 25 of the 7B stack under the paper-shaped
-    allocation (Q/K near 8 %, down above 53 %; T = 1): one batched launch per pass
-    over the block's 7 projections, alternating between two packed copies (each
-    larger than L2)."""
-    bw = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
-    rows = []
-    for w, blk, Ts, name in ((wl.workload(4, 0.5, blocks=1), 0, (1, 16), "llama2-13b block 0"),
-                             (wl.workload(5, 0.5, blocks=1), 0, (1,), "qwen2.5-7b block 0, d=0.5"),
-                             (wl.workload(3, allocation="paper"), 25, (1,),
-                              "llama2-7b block 25, paper-shaped allocation")):
-        k = wl.keep_counts(w)
-        ids = list(range(7 * blk, 7 * blk + 7))
-        Wd = [wl.weight_device(w, i, device=dev) for i in ids]
-        Md = [torch.from_numpy(wl.group_mask(w, i, int(k[i]))).to(dev) for i in ids]
-        copies = [[gs.pack(Wd[j], Md[j]) for j in range(7)] for _ in range(2)]
-        del Wd, Md
-        kept = sum(p.kept for p in copies[0])
-        layers = [w.layers[i] for i in ids]
-        for T in Ts:
-            xd = [wl.activation_device(w, i, T, device=dev) for i in ids]
-            ys = [torch.empty((T, L.out), dtype=torch.bfloat16, device=dev) for L in layers]
-            n = 50
-            with torch.cuda.stream(stream):
-                for i in range(4):
-                    gs.linear_batched_into(xd, copies[i % 2], ys, stream=stream)
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                for i in range(n):
-                    gs.linear_batched_into(xd, copies[i % 2], ys, stream=stream)
-                b.record(stream)
-                b.synchronize()
-            s_pass = a.elapsed_time(b) / 1e3 / n
-            nbytes = sum(512.0 * p.kept + 6.0 * (L.inp // 256) * ((L.out + 15) // 16) + 2.0 * T * (L.inp + L.out)
-                         for p, L in zip(copies[0], layers))
-            gbs = nbytes / s_pass / 1e9
-            rows.append({"workload": f"{name}, T={T}", "T": T, "kept_groups": kept, "us_per_block": s_pass * 1e6,
-                         "tokens/s": T / s_pass, "GB/s": gbs, "frac_of_measured_hbm": gbs / bw})
-            del xd, ys
-        del copies
-        torch.cuda.empty_cache()
-    assert gs.device_status() == gs.GS_OK
-    return rows
+    for T in BLOCK_T:
+        xs, ys = stack_inputs(torch, w, dev, T)
+        gr = [capture(torch, stream, lambda S=S: stack_pass(gs, S, xs, ys, stream)) for S in Ss]
+        s = time_replays(torch, stream, gr, reps=200)
+        nb = stack_decode_bytes(Ss[0].layers, Ss[0].kept, T)
+        rows.append({"T": T, "us_per_launch": s * 1e6, "tokens/s": T / s, "GB/s": nb / s / 1e9,
+                     "frac_of_measured_hbm": nb / s / 1e9 / hbm_peak})
+        del xs, ys, gr
+    for S in Ss:
+        S.free()
+    torch.cuda.empty_cache()
+    return {"workload": "llama2-7b block (7 projections), one batched launch per T", "per_T": rows}
 
 
 def measure_select(gs, torch, dev, stream, peaks):
@@ -698,24 +789,13 @@ def measure_select(gs, torch, dev, stream, peaks):
     lg = wl.selector_logits_device(n, 0.5, seed=1, device=dev)
     mask = torch.empty((n,), dtype=torch.uint8, device=dev)
     kept = torch.empty((1,), dtype=torch.int64, device=dev)
-    reps = 50
-    with torch.cuda.stream(stream):
-        for _ in range(5):
-            gs.select_groups(lg, mask, kept, stream=stream)
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(reps):
-            gs.select_groups(lg, mask, kept, stream=stream)
-        b.record(stream)
-        b.synchronize()
-    s_launch = a.elapsed_time(b) / 1e3 / reps
+    s = time_calls(torch, stream, lambda: gs.select_groups(lg, mask, kept, stream=stream), reps=50, warm=5)
     k = int(kept.cpu()[0])
     del lg, mask, kept
     torch.cuda.empty_cache()
-    gbs = 5.0 * n / s_launch / 1e9
+    gbs = 5.0 * n / s / 1e9
     return {"workload": "selectors of the llama2-13b stack (40 blocks), logits ~ N(0, 1)", "kernel": "k_select",
-            "selectors": n, "kept": k, "bytes_per_launch": 5 * n, "us_per_launch": s_launch * 1e6, "GB/s": gbs,
+            "selectors": n, "kept": k, "bytes_per_launch": 5 * n, "us_per_launch": s * 1e6, "GB/s": gbs,
             "frac_of_measured_hbm": gbs / bw}
 
 
@@ -733,6 +813,42 @@ def run_mask_export(args):
     return 0
 
 
+def run_block(args):
+    """One block of a stack (--block-of 4: the 13B stack, 2: the 7B block, 3: the
+    7B stack, 5: the Qwen stack at --density) at --tokens, one batched call per
+    step, cycling over two packed copies; prints one JSON line.  Used for the
+    small cases that ncu captures."""
+    import concurrent.futures as cf
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+    dev = torch.device("cuda", 0)
+    w = wl.workload(args.block_of, args.density, blocks=1)
+    pool = cf.ThreadPoolExecutor(max_workers=8)
+    Ss = [Stack(gs, torch, dev, w, pool) for _ in range(2)]
+    T = args.tokens
+    xs, ys = stack_inputs(torch, w, dev, T)
+    stream = torch.cuda.current_stream()
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            stack_pass(gs, Ss[i % 2], xs, ys, stream)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(args.steps):
+            stack_pass(gs, Ss[i % 2], xs, ys, stream)
+        b.record(stream)
+        b.synchronize()
+    s = a.elapsed_time(b) / 1e3 / args.steps
+    nb = stack_decode_bytes(Ss[0].layers, Ss[0].kept, T)
+    fl = kept_flops(Ss[0].kept, T)
+    assert gs.device_status() == gs.GS_OK
+    print(json.dumps({"workload": f"{w.name} block 0", "T": T, "kept": Ss[0].kept_groups, "us": s * 1e6,
+                      "GB/s": nb / s / 1e9, "kept_TFLOP/s": fl / s / 1e12}), flush=True)
+    return 0
+
+
 def run_layer(args):
     """One synthetic layer (random mask of the given density), one kernel family,
     timed with CUDA events; prints one JSON line.  Used for sweeps and for the
@@ -743,8 +859,6 @@ def run_layer(args):
     from paper_2609_33977_gb300 import groupsparse as gs
     T = args.tokens
     dev = torch.device("cuda", 0)
-    if args.layer == "llama2-7b-block":
-        return run_block_layers(args, gs, torch, dev)
     out, inp = (int(v) for v in args.layer.lower().split("x"))
     g = torch.Generator(device=dev)
     g.manual_seed(1234)
@@ -775,56 +889,20 @@ def run_layer(args):
     return 0
 
 
-def run_block_layers(args, gs, torch, dev):
-    """The seven LLaMA-2-7B block projections (random masks of --density) in one
-    batched call per step, timed with CUDA events over R rotated packed copies."""
-    shapes = [(o, i) for (_, o, i) in wl.LLAMA2_7B_BLOCK]
-    T = args.tokens
-    g = torch.Generator(device=dev)
-    g.manual_seed(1234)
-    R = 4
-    packs = []
-    for _ in range(R):
-        hs = []
-        for (o, i) in shapes:
-            W = (torch.randn((o, i), generator=g, device=dev) * 0.02).to(torch.bfloat16)
-            B = (torch.rand((o, i // 256), generator=g, device=dev) < args.density).to(torch.uint8)
-            hs.append(gs.pack(W, B))
-        packs.append(hs)
-    xs = [torch.randn((T, i), generator=g, device=dev).to(torch.bfloat16) for (o, i) in shapes]
-    ys = [torch.empty((T, o), dtype=torch.bfloat16, device=dev) for (o, i) in shapes]
-    for r in range(args.warmup):
-        gs.linear_batched_into(xs, packs[r % R], ys)
-    torch.cuda.synchronize()
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
-    a.record()
-    for r in range(args.steps):
-        gs.linear_batched_into(xs, packs[r % R], ys)
-    b.record()
-    b.synchronize()
-    s = a.elapsed_time(b) / 1e3 / args.steps
-    kept = sum(p.kept for p in packs[0])
-    nbytes = 512 * kept + sum(16 * (i // 256) * ((o + 63) // 64) + 2 * T * (i + o) for (o, i) in shapes)
-    assert gs.device_status() == gs.GS_OK
-    print(json.dumps({"layer": "llama2-7b-block x7 batched", "T": T, "density": args.density, "kept": kept,
-                      "us": s * 1e6, "GB/s": nbytes / s / 1e9}), flush=True)
-    return 0
-
-
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--rotate", type=int, default=0, help="rotated packed copies (0 = enough to exceed 3x L2)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--oracle-single-thread", action="store_true",
                     help="internal: time the oracle sample only and print it (run with one BLAS thread)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--headline-only", action="store_true", help="skip the per-GPU characterisations")
     ap.add_argument("--layer", default=None, help="single-layer mode: OUTxIN (random mask of --density)")
+    ap.add_argument("--block-of", type=int, default=0,
+                    help="block mode: block 0 of workload 2, 3, 4 or 5, at --tokens")
     ap.add_argument("--tokens", type=int, default=16)
     ap.add_argument("--density", type=float, default=0.5)
     ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
@@ -834,13 +912,15 @@ def main():
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.oracle_single_thread:
-        _, layers = block_inputs()
-        print(json.dumps(oracle_sample_rate(layers, args.cpu_seconds)), flush=True)
+        w, layers = oracle_block_inputs()
+        print(json.dumps(oracle_sample_rate(w, layers, args.cpu_seconds)), flush=True)
         return 0
     if args.impl == "reference":
         return run_reference(args)
     if args.layer:
         return run_layer(args)
+    if args.block_of:
+        return run_block(args)
     if args.mask_export:
         return run_mask_export(args)
     return run_ours(args)
