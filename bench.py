@@ -508,7 +508,12 @@ def run_ours(args):
                                              "launches_per_pass": len(S.layers)}}
     torch.cuda.empty_cache()
 
-    # ---- end to end through the public API with host buffers (no graph)
+    # ---- end to end through the public API with host buffers (no graph); the
+    # step graph (per-block batched calls, as the e2e path makes) writes the
+    # device-resident results it is compared with
+    with torch.cuda.stream(stream):
+        g_step.replay()
+    stream.synchronize()
     e2e = measure_e2e(gs, torch, dev, stream, S, xs, ys, tokens_per_step, world, args)
 
     # ---- per-GPU characterisations (N = 1 only: at N > 1 every rank would repeat them
