@@ -83,6 +83,37 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
                   int32_t group_in, void* stream, gs_packed** handle);
 
 /*
+ * gs_pack_groups - gs_pack for other group shapes.  Sec. 2.1 splits W into
+ * non-overlapping g_out x g_in groups and B[G_out][G_in] keeps or prunes each
+ * (Eq. 1 with M = B (x) 1_{g_out x g_in}); the Sec. 3.5 granularity ablation
+ * and App. E evaluate 1 x 128, 1 x 256, 16 x 16, 32 x 32, 64 x 64 and
+ * 128 x 128.  Supported here: (1, 256), which is gs_pack itself, and square
+ * g x g with g in {16, 32, 64, 128}; other shapes return GS_ERR_UNSUPPORTED.
+ *
+ * Packed layout of square groups (bit-exact, deterministic): column block v
+ * (input columns [g v, g v + g)) owns packed tiles [offsets[v], offsets[v+1]);
+ * inside a column block the kept block rows u ascend; row_idx[j] is the block
+ * row of tile j and tiles[j] is a bit copy of the g x g block of W at rows
+ * [g u, g u + g), columns [g v, g v + g), row-major.
+ *
+ * W_dev     bf16 [out][in] row-major, caller-owned, read only.
+ * mask_dev  uint8 [out/g_out][in/g_in] row-major; nonzero = keep.  Read only.
+ * out, in   multiples of g_out and g_in (the groups tile W exactly);
+ *           (out/g_out)(in/g_in) < 2^31 and in/g_in <= 65535.
+ * stream, handle: as for gs_pack (one synchronization to size the buffers).
+ * gs_linear, gs_linear_ex (the kernel family is chosen by the handle: square
+ * groups have one tensor-core kernel for every token count),
+ * gs_linear_batched, gs_unpack, gs_packed_info, gs_packed_export and gs_free
+ * accept the handle.
+ * Errors: INVALID_ARG (nulls, sizes, alignment), UNSUPPORTED (shape), OOM, CUDA.
+ */
+gs_status gs_pack_groups(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t g_out,
+                         int32_t g_in, void* stream, gs_packed** handle);
+
+/* gs_packed_group_shape - the group shape a handle was packed with (either pointer may be NULL). */
+gs_status gs_packed_group_shape(const gs_packed* p, int32_t* g_out, int32_t* g_in);
+
+/*
  * gs_linear - y = x W_hat^T for the packed weight (Eq. 1 applied as a linear
  * projection, no bias), fp32 accumulation, bf16 output rounded to nearest even.
  *
@@ -170,6 +201,9 @@ gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t*
  * that gs_pack describes.  Sizes: offsets int64[G+1], row_idx int32[K],
  * tiles uint16[K*256], win_off16 int32[G*(ceil(out/16)+1)],
  * kmask16 uint16[G*ceil(out/16)], with K = kept_groups.  Any pointer may be NULL.
+ * For handles of square g x g groups (gs_pack_groups): offsets int64[in/g+1],
+ * row_idx int32[K] (block rows), tiles uint16[K*g*g]; win_off16 and kmask16
+ * must be NULL (INVALID_ARG otherwise).
  */
 gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* row_idx_host,
                            uint16_t* tiles_host, int32_t* win_off16_host, uint16_t* kmask16_host);

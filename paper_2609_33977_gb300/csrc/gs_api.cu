@@ -37,6 +37,7 @@ void free_buffers(gs_packed* p) {
   if (p->win_off16) cudaFree(p->win_off16);
   if (p->kmask16) cudaFree(p->kmask16);
   decode_release(p);
+  sq_release(p);
   if (cur >= 0 && cur != p->device) cudaSetDevice(cur);
   p->offsets = nullptr;
   p->row_idx = nullptr;
@@ -55,8 +56,8 @@ gs_status dev_alloc(void** ptr, size_t bytes, size_t* total) {
 
 gs_status check_handle(const gs_packed* p) {
   if (!p) return GS_ERR_INVALID_ARG;
-  if (p->out <= 0 || p->in <= 0 || p->G <= 0 || !p->offsets || !p->win_off16 || !p->kmask16)
-    return GS_ERR_INVALID_ARG;
+  if (p->out <= 0 || p->in <= 0 || p->G <= 0 || !p->offsets) return GS_ERR_INVALID_ARG;
+  if (is_square(p) ? (!p->gwoff || !p->gwmask) : (!p->win_off16 || !p->kmask16)) return GS_ERR_INVALID_ARG;
   return GS_OK;
 }
 
@@ -139,6 +140,9 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
   p->in = in;
   p->G = (int32_t)G;
   p->nw16 = (int32_t)((out + kWin16 - 1) / kWin16);
+  p->g_out = 1;
+  p->g_in = kGroupIn;
+  p->Gout = (int32_t)out;
 
   size_t total = 0;
   int32_t* cnt = nullptr;
@@ -181,6 +185,52 @@ fail:
   return st;
 }
 
+gs_status gs_pack_groups(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t g_out,
+                         int32_t g_in, void* stream, gs_packed** handle) {
+  if (handle) *handle = nullptr;
+  if (!W_dev || !mask_dev || !handle) return GS_ERR_INVALID_ARG;
+  if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX || g_out <= 0 || g_in <= 0) return GS_ERR_INVALID_ARG;
+  if (g_out == 1 && g_in == kGroupIn) return gs_pack(W_dev, mask_dev, out, in, g_in, stream, handle);
+  if (!sq_shape_supported(g_out, g_in)) return GS_ERR_UNSUPPORTED;
+  if (out % g_out != 0 || in % g_in != 0) return GS_ERR_INVALID_ARG;   // the groups must tile W exactly
+  if (!aligned16(W_dev)) return GS_ERR_INVALID_ARG;
+  const int64_t Gout = out / g_out, Gin = in / g_in;
+  if (Gout * Gin >= (int64_t)INT32_MAX || Gin > 65535) return GS_ERR_UNSUPPORTED;
+  gs_packed* p = new (std::nothrow) gs_packed;
+  if (!p) return GS_ERR_OOM;
+  std::memset(p, 0, sizeof(*p));
+  if (cudaGetDevice(&p->device) != cudaSuccess) {
+    delete p;
+    return GS_ERR_CUDA;
+  }
+  if (!device_error_flag()) {
+    delete p;
+    return GS_ERR_CUDA;
+  }
+  p->out = out;
+  p->in = in;
+  p->g_out = g_out;
+  p->g_in = g_in;
+  p->G = (int32_t)Gin;
+  p->Gout = (int32_t)Gout;
+  p->nwin = (int32_t)((out + 127) / 128);
+  const gs_status st = sq_pack(W_dev, mask_dev, p, static_cast<cudaStream_t>(stream));
+  if (st != GS_OK) {
+    free_buffers(p);
+    delete p;
+    return st;
+  }
+  *handle = p;
+  return GS_OK;
+}
+
+gs_status gs_packed_group_shape(const gs_packed* p, int32_t* g_out, int32_t* g_in) {
+  if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
+  if (g_out) *g_out = p->g_out;
+  if (g_in) *g_in = p->g_in;
+  return GS_OK;
+}
+
 static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, void* y_dev, void* stream,
                              gs_algo algo) {
   if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
@@ -190,6 +240,7 @@ static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, v
   if (!x_dev || !y_dev) return GS_ERR_INVALID_ARG;
   if (!aligned16(x_dev) || !aligned16(y_dev)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (is_square(p)) return sq_linear_batched(&x_dev, &p, 1, T, &y_dev, s);   // one kernel family for every T
   if (algo == GS_ALGO_AUTO)
     algo = (T >= kPrefillMinTokens && p->G <= prefill_max_chunks()) ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
   if (algo == GS_ALGO_PREFILL) return launch_prefill(x_dev, p, T, y_dev, s);
@@ -227,6 +278,32 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
   }
   if (T == 0) return GS_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  {
+    // square-group layers take their own launches; the 1 x 256 layers continue below
+    std::vector<const void*> xq;
+    std::vector<const gs_packed*> pq;
+    std::vector<void*> yq;
+    std::vector<const void*> xr;
+    std::vector<const gs_packed*> pr;
+    std::vector<void*> yr;
+    for (int i = 0; i < n; ++i) {
+      if (is_square(ps[i])) {
+        xq.push_back(xs_dev[i]);
+        pq.push_back(ps[i]);
+        yq.push_back(ys_dev[i]);
+      } else {
+        xr.push_back(xs_dev[i]);
+        pr.push_back(ps[i]);
+        yr.push_back(ys_dev[i]);
+      }
+    }
+    if (!pq.empty()) {
+      const gs_status st = sq_linear_batched(xq.data(), pq.data(), (int)pq.size(), T, yq.data(), s);
+      if (st != GS_OK) return st;
+      if (pr.empty()) return GS_OK;
+      return gs_linear_batched((int32_t)pr.size(), xr.data(), pr.data(), T, yr.data(), stream);
+    }
+  }
   if (T >= kPrefillMinTokens) {
     // layers the prefill kernel takes share batched launches; any other goes alone
     std::vector<const void*> xp;
@@ -273,6 +350,7 @@ gs_status gs_select_groups(const float* logits_dev, int64_t n, uint8_t* mask_dev
 
 gs_status gs_unpack(const gs_packed* p, void* W_hat_dev, void* stream) {
   if (check_handle(p) != GS_OK || !W_hat_dev || !aligned16(W_hat_dev)) return GS_ERR_INVALID_ARG;
+  if (is_square(p)) return sq_unpack(p, W_hat_dev, static_cast<cudaStream_t>(stream));
   return launch_unpack(p, W_hat_dev, static_cast<cudaStream_t>(stream));
 }
 
@@ -289,13 +367,15 @@ gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t*
 gs_status gs_packed_export(const gs_packed* p, int64_t* offsets_host, int32_t* row_idx_host, uint16_t* tiles_host,
                            int32_t* win_off16_host, uint16_t* kmask16_host) {
   if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
+  if (is_square(p) && (win_off16_host || kmask16_host)) return GS_ERR_INVALID_ARG;   // no 16-row windows
   if (cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
   const size_t G = (size_t)p->G, nw = (size_t)p->nw16, K = (size_t)p->kept;
   if (offsets_host && cudaMemcpy(offsets_host, p->offsets, sizeof(int64_t) * (G + 1), cudaMemcpyDeviceToHost))
     return GS_ERR_CUDA;
   if (row_idx_host && K && cudaMemcpy(row_idx_host, p->row_idx, sizeof(int32_t) * K, cudaMemcpyDeviceToHost))
     return GS_ERR_CUDA;
-  if (tiles_host && K && cudaMemcpy(tiles_host, p->tiles, (size_t)kTileBytes * K, cudaMemcpyDeviceToHost))
+  const size_t tile_bytes = 2 * (size_t)p->g_out * (size_t)p->g_in;
+  if (tiles_host && K && cudaMemcpy(tiles_host, p->tiles, tile_bytes * K, cudaMemcpyDeviceToHost))
     return GS_ERR_CUDA;
   if (win_off16_host &&
       cudaMemcpy(win_off16_host, p->win_off16, sizeof(int32_t) * G * (nw + 1), cudaMemcpyDeviceToHost))

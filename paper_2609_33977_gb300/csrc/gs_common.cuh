@@ -55,6 +55,16 @@ struct gs_packed {
   alignas(64) unsigned char wmaps[10][128];
   alignas(64) unsigned char wmaps_full[10][128];   // same, box heights 16, 32, ..., 160 (whole slices)
   bool wmaps_valid;
+  // group shape (Sec. 2.1: g_out x g_in groups).  gs_pack handles are 1 x 256;
+  // square g x g handles (gs_pack_groups) use the fields below instead of the
+  // 1 x 256 window metadata: G = in / g column blocks, row_idx holds each
+  // kept tile's block row, tiles holds g x g row-major blocks.
+  int32_t g_out, g_in;
+  int32_t Gout;       // out / g_out
+  int32_t nwin;       // square groups: ceil(out / 128) windows of 128 output rows
+  int32_t* gwoff;     // [G][nwin + 1]: first packed tile of column block v in window w (+ end)
+  uint8_t* gwmask;    // [G][nwin]: bit i = block row (128/g) w + i kept in column block v
+  alignas(64) unsigned char gmaps[8][128];   // W slice descriptors, box heights g, 2g, ..., 128 rows
 };
 
 namespace gs {
@@ -62,6 +72,10 @@ namespace gs {
 // 2-D bf16 TMA descriptor (map: 128-byte, 64-byte aligned buffer); false on failure
 bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
                          uint32_t box_outer, bool swizzle128);
+
+// 2-D bf16 descriptor with a 32-, 64- or 128-byte swizzle (box_inner * 2 <= swizzle_bytes)
+bool encode_tmap_2d_bf16_swz(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                             uint32_t box_outer, int swizzle_bytes);
 
 // 3-D "slab" bf16 descriptor over a row-major [rows][row_elems] matrix: a box
 // of box_rows rows x box_slabs 64-element slabs lands in shared memory as
@@ -87,6 +101,9 @@ uint64_t take_injected_wait(int family);
 
 // pack.cu
 gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t s, int32_t* cnt_tmp);
+// exclusive scan of cnt[G][nw] (chunk-major) into win_off[G][nw + 1] and offsets[G + 1]
+gs_status launch_scan_counts(const int32_t* cnt, int32_t G, int32_t nw, int32_t* win_off, int64_t* offsets,
+                             cudaStream_t s);
 gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s);
 gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
 
@@ -108,5 +125,14 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
 gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T,
                                  void* const* ys, cudaStream_t s);
 int prefill_max_chunks();
+
+// groups.cu: square g x g groups
+bool sq_shape_supported(int g_out, int g_in);
+gs_status sq_pack(const void* W, const uint8_t* mask, gs_packed* p, cudaStream_t s);   // p: shape fields set
+gs_status sq_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
+gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
+                            cudaStream_t s);
+void sq_release(gs_packed* p);
+inline bool is_square(const gs_packed* p) { return p->g_out > 1; }
 
 }  // namespace gs

@@ -1,0 +1,600 @@
+// Square g x g groups (Sec. 2.1 with g_out = g_in = g; the Sec. 3.5 ablation
+// and App. E evaluate g = 16, 32, 64 and 128): packing, unpacking and the
+// group-sparse linear y = x (W (.) M)^T with M = B (x) 1_{g x g} (Eq. 1).
+//
+// Packed layout (the same sequential definition as the 1 x 256 layout, per
+// column block): column block v (input columns [g v, g v + g)) owns packed
+// tiles [offsets[v], offsets[v + 1]); inside a column block the kept block
+// rows u ascend; tile j is the g x g block of W at rows g u.., columns g v..,
+// row-major, a bit copy, and row_idx[j] = u.  Per (column block, window of
+// 128 output rows) the library also keeps the first tile of the window's
+// slice and a bitmask of its kept block rows.
+//
+// Linear.  A unit of work is 128 tokens x one window of 128 output rows,
+// R = 128 / g block rows.  In column block v the window's kept tiles are one
+// contiguous slice of the packed tiles, i.e. a dense [n g x g] matrix that
+// one TMA box loads, next to one box of the 128 tokens' x columns of v.  Each
+// kept tile is a whole tensor-core operand: its MMAs (M = 128 tokens, N = g
+// rows, K = g) accumulate straight into its block row's g columns of a
+// 128-column TMEM accumulator, so nothing is gathered or scattered, and the
+// accumulator is read once per unit.  Pruned tiles cost neither bytes nor
+// FLOPs.  Token rows beyond T read as zero (TMA fill) and are not stored; the
+// same kernel serves every token count.
+//
+// Roles (one CTA per SM, persistent over units): warp 0 TMA producer, warp 1
+// TMEM allocator + single-thread MMA issuer, warps 2..5 epilogue (warp w reads
+// TMEM lanes 32 (w % 4) ..).  Two accumulator buffers let the epilogue of one
+// unit overlap the MMAs of the next.  Shared-memory operands use the swizzle
+// whose width is one operand row: 32 B (g = 16), 64 B (g = 32), 128 B
+// (g = 64; g = 128 as two 64-column slabs).  Every mbarrier wait is bounded;
+// a wait that runs out raises the CTA's abort flag and the library's device
+// error flag, and every role winds down.
+#include "gs_common.cuh"
+#include "gs_sm100.cuh"
+
+#include <cuda.h>
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+namespace gs {
+namespace {
+using namespace sm100;
+
+constexpr int kSqM = 128;                 // tokens per unit (TMEM lanes)
+constexpr int kSqWin = 128;               // output rows per window (accumulator columns)
+constexpr int kSqAccBufs = 2;
+constexpr uint32_t kSqTmemCols = kSqAccBufs * kSqWin;
+constexpr int kSqEpiWarps = 4;
+constexpr int kSqThreads = (2 + kSqEpiWarps) * 32;
+constexpr int kSqMaxLayers = 8;
+constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R <= 8)
+constexpr int kSqSlabBytes = 128 * 128;   // one operand slab: 128 rows x 128-byte pitch (the largest swizzle)
+constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
+constexpr uint64_t kSqDrainLimitNs = 200000000ull;
+
+template <int G>
+struct Sq {
+  static constexpr int R = kSqWin / G;                  // block rows per window
+  static constexpr int kSlabs = G > 64 ? 2 : 1;         // 64-column slabs per operand row
+  static constexpr int kRowB = G >= 64 ? 128 : 2 * G;   // operand row bytes within a slab = swizzle width
+  static constexpr int kRegion = kSlabs * kSqSlabBytes; // bytes reserved per operand per stage
+  static constexpr int kStageBytes = 2 * kRegion;       // x box, then W slice
+  static constexpr int kStages = G > 64 ? 3 : 6;
+  static constexpr uint32_t kSwz = G >= 64 ? 2u : (G == 32 ? 4u : 6u);   // UMMA layout: 128 / 64 / 32-byte swizzle
+  static constexpr uint32_t kSBO = 8 * kRowB;           // bytes between 8-row core groups
+  static constexpr int kKSteps = G / 16;
+  static constexpr uint32_t kXBoxBytes = kSqM * 2 * G;  // full x box (rows past T are zero-filled and counted)
+  static constexpr int kSmem = kStages * kStageBytes + 2 * 32 * 8 + 1024;
+  static_assert(R >= 1 && R <= kSqMaxMaps, "window holds 1..8 block rows");
+  static_assert(kSmem <= 227 * 1024, "shared memory budget");
+  static_assert(kStageBytes % 1024 == 0, "stages keep 1024-byte alignment");
+};
+
+struct SqLayer {
+  CUtensorMap xmap;                  // x [T][in]: box g x 128 rows (g = 128: two 64-wide slabs)
+  CUtensorMap wmap[kSqMaxMaps];      // tiles as [K g][g]: box heights g, 2g, ..., R g
+  const int32_t* gwoff;              // [Gin][nwin + 1]
+  const uint8_t* gwmask;             // [Gin][nwin]
+  uint16_t* y;
+  int32_t out, Gin, nwin, n_m, tile_begin;
+};
+struct SqParams {
+  SqLayer L[kSqMaxLayers];
+  int32_t n_layers, T, n_tiles;
+  int* err;
+};
+
+__device__ __forceinline__ int sq_layer_of(const SqParams& P, int t) {
+  int l = 0;
+  while (l + 1 < P.n_layers && P.L[l + 1].tile_begin <= t) ++l;
+  return l;
+}
+
+// UMMA shared-memory descriptor, K-major operand with the given swizzle
+// (layout type 2 / 4 / 6 = 128 / 64 / 32 bytes) and 8-row group stride.
+__device__ __forceinline__ uint64_t sq_desc(uint32_t saddr, uint32_t sbo, uint32_t swz) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1 << 16;                          // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;     // stride byte offset
+  d |= (uint64_t)1 << 46;                          // descriptor version
+  d |= (uint64_t)swz << 61;
+  return d;
+}
+
+// One round of a unit's items: column blocks c0 .. c0 + 31 whose window slice is
+// non-empty, written to buf in order as {v | n << 16 | mask << 24, first tile}.
+__device__ __forceinline__ int sq_items(const SqLayer& L, int w, int c0, int lane, uint2* buf) {
+  const int v = c0 + lane;
+  int p0 = 0, p1 = 0;
+  uint32_t mk = 0u;
+  if (v < L.Gin) {
+    const int32_t* wo = L.gwoff + (int64_t)v * (L.nwin + 1);
+    p0 = wo[w];
+    p1 = wo[w + 1];
+    mk = L.gwmask[(int64_t)v * L.nwin + w];
+  }
+  const bool ne = p1 > p0;
+  const uint32_t ballot = __ballot_sync(0xffffffffu, ne);
+  if (ne) buf[__popc(ballot & ((1u << lane) - 1u))] = make_uint2((uint32_t)v | ((uint32_t)(p1 - p0) << 16) | (mk << 24),
+                                                                 (uint32_t)p0);
+  __syncwarp();
+  return __popc(ballot);
+}
+
+__device__ __forceinline__ uint32_t sq_pack_bf16x2(float lo, float hi, bool keep) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(keep ? lo : 0.f, keep ? hi : 0.f);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ SqParams P) {
+  using C = Sq<G>;
+  extern __shared__ uint8_t sq_smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[C::kStages];
+  __shared__ __align__(8) uint64_t empty_bar[C::kStages];
+  __shared__ __align__(8) uint64_t afull_bar[kSqAccBufs];
+  __shared__ __align__(8) uint64_t aempty_bar[kSqAccBufs];
+  __shared__ __align__(8) uint64_t drain_bar;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sq_smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint2* ibuf = reinterpret_cast<uint2*>(smem + C::kStages * C::kStageBytes) + (warp < 2 ? warp : 0) * 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int b = 0; b < kSqAccBufs; ++b) {
+      mbar_init(&afull_bar[b], 1);
+      mbar_init(&aempty_bar[b], kSqEpiWarps);
+    }
+    mbar_init(&drain_bar, 1);
+    abort_s = 0;
+    fence_mbar_init();
+    for (int l = 0; l < P.n_layers; ++l) {
+      prefetch_tmap(&P.L[l].xmap);
+      for (int h = 0; h < C::R; ++h) prefetch_tmap(&P.L[l].wmap[h]);
+    }
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_s, kSqTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  volatile int* abort_flag = &abort_s;
+  const int n_tiles = P.n_tiles;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    uint32_t stage = 0, phase = 0;
+    uint32_t armed = 0u, armed_par = 0u;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      const SqLayer& L = P.L[sq_layer_of(P, t)];
+      const int lt = t - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      for (int c0 = 0; c0 < L.Gin && ok; c0 += 32) {
+        const int n_it = sq_items(L, w, c0, lane, ibuf);
+        if (lane == 0) {
+          for (int it = 0; it < n_it && ok; ++it) {
+            const uint2 e = ibuf[it];
+            const int v = (int)(e.x & 0xFFFFu), n = (int)((e.x >> 16) & 0xFFu), p0 = (int)e.y;
+            if (!mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kSqWaitLimitNs, kDevErrTimeout)) {
+              ok = false;
+              break;
+            }
+            uint8_t* sx = smem + stage * C::kStageBytes;
+            mbar_arrive_expect_tx(&full_bar[stage], C::kXBoxBytes + (uint32_t)(n * G * 2 * G));
+            if constexpr (G > 64) {
+              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kSqM, v * (G / 64));
+              tma_load_3d(sx + C::kRegion, &L.wmap[0], &full_bar[stage], 0, p0 * G, 0);
+            } else {
+              tma_load_2d(sx, &L.xmap, &full_bar[stage], v * G, m * kSqM);
+              tma_load_2d(sx + C::kRegion, &L.wmap[n - 1], &full_bar[stage], 0, p0 * G);
+            }
+            armed |= 1u << stage;
+            armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+            if (++stage == (uint32_t)C::kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      }
+    }
+    if (lane == 0 && !ok) {
+      // let copies already in flight land before the CTA retires
+      for (int s = 0; s < C::kStages; ++s) {
+        if (!((armed >> s) & 1u)) continue;
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(&full_bar[s], (armed_par >> s) & 1u))
+          if (globaltimer_ns() - t0 > kSqDrainLimitNs) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    uint32_t stage = 0, phase = 0;
+    int buf = 0;
+    uint32_t ae_ph = 0u;
+    bool ok = true;
+    constexpr uint32_t idesc = idesc_bf16_f32(kSqM, G);
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      const SqLayer& L = P.L[sq_layer_of(P, t)];
+      const int w = (t - L.tile_begin) / L.n_m;
+      if (lane == 0) {
+        ok = mbar_wait_bounded(&aempty_bar[buf], ((ae_ph >> buf) & 1u) ^ 1u, abort_flag, P.err, kSqWaitLimitNs,
+                               kDevErrTimeout);
+        ae_ph ^= 1u << buf;
+        tc_fence_after();
+      }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      const uint32_t d0 = tmem + (uint32_t)(buf * kSqWin);
+      uint32_t seen = 0u;   // block rows of this unit whose accumulator slice holds a result
+      for (int c0 = 0; c0 < L.Gin && ok; c0 += 32) {
+        const int n_it = sq_items(L, w, c0, lane, ibuf);
+        if (lane == 0) {
+          for (int it = 0; it < n_it && ok; ++it) {
+            const uint32_t mk = ibuf[it].x >> 24;
+            if (!mbar_wait_bounded(&full_bar[stage], phase, abort_flag, P.err, kSqWaitLimitNs, kDevErrTimeout)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sx = smem_u32(smem + stage * C::kStageBytes);
+            int i = 0;
+#pragma unroll
+            for (int b = 0; b < C::R; ++b) {
+              if (!((mk >> b) & 1u)) continue;
+              const uint32_t d = d0 + (uint32_t)(b * G);
+#pragma unroll
+              for (int kk = 0; kk < C::kKSteps; ++kk) {
+                const uint32_t koff = (uint32_t)((kk >> 2) * kSqSlabBytes + (kk & 3) * 32);
+                const uint64_t ad = sq_desc(sx + koff, C::kSBO, C::kSwz);
+                const uint64_t bd = sq_desc(sx + C::kRegion + (uint32_t)(i * G * C::kRowB) + koff, C::kSBO, C::kSwz);
+                mma_bf16_ss(d, ad, bd, idesc, (((seen >> b) & 1u) | (uint32_t)kk) != 0u ? 1u : 0u);
+              }
+              seen |= 1u << b;
+              ++i;
+            }
+            mma_commit(&empty_bar[stage]);
+            if (++stage == (uint32_t)C::kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      }
+      if (!ok) break;
+      if (lane == 0) mma_commit(&afull_bar[buf]);   // the unit's accumulator is complete once its MMAs are
+      buf ^= 1;
+    }
+    if (lane == 0) {
+      mma_commit(&drain_bar);
+      mbar_wait_bounded(&drain_bar, 0u, nullptr, P.err, kSqWaitLimitNs, kDevErrTimeout);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;   // TMEM lane quarter this warp may access
+    int buf = 0;
+    uint32_t af_ph = 0u;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      const SqLayer& L = P.L[sq_layer_of(P, t)];
+      const int lt = t - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      // block rows with at least one kept tile in the unit (the others are zero)
+      uint32_t seen = 0u;
+      for (int v = lane; v < L.Gin; v += 32) seen |= L.gwmask[(int64_t)v * L.nwin + w];
+      seen = __reduce_or_sync(0xffffffffu, seen);
+      if (!mbar_wait_bounded(&afull_bar[buf], (af_ph >> buf) & 1u, abort_flag, P.err, kSqWaitLimitNs,
+                             kDevErrTimeout)) {
+        ok = false;
+        break;
+      }
+      af_ph ^= 1u << buf;
+      tc_fence_after();
+      const int tok = m * kSqM + 32 * q + lane;
+      uint16_t* yrow = L.y + (int64_t)tok * L.out;
+#pragma unroll 1
+      for (int j = 0; j < kSqWin / 32; ++j) {
+        uint32_t v[32];
+        tmem_ld_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kSqWin + 32 * j), v);
+        tmem_wait_ld();
+        reg_fence(v);
+        const int r0 = w * kSqWin + 32 * j;
+        if (tok < P.T) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int rb = r0 + 8 * k;
+            const bool keep = (seen >> ((32 * j + 8 * k) / G)) & 1u;
+            if (rb + 8 <= L.out) {
+              const float* f = reinterpret_cast<const float*>(v + 8 * k);
+              *reinterpret_cast<uint4*>(yrow + rb) =
+                  make_uint4(sq_pack_bf16x2(f[0], f[1], keep), sq_pack_bf16x2(f[2], f[3], keep),
+                             sq_pack_bf16x2(f[4], f[5], keep), sq_pack_bf16x2(f[6], f[7], keep));
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&aempty_bar[buf]);
+      buf ^= 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kSqTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ packing
+// count: gwmask[v][w] = kept block rows of window w in column block v
+__global__ void k_sq_count(const uint8_t* __restrict__ mask, int32_t Gout, int32_t Gin, int32_t R, int32_t nwin,
+                           uint8_t* __restrict__ gwmask, int32_t* __restrict__ cnt) {
+  const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;   // e = v * nwin + w
+  if (e >= (int64_t)Gin * nwin) return;
+  const int v = (int)(e / nwin), w = (int)(e % nwin);
+  uint32_t bits = 0;
+  for (int i = 0; i < R; ++i) {
+    const int u = w * R + i;
+    if (u < Gout && mask[(int64_t)u * Gin + v] != 0) bits |= 1u << i;
+  }
+  gwmask[e] = (uint8_t)bits;
+  cnt[e] = __popc(bits);
+}
+
+__device__ __forceinline__ uint4 sq_ld16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+
+// compact + copy: one warp per group (u, v); a kept group's g x g block is
+// copied to its tile (16 bytes per lane per step) and its block row recorded
+__global__ void k_sq_compact(const uint16_t* __restrict__ W, const uint8_t* __restrict__ mask, int32_t g,
+                             int32_t in, int32_t Gout, int32_t Gin, int32_t R, int32_t nwin,
+                             const int32_t* __restrict__ gwoff, const uint8_t* __restrict__ gwmask,
+                             int32_t* __restrict__ row_idx, uint16_t* __restrict__ tiles) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const int per_row = g / 8;   // 16-byte pieces per block row
+  for (int64_t e = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < (int64_t)Gout * Gin;
+       e += warps) {
+    const int u = (int)(e / Gin), v = (int)(e % Gin);
+    if (mask[e] == 0) continue;
+    const int w = u / R, i = u % R;
+    const uint32_t mk = gwmask[(int64_t)v * nwin + w];
+    const int64_t j = gwoff[(int64_t)v * (nwin + 1) + w] + __popc(mk & ((1u << i) - 1u));
+    uint16_t* dst = tiles + j * (int64_t)g * g;
+    for (int c = lane; c < g * per_row; c += 32) {
+      const int r = c / per_row, k8 = c % per_row;
+      reinterpret_cast<uint4*>(dst + (int64_t)r * g)[k8] =
+          sq_ld16(W + ((int64_t)g * u + r) * in + (int64_t)g * v + 8 * k8);
+    }
+    if (lane == 0) row_idx[j] = u;
+  }
+}
+
+// unpack: one warp per group; kept groups copied back, pruned groups +0.0
+__global__ void k_sq_unpack(const uint16_t* __restrict__ tiles, int32_t g, int32_t in, int32_t Gout, int32_t Gin, int32_t R, int32_t nwin,
+                            const int32_t* __restrict__ gwoff, const uint8_t* __restrict__ gwmask,
+                            uint16_t* __restrict__ W_hat) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const int per_row = g / 8;
+  for (int64_t e = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < (int64_t)Gout * Gin;
+       e += warps) {
+    const int u = (int)(e / Gin), v = (int)(e % Gin);
+    const int w = u / R, i = u % R;
+    const uint32_t mk = gwmask[(int64_t)v * nwin + w];
+    const bool kept = (mk >> i) & 1u;
+    const int64_t j = gwoff[(int64_t)v * (nwin + 1) + w] + __popc(mk & ((1u << i) - 1u));
+    const uint16_t* src = tiles + j * (int64_t)g * g;
+    for (int c = lane; c < g * per_row; c += 32) {
+      const int r = c / per_row, k8 = c % per_row;
+      const uint4 val = kept ? sq_ld16(src + (int64_t)r * g + 8 * k8) : make_uint4(0u, 0u, 0u, 0u);
+      reinterpret_cast<uint4*>(W_hat + ((int64_t)g * u + r) * in + (int64_t)g * v)[k8] = val;
+    }
+  }
+}
+
+int sq_grid_for(int64_t warps_needed) {
+  int64_t b = (warps_needed + 7) / 8;
+  if (b < 1) b = 1;
+  if (b > (1 << 20)) b = 1 << 20;
+  return (int)b;
+}
+
+int sq_sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int G>
+cudaError_t sq_set_attr() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, []() {
+    err = cudaFuncSetAttribute(k_sq<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sq<G>::kSmem);
+  });
+  return err;
+}
+
+template <int G>
+gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int* idx, int nb, int64_t T,
+                    void* const* ys, int* err, cudaStream_t s) {
+  if (sq_set_attr<G>() != cudaSuccess) return GS_ERR_CUDA;
+  SqParams P;
+  std::memset(&P, 0, sizeof(P));
+  int64_t tiles = 0;
+  for (int k = 0; k < nb; ++k) {
+    const gs_packed* p = ps[idx[k]];
+    SqLayer& L = P.L[k];
+    bool ok;
+    if (G > 64)
+      ok = encode_tmap_slabs_bf16(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, kSqM, 2);
+    else
+      ok = encode_tmap_2d_bf16_swz(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, G, kSqM, Sq<G>::kRowB);
+    if (!ok) return GS_ERR_CUDA;
+    for (int h = 0; h < Sq<G>::R; ++h) std::memcpy(&L.wmap[h], p->gmaps[h], sizeof(CUtensorMap));
+    L.gwoff = p->gwoff;
+    L.gwmask = p->gwmask;
+    L.y = static_cast<uint16_t*>(ys[idx[k]]);
+    L.out = (int32_t)p->out;
+    L.Gin = p->G;
+    L.nwin = p->nwin;
+    L.n_m = (int32_t)((T + kSqM - 1) / kSqM);
+    L.tile_begin = (int32_t)tiles;
+    tiles += (int64_t)L.n_m * L.nwin;
+  }
+  if (tiles > INT32_MAX) return GS_ERR_UNSUPPORTED;
+  P.n_layers = nb;
+  P.T = (int32_t)T;
+  P.n_tiles = (int32_t)tiles;
+  P.err = err;
+  const int grid = (int)std::min<int64_t>(tiles, sq_sm_count());
+  k_sq<G><<<grid, kSqThreads, Sq<G>::kSmem, s>>>(P);
+  note_launch();
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
+
+}  // namespace
+
+bool sq_shape_supported(int g_out, int g_in) {
+  return g_out == g_in && (g_out == 16 || g_out == 32 || g_out == 64 || g_out == 128);
+}
+
+gs_status sq_pack(const void* W, const uint8_t* mask, gs_packed* p, cudaStream_t s) {
+  const int g = p->g_out;
+  const int R = kSqWin / g;
+  const int64_t Gin = p->G, Gout = p->Gout, nwin = p->nwin;
+  const int64_t E = Gin * nwin;
+  size_t total = 0;
+  auto alloc = [&](void** ptr, size_t bytes) -> gs_status {
+    if (bytes == 0) {
+      *ptr = nullptr;
+      return GS_OK;
+    }
+    const gs_status st = lib_malloc(ptr, bytes);
+    if (st == GS_OK) total += bytes;
+    return st;
+  };
+  gs_status st;
+  int32_t* cnt = nullptr;
+  if ((st = alloc((void**)&p->offsets, sizeof(int64_t) * (size_t)(Gin + 1))) != GS_OK) return st;
+  if ((st = alloc((void**)&p->gwoff, sizeof(int32_t) * (size_t)(Gin * (nwin + 1)))) != GS_OK) return st;
+  if ((st = alloc((void**)&p->gwmask, (size_t)E)) != GS_OK) return st;
+  if ((st = lib_malloc((void**)&cnt, sizeof(int32_t) * (size_t)E)) != GS_OK) return st;
+  k_sq_count<<<(unsigned)((E + 255) / 256), 256, 0, s>>>(mask, (int32_t)Gout, (int32_t)Gin, R, (int32_t)nwin,
+                                                         p->gwmask, cnt);
+  note_launch();
+  st = cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+  if (st == GS_OK) st = launch_scan_counts(cnt, (int32_t)Gin, (int32_t)nwin, p->gwoff, p->offsets, s);
+  int64_t kept = 0;
+  if (st == GS_OK && (cudaMemcpyAsync(&kept, p->offsets + Gin, sizeof(int64_t), cudaMemcpyDeviceToHost, s) !=
+                          cudaSuccess ||
+                      cudaStreamSynchronize(s) != cudaSuccess))
+    st = GS_ERR_CUDA;
+  cudaFree(cnt);
+  if (st != GS_OK) return st;
+  p->kept = kept;
+  const size_t tile_elems = (size_t)g * (size_t)g;
+  if ((st = alloc((void**)&p->row_idx, sizeof(int32_t) * (size_t)kept)) != GS_OK) return st;
+  if ((st = alloc((void**)&p->tiles, 2 * tile_elems * (size_t)kept)) != GS_OK) return st;
+  p->device_bytes = total;
+  if (kept > 0) {
+    k_sq_compact<<<sq_grid_for(Gout * Gin), 256, 0, s>>>(static_cast<const uint16_t*>(W), mask, g, (int32_t)p->in,
+                                                         (int32_t)Gout, (int32_t)Gin, R, (int32_t)nwin, p->gwoff,
+                                                         p->gwmask, p->row_idx, p->tiles);
+    note_launch();
+    if (cudaGetLastError() != cudaSuccess) return GS_ERR_CUDA;
+    // W slice descriptors: the tiles as a [K g][g] matrix (g = 128: 64-wide slabs)
+    for (int h = 0; h < R; ++h) {
+      CUtensorMap m;
+      const bool ok = g > 64 ? encode_tmap_slabs_bf16(&m, p->tiles, (uint64_t)g, (uint64_t)kept * g, (uint32_t)g, 2)
+                             : encode_tmap_2d_bf16_swz(&m, p->tiles, (uint64_t)g, (uint64_t)kept * g, (uint32_t)g,
+                                                       (uint32_t)((h + 1) * g), g >= 64 ? 128 : 2 * g);
+      if (!ok) return GS_ERR_CUDA;
+      std::memcpy(p->gmaps[h], &m, sizeof(m));
+    }
+  }
+  return GS_OK;
+}
+
+gs_status sq_unpack(const gs_packed* p, void* W_hat, cudaStream_t s) {
+  const int g = p->g_out;
+  k_sq_unpack<<<sq_grid_for((int64_t)p->Gout * p->G), 256, 0, s>>>(
+      p->tiles, g, (int32_t)p->in, p->Gout, p->G, kSqWin / g, p->nwin, p->gwoff, p->gwmask,
+      static_cast<uint16_t*>(W_hat));
+  note_launch();
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
+
+void sq_release(gs_packed* p) {
+  if (p->gwoff) cudaFree(p->gwoff);
+  if (p->gwmask) cudaFree(p->gwmask);
+  p->gwoff = nullptr;
+  p->gwmask = nullptr;
+}
+
+gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
+                            cudaStream_t s) {
+  if (T <= 0 || n <= 0) return GS_OK;
+  int* err = device_error_flag();
+  if (!err) return GS_ERR_CUDA;
+  // layers without kept groups produce zeros; the others share launches by
+  // group size, up to kSqMaxLayers each, most work per unit first
+  std::vector<int> order[4];
+  for (int i = 0; i < n; ++i) {
+    const gs_packed* p = ps[i];
+    if (p->kept == 0) {
+      if (cudaMemsetAsync(ys[i], 0, (size_t)T * (size_t)p->out * 2, s) != cudaSuccess) return GS_ERR_CUDA;
+      continue;
+    }
+    const int gi = p->g_out == 16 ? 0 : p->g_out == 32 ? 1 : p->g_out == 64 ? 2 : 3;
+    order[gi].push_back(i);
+  }
+  for (int gi = 0; gi < 4; ++gi) {
+    std::vector<int>& o = order[gi];
+    std::stable_sort(o.begin(), o.end(), [&](int a, int b) {
+      return (double)ps[a]->kept / ps[a]->nwin > (double)ps[b]->kept / ps[b]->nwin;
+    });
+    for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
+      const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
+      gs_status st;
+      switch (gi) {
+        case 0: st = sq_launch<16>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        case 1: st = sq_launch<32>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        case 2: st = sq_launch<64>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        default: st = sq_launch<128>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+      }
+      if (st != GS_OK) return st;
+    }
+  }
+  return GS_OK;
+}
+
+}  // namespace gs

@@ -200,6 +200,13 @@ gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }
 
+gs_status launch_scan_counts(const int32_t* cnt, int32_t G, int32_t nw, int32_t* win_off, int64_t* offsets,
+                             cudaStream_t s) {
+  k_pack_scan<<<1, kScanThreads, 0, s>>>(cnt, G, nw, win_off, offsets);
+  note_launch();
+  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
+
 gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s) {
   if (p->kept == 0) return GS_OK;
   k_pack_compact<<<grid_for(p->out, 8), 256, 0, s>>>(static_cast<const uint16_t*>(W), (int32_t)p->out,

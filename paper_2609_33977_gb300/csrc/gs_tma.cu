@@ -43,6 +43,28 @@ bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t o
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_tmap_2d_bf16_swz(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                             uint32_t box_outer, int swizzle_bytes) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  CUtensorMapSwizzle sw;
+  switch (swizzle_bytes) {
+    case 32: sw = CU_TENSOR_MAP_SWIZZLE_32B; break;
+    case 64: sw = CU_TENSOR_MAP_SWIZZLE_64B; break;
+    case 128: sw = CU_TENSOR_MAP_SWIZZLE_128B; break;
+    default: return false;
+  }
+  // a swizzled box row must fit the swizzle width
+  if (box_inner * 2u > (uint32_t)swizzle_bytes) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(static_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool encode_tmap_slabs_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows, uint32_t box_rows,
                             uint32_t box_slabs) {
   EncodeTiledFn fn = encode_fn();

@@ -31,6 +31,8 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib = ctypes.CDLL(str(path))
     vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
     lib.gs_pack.argtypes = [vp, vp, i64, i64, i32, vp, ctypes.POINTER(vp)]
+    lib.gs_pack_groups.argtypes = [vp, vp, i64, i64, i32, i32, vp, ctypes.POINTER(vp)]
+    lib.gs_packed_group_shape.argtypes = [vp, _c_i32p, _c_i32p]
     lib.gs_linear.argtypes = [vp, vp, i64, vp, vp]
     lib.gs_linear_ex.argtypes = [vp, vp, i64, vp, vp, ctypes.c_int]
     lib.gs_linear_batched.argtypes = [i32, ctypes.POINTER(vp), ctypes.POINTER(vp), i64, ctypes.POINTER(vp), vp]
@@ -50,7 +52,8 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib.gs_debug_inject_wait.argtypes = [ctypes.c_int, ctypes.c_uint64]
     for fn in (lib.gs_pack, lib.gs_linear, lib.gs_linear_ex, lib.gs_linear_batched, lib.gs_unpack,
                lib.gs_packed_info, lib.gs_packed_export, lib.gs_device_status, lib.gs_select_groups,
-               lib.gs_preserved_rates, lib.gs_debug_fail_alloc, lib.gs_debug_inject_wait):
+               lib.gs_preserved_rates, lib.gs_debug_fail_alloc, lib.gs_debug_inject_wait, lib.gs_pack_groups,
+               lib.gs_packed_group_shape):
         fn.restype = ctypes.c_int
     return lib
 
@@ -86,10 +89,12 @@ def _require_cuda(t: torch.Tensor, dtype: torch.dtype, name: str) -> None:
 class Packed:
     """A packed group-sparse weight (owns the library handle)."""
 
-    def __init__(self, handle: int, out: int, inp: int):
+    def __init__(self, handle: int, out: int, inp: int, g_out: int = 1, g_in: int = 256):
         self._h = ctypes.c_void_p(handle)
         self.out = out
         self.inp = inp
+        self.g_out = g_out
+        self.g_in = g_in
 
     @property
     def handle(self) -> ctypes.c_void_p:
@@ -99,7 +104,7 @@ class Packed:
 
     @property
     def G(self) -> int:
-        return self.inp // 256
+        return self.inp // self.g_in
 
     def info(self):
         out, inp, kept = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
@@ -113,9 +118,17 @@ class Packed:
         return self.info()["kept"]
 
     def export(self):
-        """Host copies of the packed layout: offsets, row_idx, tiles, win_off16, kmask16."""
+        """Host copies of the packed layout: offsets, row_idx, tiles, win_off16, kmask16
+        (square groups: offsets, row_idx = block rows, tiles [K, g, g])."""
         K = self.kept
         G = self.G
+        if self.g_out > 1:
+            offsets = np.zeros(G + 1, np.int64)
+            rows = np.zeros(max(K, 1), np.int32)
+            tiles = np.zeros((max(K, 1), self.g_out, self.g_in), np.uint16)
+            _check(lib.gs_packed_export(self.handle, offsets.ctypes.data_as(_c_i64p), rows.ctypes.data_as(_c_i32p),
+                                        tiles.ctypes.data_as(_c_u16p), None, None), "gs_packed_export")
+            return {"offsets": offsets, "row_idx": rows[:K], "tiles": tiles[:K]}
         nw16 = (self.out + 15) // 16
         offsets = np.zeros(G + 1, np.int64)
         row_idx = np.zeros(max(K, 1), np.int32)
@@ -152,6 +165,23 @@ def pack(W: torch.Tensor, mask: torch.Tensor, stream: Optional[torch.cuda.Stream
     _check(lib.gs_pack(W.data_ptr(), mask.data_ptr(), out, inp, 256, _stream_ptr(stream), ctypes.byref(h)),
            "gs_pack")
     return Packed(h.value, out, inp)
+
+
+def pack_groups(W: torch.Tensor, mask: torch.Tensor, g_out: int, g_in: int,
+                stream: Optional[torch.cuda.Stream] = None) -> Packed:
+    """Pack a bf16 weight [out, in] with a group mask [out/g_out, in/g_in] (nonzero = keep)
+    for g_out x g_in groups: (1, 256) or square g x g, g in {16, 32, 64, 128}."""
+    _require_cuda(W, torch.bfloat16, "W")
+    if mask.dtype == torch.bool:
+        mask = mask.to(torch.uint8)
+    _require_cuda(mask, torch.uint8, "mask")
+    out, inp = W.shape
+    if out % g_out or inp % g_in or tuple(mask.shape) != (out // g_out, inp // g_in):
+        raise ValueError("mask must be [out/g_out, in/g_in] and the groups must tile W")
+    h = ctypes.c_void_p()
+    _check(lib.gs_pack_groups(W.data_ptr(), mask.data_ptr(), out, inp, g_out, g_in, _stream_ptr(stream),
+                              ctypes.byref(h)), "gs_pack_groups")
+    return Packed(h.value, out, inp, g_out, g_in)
 
 
 def linear_into(x: torch.Tensor, p: Packed, y: torch.Tensor, algo: int = ALGO_AUTO,
