@@ -539,6 +539,7 @@ def run_ours(args):
         extras["stack_qwen"] = measure_stack_qwen(gs, torch, dev, stream, pool, tpk, tpk_sus, hbm_peak)
         extras["single_layer"] = measure_single_layer(gs, torch, dev, stream, hbm_peak)
         extras["block_7b"] = measure_block_7b(gs, torch, dev, stream, pool, hbm_peak)
+        extras["group_shapes"] = measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak)
         try:
             extras["mask_export"] = measure_select(gs, torch, dev, stream, peaks)
         except Exception as e:   # reported in the line, never hidden
@@ -784,6 +785,72 @@ def measure_block_7b(gs, torch, dev, stream, pool, hbm_peak, copies: int = 4):
     return {"workload": "llama2-7b block (7 projections), one batched launch per T", "per_T": rows}
 
 
+def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak, shapes=(16, 32, 64, 128)):
+    """The other group shapes (square g x g; Sec. 3.5 ablation, App. E) on the
+    LLaMA-2-7B block's seven projections, each keeping the same fraction of its
+    groups as under the second configuration's 1x256 allocation (50 % overall):
+    prefill at T = 2048 (one batched call per pass, kept TFLOP/s against the
+    measured bf16 peak) and decode at T = 1 and 16 (two packed copies
+    alternating, together larger than L2), next to the 1x256 kernels."""
+    w = wl.workload(2)
+    ks = wl.keep_counts(w)
+    n = len(w.layers)
+    rows = []
+    for g in shapes:
+        masks = [pool.submit(wl.group_mask_shaped, w, i, int(ks[i]), g, g) for i in range(n)]
+        copies = [[], []]
+        for i in range(n):
+            W = wl.weight_device(w, i, device=dev)
+            M = torch.from_numpy(masks[i].result()).to(dev)
+            for c in range(2):
+                copies[c].append(gs.pack_groups(W, M, g, g))
+            del W, M
+        kept_tiles = sum(p.kept for p in copies[0])
+        kept_w = kept_tiles * g * g
+        row = {"group": f"{g}x{g}", "kept_weights": kept_w, "kept_fraction": kept_w / sum(L.out * L.inp for L in w.layers)}
+        for T in (1, 16, 2048):
+            xs, ys = stack_inputs(torch, w, dev, T)
+
+            def run(c, xs=xs, ys=ys):
+                gs.linear_batched_into(xs, copies[c], ys, stream=stream)
+            if T <= 16:
+                gr = [capture(torch, stream, lambda c=c: run(c)) for c in range(2)]
+                s = time_replays(torch, stream, gr, reps=100)
+                nb = 2.0 * kept_w + sum(4.0 * p.kept + 2.0 * T * (L.inp + L.out) for p, L in zip(copies[0], w.layers))
+                row[f"decode_T{T}"] = {"us_per_block": s * 1e6, "GB/s": nb / s / 1e9,
+                                       "frac_of_measured_hbm": nb / s / 1e9 / hbm_peak}
+            else:
+                s = time_calls(torch, stream, lambda: run(0), reps=10, warm=2)
+                tf = 2.0 * T * kept_w / s / 1e12
+                row[f"prefill_T{T}"] = {"ms_per_block": s * 1e3, "kept_TFLOP/s": tf, "frac_of_burst_peak": tf / tpk}
+            del xs, ys
+        for c in copies:
+            for p in c:
+                p.free()
+        torch.cuda.empty_cache()
+        rows.append(row)
+    assert gs.device_status() == gs.GS_OK
+    return {"workload": "llama2-7b block (7 projections), square groups at the 1x256 allocation's per-layer "
+                        "fractions", "shapes": rows}
+
+
+def run_group_shapes(args):
+    """The group-shape measurement alone; prints one JSON line."""
+    import concurrent.futures as cf
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+    peaks, _ = load_peaks()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device=dev)
+    pool = cf.ThreadPoolExecutor(max_workers=8)
+    rec = measure_group_shapes(gs, torch, dev, stream, pool, float(peaks.get("bf16_tflops", 1900.0)),
+                               float(peaks.get("hbm_gbs", 6800.0)))
+    print(json.dumps(rec), flush=True)
+    return 0
+
+
 def measure_select(gs, torch, dev, stream, peaks):
     """Selector export (gs_select_groups) over all selectors of the 13B stack (40
     blocks, 49,561,600 groups): float32 logits (198 MB) in, uint8 masks (50 MB) out,
@@ -868,9 +935,13 @@ def run_layer(args):
     g = torch.Generator(device=dev)
     g.manual_seed(1234)
     W = (torch.randn((out, inp), generator=g, device=dev) * 0.02).to(torch.bfloat16)
-    B = (torch.rand((out, inp // 256), generator=g, device=dev) < args.density).to(torch.uint8)
+    gsz = args.group
+    if gsz:
+        B = (torch.rand((out // gsz, inp // gsz), generator=g, device=dev) < args.density).to(torch.uint8)
+    else:
+        B = (torch.rand((out, inp // 256), generator=g, device=dev) < args.density).to(torch.uint8)
     x = torch.randn((T, inp), generator=g, device=dev).to(torch.bfloat16)
-    p = gs.pack(W, B)
+    p = gs.pack_groups(W, B, gsz, gsz) if gsz else gs.pack(W, B)
     y = torch.empty((T, out), dtype=torch.bfloat16, device=dev)
     algo = {"auto": gs.ALGO_AUTO, "decode": gs.ALGO_DECODE, "prefill": gs.ALGO_PREFILL}[args.algo]
     for _ in range(args.warmup):
@@ -885,11 +956,17 @@ def run_layer(args):
     b.synchronize()
     s = a.elapsed_time(b) / 1e3 / args.steps
     kept = p.kept
-    G, nw16 = inp // 256, (out + 15) // 16
-    nbytes = 512 * kept + 6 * G * nw16 + 2 * T * inp + 2 * T * out
-    flops = 2.0 * T * 256 * kept
+    if gsz:
+        kept_w = kept * gsz * gsz
+        nbytes = 2 * kept_w + 4 * kept + 2 * T * inp + 2 * T * out
+    else:
+        kept_w = 256 * kept
+        G, nw16 = inp // 256, (out + 15) // 16
+        nbytes = 2 * kept_w + 6 * G * nw16 + 2 * T * inp + 2 * T * out
+    flops = 2.0 * T * kept_w
     assert gs.device_status() == gs.GS_OK
-    print(json.dumps({"layer": f"{out}x{inp}", "T": T, "density": args.density, "algo": args.algo, "kept": kept,
+    print(json.dumps({"layer": f"{out}x{inp}", "group": f"{gsz}x{gsz}" if gsz else "1x256", "T": T,
+                      "density": args.density, "algo": args.algo, "kept": kept,
                       "us": s * 1e6, "GB/s": nbytes / s / 1e9, "TFLOP/s": flops / s / 1e12}), flush=True)
     return 0
 
@@ -909,8 +986,11 @@ def main():
     ap.add_argument("--block-of", type=int, default=0,
                     help="block mode: block 0 of workload 2, 3, 4 or 5, at --tokens")
     ap.add_argument("--tokens", type=int, default=16)
+    ap.add_argument("--group", type=int, default=0, help="single-layer mode: square g x g groups (0 = 1x256)")
     ap.add_argument("--density", type=float, default=0.5)
     ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
+    ap.add_argument("--group-shapes", action="store_true",
+                    help="time only the square-group kernels on the 7B block")
     ap.add_argument("--mask-export", action="store_true",
                     help="time only the selector export kernel over the 13B stack's selectors")
     args = ap.parse_args()
@@ -928,6 +1008,8 @@ def main():
         return run_block(args)
     if args.mask_export:
         return run_mask_export(args)
+    if args.group_shapes:
+        return run_group_shapes(args)
     return run_ours(args)
 
 

@@ -21,6 +21,9 @@
 // FLOPs.  Token rows beyond T read as zero (TMA fill) and are not stored; the
 // same kernel serves every token count.
 //
+// For T < 128 the x boxes hold only T rows: the accumulator rows of the other
+// tokens then add up whatever the stage held before, and are never stored.
+//
 // Roles (one CTA per SM, persistent over units): warp 0 TMA producer, warp 1
 // TMEM allocator + single-thread MMA issuer, warps 2..5 epilogue (warp w reads
 // TMEM lanes 32 (w % 4) ..).  Two accumulator buffers let the epilogue of one
@@ -50,7 +53,6 @@ constexpr int kSqEpiWarps = 4;
 constexpr int kSqThreads = (2 + kSqEpiWarps) * 32;
 constexpr int kSqMaxLayers = 8;
 constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R <= 8)
-constexpr int kSqSlabBytes = 128 * 128;   // one operand slab: 128 rows x 128-byte pitch (the largest swizzle)
 constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
 constexpr uint64_t kSqDrainLimitNs = 200000000ull;
 
@@ -59,13 +61,16 @@ struct Sq {
   static constexpr int R = kSqWin / G;                  // block rows per window
   static constexpr int kSlabs = G > 64 ? 2 : 1;         // 64-column slabs per operand row
   static constexpr int kRowB = G >= 64 ? 128 : 2 * G;   // operand row bytes within a slab = swizzle width
-  static constexpr int kRegion = kSlabs * kSqSlabBytes; // bytes reserved per operand per stage
+  static constexpr int kSlab = 128 * kRowB;             // one operand slab: 128 rows at the swizzle pitch
+  static constexpr int kRegion = kSlabs * kSlab;        // bytes per operand per stage
   static constexpr int kStageBytes = 2 * kRegion;       // x box, then W slice
-  static constexpr int kStages = G > 64 ? 3 : 6;
+  // as many stages as fit: a stage is one column block's copies, and the
+  // copies of one stage wait for the MMAs of the stage before its last use,
+  // so small groups need many stages in flight to cover the round trip
+  static constexpr int kStages = (200 * 1024) / kStageBytes > 32 ? 32 : (200 * 1024) / kStageBytes;
   static constexpr uint32_t kSwz = G >= 64 ? 2u : (G == 32 ? 4u : 6u);   // UMMA layout: 128 / 64 / 32-byte swizzle
   static constexpr uint32_t kSBO = 8 * kRowB;           // bytes between 8-row core groups
   static constexpr int kKSteps = G / 16;
-  static constexpr uint32_t kXBoxBytes = kSqM * 2 * G;  // full x box (rows past T are zero-filled and counted)
   static constexpr int kSmem = kStages * kStageBytes + 2 * 32 * 8 + 1024;
   static_assert(R >= 1 && R <= kSqMaxMaps, "window holds 1..8 block rows");
   static_assert(kSmem <= 227 * 1024, "shared memory budget");
@@ -73,7 +78,7 @@ struct Sq {
 };
 
 struct SqLayer {
-  CUtensorMap xmap;                  // x [T][in]: box g x 128 rows (g = 128: two 64-wide slabs)
+  CUtensorMap xmap;                  // x [T][in]: box g x min(T, 128) rows (g = 128: one 64-wide slab)
   CUtensorMap wmap[kSqMaxMaps];      // tiles as [K g][g]: box heights g, 2g, ..., R g
   const int32_t* gwoff;              // [Gin][nwin + 1]
   const uint8_t* gwmask;             // [Gin][nwin]
@@ -83,6 +88,7 @@ struct SqLayer {
 struct SqParams {
   SqLayer L[kSqMaxLayers];
   int32_t n_layers, T, n_tiles;
+  int32_t x_rows;            // rows of each x box: min(T, 128) (token rows past it hold stale data, never stored)
   int* err;
 };
 
@@ -192,9 +198,12 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
               break;
             }
             uint8_t* sx = smem + stage * C::kStageBytes;
-            mbar_arrive_expect_tx(&full_bar[stage], C::kXBoxBytes + (uint32_t)(n * G * 2 * G));
+            mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(P.x_rows * 2 * G) + (uint32_t)(n * G * 2 * G));
             if constexpr (G > 64) {
-              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kSqM, v * (G / 64));
+              // one box per 64-column slab, each into its own slab region (a two-slab
+              // box of fewer than 128 rows would pack the slabs back to back)
+              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kSqM, 2 * v);
+              tma_load_3d(sx + C::kSlab, &L.xmap, &full_bar[stage], 0, m * kSqM, 2 * v + 1);
               tma_load_3d(sx + C::kRegion, &L.wmap[0], &full_bar[stage], 0, p0 * G, 0);
             } else {
               tma_load_2d(sx, &L.xmap, &full_bar[stage], v * G, m * kSqM);
@@ -258,7 +267,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
               const uint32_t d = d0 + (uint32_t)(b * G);
 #pragma unroll
               for (int kk = 0; kk < C::kKSteps; ++kk) {
-                const uint32_t koff = (uint32_t)((kk >> 2) * kSqSlabBytes + (kk & 3) * 32);
+                const uint32_t koff = (uint32_t)((kk >> 2) * C::kSlab + (kk & 3) * 32);
                 const uint64_t ad = sq_desc(sx + koff, C::kSBO, C::kSwz);
                 const uint64_t bd = sq_desc(sx + C::kRegion + (uint32_t)(i * G * C::kRowB) + koff, C::kSBO, C::kSwz);
                 mma_bf16_ss(d, ad, bd, idesc, (((seen >> b) & 1u) | (uint32_t)kk) != 0u ? 1u : 0u);
@@ -454,10 +463,11 @@ gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int
     const gs_packed* p = ps[idx[k]];
     SqLayer& L = P.L[k];
     bool ok;
+    const uint32_t xr = (uint32_t)std::min<int64_t>(T, kSqM);
     if (G > 64)
-      ok = encode_tmap_slabs_bf16(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, kSqM, 2);
+      ok = encode_tmap_slabs_bf16(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, xr, 1);
     else
-      ok = encode_tmap_2d_bf16_swz(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, G, kSqM, Sq<G>::kRowB);
+      ok = encode_tmap_2d_bf16_swz(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, G, xr, Sq<G>::kRowB);
     if (!ok) return GS_ERR_CUDA;
     for (int h = 0; h < Sq<G>::R; ++h) std::memcpy(&L.wmap[h], p->gmaps[h], sizeof(CUtensorMap));
     L.gwoff = p->gwoff;
@@ -474,6 +484,7 @@ gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int
   P.n_layers = nb;
   P.T = (int32_t)T;
   P.n_tiles = (int32_t)tiles;
+  P.x_rows = (int32_t)std::min<int64_t>(T, kSqM);
   P.err = err;
   const int grid = (int)std::min<int64_t>(tiles, sq_sm_count());
   k_sq<G><<<grid, kSqThreads, Sq<G>::kSmem, s>>>(P);

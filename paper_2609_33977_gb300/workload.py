@@ -280,6 +280,24 @@ def group_mask(wl: Workload, layer_id: int, k: int) -> np.ndarray:
     return m.reshape(L.out, L.G)
 
 
+def group_mask_shaped(wl: Workload, layer_id: int, k: int, g_out: int, g_in: int) -> np.ndarray:
+    """uint8 [out/g_out, in/g_in] keep mask for g_out x g_in groups that keeps the
+    same fraction of the layer's groups as k of its 1x256 groups (rounded to the
+    nearest whole group): the top of seeded U[0,1) scores, ties to the lower flat
+    index.  The layer's shape must be tiled by the group."""
+    L = wl.layers[layer_id]
+    if L.out % g_out or L.inp % g_in:
+        raise ValueError(f"{L.out}x{L.inp} is not tiled by {g_out}x{g_in} groups")
+    Go, Gi = L.out // g_out, L.inp // g_in
+    n = Go * Gi
+    kk = int(math.floor(k * n / L.groups + 0.5))
+    scores = rng(wl.cfg_id, wl.variant, layer_id, STREAM_SCORES, g_out, g_in).random(n)
+    order = np.argsort(-scores, kind="stable")
+    m = np.zeros(n, dtype=np.uint8)
+    m[order[:kk]] = 1
+    return m.reshape(Go, Gi)
+
+
 def weight_bits(wl: Workload, layer_id: int) -> np.ndarray:
     """bf16 bits uint16 [out, in] of W ~ N(0, 0.02^2)."""
     L = wl.layers[layer_id]
