@@ -87,8 +87,11 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
  * non-overlapping g_out x g_in groups and B[G_out][G_in] keeps or prunes each
  * (Eq. 1 with M = B (x) 1_{g_out x g_in}); the Sec. 3.5 granularity ablation
  * and App. E evaluate 1 x 128, 1 x 256, 16 x 16, 32 x 32, 64 x 64 and
- * 128 x 128.  Supported here: (1, 256), which is gs_pack itself, and square
- * g x g with g in {16, 32, 64, 128}; other shapes return GS_ERR_UNSUPPORTED.
+ * 128 x 128.  Supported here: (1, 256), which is gs_pack itself, (1, 128),
+ * whose layout is gs_pack's with 128-wide chunks (offsets, row_idx, tiles of
+ * 128 bf16, win_off16 and kmask16 as gs_pack describes them, over chunks of
+ * 128 input columns), and square g x g with g in {16, 32, 64, 128}; other
+ * shapes return GS_ERR_UNSUPPORTED.
  *
  * Packed layout of square groups (bit-exact, deterministic): column block v
  * (input columns [g v, g v + g)) owns packed tiles [offsets[v], offsets[v+1]);
@@ -201,6 +204,8 @@ gs_status gs_packed_info(const gs_packed* p, int64_t* out, int64_t* in, int64_t*
  * that gs_pack describes.  Sizes: offsets int64[G+1], row_idx int32[K],
  * tiles uint16[K*256], win_off16 int32[G*(ceil(out/16)+1)],
  * kmask16 uint16[G*ceil(out/16)], with K = kept_groups.  Any pointer may be NULL.
+ * For 1 x 128 handles the chunks are 128 wide: G = in/128 and tiles
+ * uint16[K*128].
  * For handles of square g x g groups (gs_pack_groups): offsets int64[in/g+1],
  * row_idx int32[K] (block rows), tiles uint16[K*g*g]; win_off16 and kmask16
  * must be NULL (INVALID_ARG otherwise).

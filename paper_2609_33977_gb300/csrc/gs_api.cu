@@ -113,15 +113,17 @@ using namespace gs;
 
 extern "C" {
 
-gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t group_in,
-                  void* stream, gs_packed** handle) {
+// Row groups 1 x kw (kw = 256 or 128): the chunk-major layout and everything
+// the decode and prefill kernels need.
+static gs_status pack_rows(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t kw,
+                           void* stream, gs_packed** handle) {
   if (handle) *handle = nullptr;
   if (!W_dev || !mask_dev || !handle) return GS_ERR_INVALID_ARG;
   if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX) return GS_ERR_INVALID_ARG;
-  if (group_in != kGroupIn) return GS_ERR_UNSUPPORTED;
-  if (in % kGroupIn != 0) return GS_ERR_INVALID_ARG;
+  if (kw != 256 && kw != 128) return GS_ERR_UNSUPPORTED;
+  if (in % kw != 0) return GS_ERR_INVALID_ARG;
   if (!aligned16(W_dev)) return GS_ERR_INVALID_ARG;
-  const int64_t G = in / kGroupIn;
+  const int64_t G = in / kw;
   if (out * G >= (int64_t)INT32_MAX) return GS_ERR_UNSUPPORTED;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
 
@@ -141,7 +143,7 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
   p->G = (int32_t)G;
   p->nw16 = (int32_t)((out + kWin16 - 1) / kWin16);
   p->g_out = 1;
-  p->g_in = kGroupIn;
+  p->g_in = kw;
   p->Gout = (int32_t)out;
 
   size_t total = 0;
@@ -170,7 +172,7 @@ gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64
   cudaFree(cnt);
   cnt = nullptr;
   if ((st = dev_alloc((void**)&p->row_idx, sizeof(int32_t) * (size_t)p->kept, &total)) != GS_OK) goto fail;
-  if ((st = dev_alloc((void**)&p->tiles, (size_t)kTileBytes * (size_t)p->kept, &total)) != GS_OK) goto fail;
+  if ((st = dev_alloc((void**)&p->tiles, 2 * (size_t)kw * (size_t)p->kept, &total)) != GS_OK) goto fail;
   p->device_bytes = total;
   if ((st = launch_pack_compact(W_dev, p, s)) != GS_OK) goto fail;
   if ((st = decode_prepare(p, s)) != GS_OK) goto fail;
@@ -185,12 +187,20 @@ fail:
   return st;
 }
 
+gs_status gs_pack(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t group_in,
+                  void* stream, gs_packed** handle) {
+  if (handle) *handle = nullptr;
+  if (!W_dev || !mask_dev || !handle) return GS_ERR_INVALID_ARG;
+  if (group_in != kGroupIn) return GS_ERR_UNSUPPORTED;
+  return pack_rows(W_dev, mask_dev, out, in, kGroupIn, stream, handle);
+}
+
 gs_status gs_pack_groups(const void* W_dev, const uint8_t* mask_dev, int64_t out, int64_t in, int32_t g_out,
                          int32_t g_in, void* stream, gs_packed** handle) {
   if (handle) *handle = nullptr;
   if (!W_dev || !mask_dev || !handle) return GS_ERR_INVALID_ARG;
   if (out <= 0 || in <= 0 || out > INT32_MAX || in > INT32_MAX || g_out <= 0 || g_in <= 0) return GS_ERR_INVALID_ARG;
-  if (g_out == 1 && g_in == kGroupIn) return gs_pack(W_dev, mask_dev, out, in, g_in, stream, handle);
+  if (g_out == 1 && (g_in == 256 || g_in == 128)) return pack_rows(W_dev, mask_dev, out, in, g_in, stream, handle);
   if (!sq_shape_supported(g_out, g_in)) return GS_ERR_UNSUPPORTED;
   if (out % g_out != 0 || in % g_in != 0) return GS_ERR_INVALID_ARG;   // the groups must tile W exactly
   if (!aligned16(W_dev)) return GS_ERR_INVALID_ARG;
@@ -302,6 +312,23 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
       if (st != GS_OK) return st;
       if (pr.empty()) return GS_OK;
       return gs_linear_batched((int32_t)pr.size(), xr.data(), pr.data(), T, yr.data(), stream);
+    }
+    // 1 x 128 and 1 x 256 layers take separate launches (one chunk width per kernel)
+    int n128 = 0;
+    for (int i = 0; i < n; ++i) n128 += ps[i]->g_in == 128 ? 1 : 0;
+    if (n128 > 0 && n128 < n) {
+      std::vector<const void*> xa, xb;
+      std::vector<const gs_packed*> pa, pb;
+      std::vector<void*> ya, yb;
+      for (int i = 0; i < n; ++i) {
+        const bool narrow = ps[i]->g_in == 128;
+        (narrow ? xa : xb).push_back(xs_dev[i]);
+        (narrow ? pa : pb).push_back(ps[i]);
+        (narrow ? ya : yb).push_back(ys_dev[i]);
+      }
+      const gs_status st = gs_linear_batched((int32_t)pa.size(), xa.data(), pa.data(), T, ya.data(), stream);
+      if (st != GS_OK) return st;
+      return gs_linear_batched((int32_t)pb.size(), xb.data(), pb.data(), T, yb.data(), stream);
     }
   }
   if (T >= kPrefillMinTokens) {

@@ -89,7 +89,7 @@ constexpr uint64_t kDecDrainLimitNs = 200000000ull;
 struct DecLayer {
   CUtensorMap xmap;      // x [T][in] as (64, T, in/64) slabs, box 64 x T x 4, 128-byte swizzle
   const uint16_t* x;     // [T][in]
-  const uint16_t* tiles; // [kept][256]
+  const uint16_t* tiles; // [kept][chunk width]
   const int4* dmeta;     // [nblk][G]
   uint16_t* y;           // [T][out]
   float* ws;             // [nblk][nsplit][4][kPartFloats]
@@ -168,8 +168,10 @@ __device__ __forceinline__ void unit_at(const int4* lay, int n_layers, int u, Un
   U.nC = min(L.w, U.c0 + L.z) - U.c0;
 }
 
-template <int NT, int MB>
+// KW = chunk width: 256 (1 x 256 groups) or 128 (1 x 128 groups)
+template <int NT, int MB, int KW>
 __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant__ DecParams<MB> P) {
+  static_assert(KW == 128 || KW == 256, "chunk width");
   extern __shared__ uint8_t dsmem_raw[];
   __shared__ __align__(8) uint64_t w_full[kRingSeq];
   __shared__ __align__(8) uint64_t w_empty[kRingSeq];
@@ -305,7 +307,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
       prefetch(V, have_v);                       // in flight while this unit's copies are issued
       if (lane == 0) {
         const DecLayer& L = P.L[U.l];
-        const uint32_t xbytes = (uint32_t)T * kXRow;
+        const uint32_t xbytes = (uint32_t)T * (uint32_t)(2 * KW);
         // first unit only: wait for the previous grid, then issue the pending
         // x boxes and take the ticket of the unit after next
         auto resolve = [&]() {
@@ -313,7 +315,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           for (uint32_t i = 0; i < n_pend; ++i) {
             const int4 mp = mrow[i];
             if ((mp.y | mp.z) != 0)
-              tma_load_3d(ring + w_off[i], &L.xmap, &w_full[i], 0, 0, (U.c0 + (int)i) * (kGroupIn / 64));
+              tma_load_3d(ring + w_off[i], &L.xmap, &w_full[i], 0, 0, (U.c0 + (int)i) * (KW / 64));
           }
           if (u_next < P.n_units) t_ahead = n_static + atomicAdd(P.sched, 1);
           dep = true;
@@ -323,7 +325,7 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           const int4 m = m_next;
           if (i + 1 < U.nC) m_next = mrow[i + 1];
           const uint32_t cnt = __popc((uint32_t)m.y) + __popc((uint32_t)m.z);
-          const uint32_t bytes = cnt * (uint32_t)kTileBytes;
+          const uint32_t bytes = cnt * (uint32_t)(2 * KW);
           const uint32_t need = cnt ? bytes + xbytes : 0u;
           // allocate `need` contiguous bytes from a 1024-byte boundary (the swizzled x box);
           // a chunk that would straddle the end starts over at offset 0
@@ -360,8 +362,8 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
           fence_proxy_async_smem();
           mbar_arrive_expect_tx(&w_full[e], cnt ? bytes + xbytes : 0u);
           if (cnt) {
-            if (dep) tma_load_3d(dst, &L.xmap, &w_full[e], 0, 0, (U.c0 + i) * (kGroupIn / 64));
-            bulk_copy_g2s(dst + xbytes, L.tiles + (int64_t)m.x * kGroupIn, bytes, &w_full[e]);
+            if (dep) tma_load_3d(dst, &L.xmap, &w_full[e], 0, 0, (U.c0 + i) * (KW / 64));
+            bulk_copy_g2s(dst + xbytes, L.tiles + (int64_t)m.x * KW, bytes, &w_full[e]);
           }
           if (!dep) ++n_pend;
         }
@@ -431,11 +433,11 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
         if (km != 0u) {
           const bool kg = (km >> g) & 1u, kg8 = (km >> (g + 8)) & 1u;
           const uint8_t* cbase = ring + w_off[slot];
-          const uint4* sl = reinterpret_cast<const uint4*>(cbase + T * kXRow);
-          const uint4* tg = sl + (base + __popc(km & lo_g)) * 32 + 2 * qd;
-          const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * 32 + 2 * qd;
+          const uint4* sl = reinterpret_cast<const uint4*>(cbase + T * (2 * KW));
+          const uint4* tg = sl + (base + __popc(km & lo_g)) * (KW / 8) + 2 * qd;
+          const uint4* tg8 = sl + (base + __popc(km & lo_g8)) * (KW / 8) + 2 * qd;
 #pragma unroll
-          for (int b = 0; b < 8; ++b) {
+          for (int b = 0; b < KW / 32; ++b) {
             const int j = 8 * (b >> 1) + (b & 1);
             const uint4 a = kg ? tg[j] : make_uint4(0u, 0u, 0u, 0u);
             const uint4 a8 = kg8 ? tg8[j] : make_uint4(0u, 0u, 0u, 0u);
@@ -594,12 +596,12 @@ int sm_count_dec() {
   return n;
 }
 
-template <int NT, int MB>
+template <int NT, int MB, int KW>
 cudaError_t launch_nt(const DecParams<MB>& P, int grid, cudaStream_t s) {
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, []() {
-    attr_err = cudaFuncSetAttribute(k_decode<NT, MB>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
+    attr_err = cudaFuncSetAttribute(k_decode<NT, MB, KW>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
   cudaLaunchConfig_t cfg = {};
@@ -612,7 +614,7 @@ cudaError_t launch_nt(const DecParams<MB>& P, int grid, cudaStream_t s) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_decode<NT, MB>, P);
+  return cudaLaunchKernelEx(&cfg, k_decode<NT, MB, KW>, P);
 }
 
 }  // namespace
@@ -626,7 +628,8 @@ gs_status decode_prepare(gs_packed* p, cudaStream_t s) {
   // each), of equal length.  Every split costs a partial write and a global
   // reduction, so a block only slightly above kUnitBytes stays whole instead
   // of leaving a one-chunk remainder unit.
-  const double per_chunk = p->kept > 0 ? 512.0 * (double)p->kept / ((double)p->G * (double)p->nblk64) : 512.0;
+  const double gbytes = 2.0 * (double)p->g_in;   // bytes of one kept group
+  const double per_chunk = p->kept > 0 ? gbytes * (double)p->kept / ((double)p->G * (double)p->nblk64) : gbytes;
   int nsplit = (int)std::floor(per_chunk * (double)p->G / (double)kUnitBytes + 0.5);
   nsplit = std::min(p->G, std::max(nsplit, std::max(1, (p->G + kMaxCpu - 1) / kMaxCpu)));
   const int cpu = (p->G + nsplit - 1) / nsplit;
@@ -714,6 +717,10 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
                         cudaStream_t s) {
   if (n <= 0 || T <= 0) return GS_OK;
   if (n > kMaxBatch || T > kMaxT) return GS_ERR_UNSUPPORTED;
+  const int kw = ps[0]->g_in;   // one chunk width per launch
+  for (int i = 1; i < n; ++i)
+    if (ps[i]->g_in != kw) return GS_ERR_UNSUPPORTED;
+  if (kw != 128 && kw != 256) return GS_ERR_UNSUPPORTED;
   // Unit list: layers in descending kept bytes.  Measured on the LLaMA-2-7B
   // block (per-module densities 0.3-0.7): every order that leaves the layer
   // whose blocks are split over several units (the down projection) at the end
@@ -748,7 +755,7 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     if (st != GS_OK) return st;
     if (order[k] == 0) first_slot = slot;
     L.x = static_cast<const uint16_t*>(xs[order[k]]);
-    if (!encode_tmap_slabs_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)T, (uint32_t)(kGroupIn / 64)))
+    if (!encode_tmap_slabs_bf16(&L.xmap, L.x, (uint64_t)p->in, (uint64_t)T, (uint32_t)T, (uint32_t)(kw / 64)))
       return GS_ERR_CUDA;
     L.tiles = p->tiles;
     L.dmeta = p->dmeta;
@@ -779,9 +786,11 @@ gs_status launch_decode(const gs_packed* const* ps, const void* const* xs, void*
     Q.sched = P.sched;
     Q.err = P.err;
     Q.inject_ns = P.inject_ns;
-    e = T <= 8 ? launch_nt<1>(Q, grid, s) : launch_nt<2>(Q, grid, s);
+    if (kw == 256) e = T <= 8 ? launch_nt<1, kSmallBatch, 256>(Q, grid, s) : launch_nt<2, kSmallBatch, 256>(Q, grid, s);
+    else e = T <= 8 ? launch_nt<1, kSmallBatch, 128>(Q, grid, s) : launch_nt<2, kSmallBatch, 128>(Q, grid, s);
   } else {
-    e = T <= 8 ? launch_nt<1>(P, grid, s) : launch_nt<2>(P, grid, s);
+    if (kw == 256) e = T <= 8 ? launch_nt<1, kMaxBatch, 256>(P, grid, s) : launch_nt<2, kMaxBatch, 256>(P, grid, s);
+    else e = T <= 8 ? launch_nt<1, kMaxBatch, 128>(P, grid, s) : launch_nt<2, kMaxBatch, 128>(P, grid, s);
   }
   note_launch();
   return e == cudaSuccess ? GS_OK : GS_ERR_CUDA;

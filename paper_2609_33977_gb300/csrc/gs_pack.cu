@@ -98,7 +98,9 @@ __device__ __forceinline__ uint4 ld_stream16(const void* p) {
 }
 
 // (a3) compact + copy: one warp per output row; every kept group of the row is
-// copied (512 B, 16 B per lane) to its packed slot and its row index recorded.
+// copied (KW bf16: 16 B per lane, KW / 8 lanes) to its packed slot and its row
+// index recorded.  KW = chunk width, 256 (1 x 256 groups) or 128 (1 x 128).
+template <int KW>
 __global__ void k_pack_compact(const uint16_t* __restrict__ W, int32_t out, int32_t in, int32_t G,
                                int32_t nw16, const int32_t* __restrict__ win_off16,
                                const uint16_t* __restrict__ kmask16, int32_t* __restrict__ row_idx,
@@ -139,11 +141,11 @@ __global__ void k_pack_compact(const uint16_t* __restrict__ W, int32_t out, int3
         uint4 v[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u)
-          if (u < n) v[u] = ld_stream16(W + r * in + (int64_t)cs[u] * kGroupIn + 8 * lane);
+          if (u < n && lane < KW / 8) v[u] = ld_stream16(W + r * in + (int64_t)cs[u] * KW + 8 * lane);
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           if (u < n) {
-            reinterpret_cast<uint4*>(tiles + (int64_t)ps[u] * kGroupIn)[lane] = v[u];
+            if (lane < KW / 8) reinterpret_cast<uint4*>(tiles + (int64_t)ps[u] * KW)[lane] = v[u];
             if (lane == 0) row_idx[ps[u]] = (int32_t)r;
           }
         }
@@ -154,6 +156,7 @@ __global__ void k_pack_compact(const uint16_t* __restrict__ W, int32_t out, int3
 
 // (a7) unpack: one warp per output row; kept groups copied back from their
 // packed slot, pruned groups written as +0.0.
+template <int KW>
 __global__ void k_unpack(const uint16_t* __restrict__ tiles, int32_t out, int32_t in, int32_t G,
                          int32_t nw16, const int32_t* __restrict__ win_off16,
                          const uint16_t* __restrict__ kmask16, uint16_t* __restrict__ W_hat) {
@@ -176,8 +179,10 @@ __global__ void k_unpack(const uint16_t* __restrict__ tiles, int32_t out, int32_
       for (int u = 0; u < nc; ++u) {
         const int32_t pu = __shfl_sync(0xffffffffu, pos, u);
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if ((kb >> u) & 1u) v = ld_stream16(tiles + (int64_t)pu * kGroupIn + 8 * lane);
-        reinterpret_cast<uint4*>(W_hat + r * in + (int64_t)(cb + u) * kGroupIn)[lane] = v;
+        if (lane < KW / 8) {
+          if ((kb >> u) & 1u) v = ld_stream16(tiles + (int64_t)pu * KW + 8 * lane);
+          reinterpret_cast<uint4*>(W_hat + r * in + (int64_t)(cb + u) * KW)[lane] = v;
+        }
       }
     }
   }
@@ -209,16 +214,17 @@ gs_status launch_scan_counts(const int32_t* cnt, int32_t G, int32_t nw, int32_t*
 
 gs_status launch_pack_compact(const void* W, gs_packed* p, cudaStream_t s) {
   if (p->kept == 0) return GS_OK;
-  k_pack_compact<<<grid_for(p->out, 8), 256, 0, s>>>(static_cast<const uint16_t*>(W), (int32_t)p->out,
-                                                     (int32_t)p->in, p->G, p->nw16, p->win_off16, p->kmask16,
-                                                     p->row_idx, p->tiles);
+  auto kern = p->g_in == 128 ? k_pack_compact<128> : k_pack_compact<256>;
+  kern<<<grid_for(p->out, 8), 256, 0, s>>>(static_cast<const uint16_t*>(W), (int32_t)p->out, (int32_t)p->in, p->G,
+                                           p->nw16, p->win_off16, p->kmask16, p->row_idx, p->tiles);
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }
 
 gs_status launch_unpack(const gs_packed* p, void* W_hat, cudaStream_t s) {
-  k_unpack<<<grid_for(p->out, 8), 256, 0, s>>>(p->tiles, (int32_t)p->out, (int32_t)p->in, p->G, p->nw16,
-                                               p->win_off16, p->kmask16, static_cast<uint16_t*>(W_hat));
+  auto kern = p->g_in == 128 ? k_unpack<128> : k_unpack<256>;
+  kern<<<grid_for(p->out, 8), 256, 0, s>>>(p->tiles, (int32_t)p->out, (int32_t)p->in, p->G, p->nw16, p->win_off16,
+                                           p->kmask16, static_cast<uint16_t*>(W_hat));
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }

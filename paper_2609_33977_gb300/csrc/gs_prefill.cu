@@ -60,7 +60,6 @@ constexpr int kNMax = kFW;                    // kept rows per MMA item: a whole
 constexpr int kNMaps = kNMax / 16;            // W descriptors, box heights 8, 16, ..., 80 (half a slice each)
 constexpr int kBK = 64;                       // k per slab: one 128-byte swizzle row
 constexpr int kSlabs = 2;                     // slabs per pipeline stage (a stage carries 128 k)
-constexpr int kKSteps = kGroupIn / (kBK * kSlabs);   // 2 stages per 256-wide chunk
 constexpr int kStages = 4;
 constexpr int kXSlabBytes = kBM * kBK * 2;    // 16 KB
 constexpr int kXStageBytes = kSlabs * kXSlabBytes;
@@ -213,8 +212,11 @@ __device__ __forceinline__ void gather_rows(const uint32_t* tbl, uint32_t* v) {
   }
 }
 
-template <bool kPair>
+// KW = chunk width: 256 (1 x 256 groups, two stages per chunk) or 128 (1 x 128 groups, one stage)
+template <bool kPair, int KW>
 __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__ PrefillParams P) {
+  constexpr int kKSteps = KW / (kBK * kSlabs);
+  static_assert(KW == 128 || KW == 256, "chunk width");
   constexpr int kStg = kPair ? kStages : kStagesSingle;
   constexpr int kStgBytes = kPair ? kStageBytes : kStageBytesSingle;
   extern __shared__ uint8_t smem_raw[];
@@ -319,11 +321,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
               if (rank == 0)
                 mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(2 * kXStageBytes + nr * kSlabs * kBK * 2));
               const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
-              tma_load_3d_pair(sx, &L.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+              tma_load_3d_pair(sx, &L.xmap, fb, 0, m * kPairM + (int)rank * kBM, c * (KW / kBK) + ks * kSlabs);
               tma_load_3d_pair(sx + kXStageBytes, wm, fb, 0, start + (int)rank * hn, ks * kSlabs);
             } else {
               mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(kXStageBytes + nr * kSlabs * kBK * 2));
-              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kBM, c * (kGroupIn / kBK) + ks * kSlabs);
+              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kBM, c * (KW / kBK) + ks * kSlabs);
               tma_load_3d(sx + kXStageBytes, wm, &full_bar[stage], 0, start, ks * kSlabs);
             }
             armed |= 1u << stage;
@@ -576,10 +578,10 @@ gs_status prefill_prepare_weight_maps(gs_packed* p) {
   static_assert(sizeof(p->wmaps) / sizeof(p->wmaps[0]) == kNMaps, "one W descriptor per slice height");
   for (int h = 0; h < kNMaps; ++h) {
     CUtensorMap m;
-    if (!encode_tmap_slabs_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, (uint32_t)(8 * (h + 1)), kSlabs))
+    if (!encode_tmap_slabs_bf16(&m, p->tiles, (uint64_t)p->g_in, (uint64_t)p->kept, (uint32_t)(8 * (h + 1)), kSlabs))
       return GS_ERR_CUDA;
     std::memcpy(p->wmaps[h], &m, sizeof(m));
-    if (!encode_tmap_slabs_bf16(&m, p->tiles, kGroupIn, (uint64_t)p->kept, (uint32_t)(16 * (h + 1)), kSlabs))
+    if (!encode_tmap_slabs_bf16(&m, p->tiles, (uint64_t)p->g_in, (uint64_t)p->kept, (uint32_t)(16 * (h + 1)), kSlabs))
       return GS_ERR_CUDA;
     std::memcpy(p->wmaps_full[h], &m, sizeof(m));
   }
@@ -595,11 +597,21 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, []() {
-    attr_err = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    attr_err = cudaFuncSetAttribute(k_prefill<true, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesSingle);
+      attr_err = cudaFuncSetAttribute(k_prefill<false, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      kSmemBytesSingle);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(k_prefill<true, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(k_prefill<false, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      kSmemBytesSingle);
   });
   if (attr_err != cudaSuccess) return GS_ERR_CUDA;
+  const int kw = ps[0]->g_in;   // one chunk width per launch
+  for (int i = 1; i < n; ++i)
+    if (ps[i]->g_in != kw) return GS_ERR_UNSUPPORTED;
+  if (kw != 128 && kw != 256) return GS_ERR_UNSUPPORTED;
   // Up to 128 tokens a pair tile (256 tokens) would be half empty: each CTA
   // then takes a 128-token tile of its own.
   const bool pair = T > kBM;
@@ -669,11 +681,12 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      e = cudaLaunchKernelEx(&cfg, k_prefill<true>, P);
+      e = kw == 256 ? cudaLaunchKernelEx(&cfg, k_prefill<true, 256>, P) : cudaLaunchKernelEx(&cfg, k_prefill<true, 128>, P);
     } else {
       const int64_t max_ctas = sm_count();
       const int grid = (int)(tiles < max_ctas ? tiles : max_ctas);
-      k_prefill<false><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
+      if (kw == 256) k_prefill<false, 256><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
+      else k_prefill<false, 128><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
       e = cudaGetLastError();
     }
     note_launch();

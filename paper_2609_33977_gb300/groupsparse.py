@@ -132,7 +132,7 @@ class Packed:
         nw16 = (self.out + 15) // 16
         offsets = np.zeros(G + 1, np.int64)
         row_idx = np.zeros(max(K, 1), np.int32)
-        tiles = np.zeros((max(K, 1), 256), np.uint16)
+        tiles = np.zeros((max(K, 1), self.g_in), np.uint16)
         win = np.zeros((G, nw16 + 1), np.int32)
         km = np.zeros((G, nw16), np.uint16)
         _check(lib.gs_packed_export(self.handle, offsets.ctypes.data_as(_c_i64p), row_idx.ctypes.data_as(_c_i32p),
@@ -170,7 +170,7 @@ def pack(W: torch.Tensor, mask: torch.Tensor, stream: Optional[torch.cuda.Stream
 def pack_groups(W: torch.Tensor, mask: torch.Tensor, g_out: int, g_in: int,
                 stream: Optional[torch.cuda.Stream] = None) -> Packed:
     """Pack a bf16 weight [out, in] with a group mask [out/g_out, in/g_in] (nonzero = keep)
-    for g_out x g_in groups: (1, 256) or square g x g, g in {16, 32, 64, 128}."""
+    for g_out x g_in groups: (1, 256), (1, 128) or square g x g, g in {16, 32, 64, 128}."""
     _require_cuda(W, torch.bfloat16, "W")
     if mask.dtype == torch.bool:
         mask = mask.to(torch.uint8)

@@ -146,3 +146,85 @@ def test_deterministic_and_group_shape_reported(gs):
     go, gi = ctypes.c_int32(), ctypes.c_int32()
     assert gs.lib.gs_packed_group_shape(p.handle, ctypes.byref(go), ctypes.byref(gi)) == 0
     assert (go.value, gi.value) == (64, 64)
+
+
+# --------------------------------------------------------------------- 1 x 128 groups
+
+def window_metadata(B):
+    """Per (chunk, 16-row window): first packed row and kept-row bitmask, derived
+    from the mask by counting (the layout's definition with 128-wide chunks)."""
+    out, G = B.shape
+    nw = (out + 15) // 16
+    win = np.zeros((G, nw + 1), np.int64)
+    km = np.zeros((G, nw), np.int64)
+    pos = 0
+    for c in range(G):
+        for w in range(nw):
+            win[c, w] = pos
+            for i in range(16):
+                r = 16 * w + i
+                if r < out and B[r, c]:
+                    km[c, w] |= 1 << i
+                    pos += 1
+        win[c, nw] = pos
+    return win, km
+
+
+@pytest.mark.parametrize("out,inp,d,seed", [(1, 128, 1.0, 1), (17, 384, 0.5, 2), (300, 768, 0.5, 3),
+                                            (4096, 4096, 0.5, 4), (11008, 4096, 0.45, 5), (4096, 11008, 0.5, 6),
+                                            (512, 3584, 0.3, 7), (129, 256, 0.0, 8)])
+def test_narrow_rows_pack_and_unpack(gs, out, inp, d, seed):
+    import torch
+    Wb = wl.random_weight_bits(out, inp, seed=seed)
+    B = wl.random_mask(out, inp // 128, d, seed=seed + 900)
+    p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), 1, 128)
+    ref = orc.pack_groups(Wb, B, 1, 128)
+    got = p.export()
+    assert np.array_equal(got["offsets"], ref.offsets)
+    assert np.array_equal(got["row_idx"], ref.block_row)
+    assert np.array_equal(got["tiles"], ref.tiles.reshape(-1, 128))
+    win, km = window_metadata(B)
+    assert np.array_equal(got["win_off16"], win) and np.array_equal(got["kmask16"], km)
+    Wh = to_bits(gs.unpack(p))
+    assert np.array_equal(Wh, orc.unpack_groups(ref))
+
+
+@pytest.mark.parametrize("T", [1, 5, 16, 17, 33, 64, 128, 129, 300, 2048])
+def test_narrow_rows_linear(gs, T):
+    import torch
+    for out, inp, d, seed in [(300, 768, 0.5, 11), (4096, 4096, 0.5, 12), (4096, 11008, 0.5, 13),
+                              (512, 3584, 0.3, 14)]:
+        Wb = wl.random_weight_bits(out, inp, seed=seed)
+        B = wl.random_mask(out, inp // 128, d, seed=seed + 900)
+        p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), 1, 128)
+        xb = wl.random_activation_bits(T, inp, seed=T + seed)
+        x = to_dev(xb)
+        toks = None if T <= 300 else sample_tokens(T, seed)
+        for algo in ((gs.ALGO_DECODE, gs.ALGO_PREFILL) if T <= 300 else (gs.ALGO_PREFILL,)):
+            y = to_bits(gs.linear(x, p, algo=algo))
+            if toks is None:
+                yr, A = orc.linear(xb, Wb, B, 1, 128)
+                yg = bf16_to_f64(y)
+            else:
+                yr, A = orc.linear_tokens(xb, Wb, B, toks, 1, 128)
+                yg = bf16_to_f64(y[np.asarray(toks)])
+            assert np.all(np.abs(yg - yr) <= REL * A + ABS), (out, inp, T, algo)
+
+
+def test_narrow_rows_batched_with_other_shapes(gs):
+    import torch
+    shapes = [(1, 128), (1, 256), (32, 32), (1, 128)]
+    layers = []
+    for i, (go, gi) in enumerate(shapes):
+        Wb = wl.random_weight_bits(1024, 2048, seed=80 + i)
+        B = wl.random_mask(1024 // go, 2048 // gi, 0.5, seed=90 + i)
+        p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), go, gi)
+        layers.append((Wb, B, p, go, gi))
+    for T in (3, 16, 200):
+        xbs = [wl.random_activation_bits(T, 2048, seed=100 + i + T) for i in range(len(layers))]
+        ys = [torch.empty((T, 1024), dtype=torch.bfloat16, device="cuda") for _ in layers]
+        gs.linear_batched_into([to_dev(b) for b in xbs], [l[2] for l in layers], ys)
+        for (Wb, B, p, go, gi), xb, y in zip(layers, xbs, ys):
+            yr, A = orc.linear(xb, Wb, B, go, gi)
+            assert np.all(np.abs(bf16_to_f64(to_bits(y)) - yr) <= REL * A + ABS), (go, gi, T)
+    assert gs.device_status() == gs.GS_OK
