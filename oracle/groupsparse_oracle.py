@@ -25,6 +25,11 @@ float64 without rounding).  Each function follows one definition:
   selector logit l keeps its group when sigmoid(l) > 1/2; App. F applies the
   same rule when the masks are exported, then reports each projection's
   preserved rate (active / total weights), the Q/K/V rates averaged.
+* training-side selectors, Sec. 2.2: a Gumbel-Sigmoid sample (logistic noise
+  passed in, temperature tau) gives binary selectors for the forward pass and
+  a relaxation whose derivative the straight-through estimator uses in the
+  backward pass; the backward of y = x W_hat^T gives the selector-logit and
+  input gradients.
 
 Readings where the paper is silent (all listed in the design notes):
 * groups are 1 x 256 along the input dimension, aligned at multiples of 256;
@@ -46,7 +51,10 @@ cell-by-cell one-hot orientation, brute force over every 16x16 mask of a
 masks, and the 1x256 layout identity; for token subsets: a hand-derived golden
 case whose token list is out of order and repeats a row, and int64 loops per
 listed token; for the kept count: hand-written masks with keep bytes other
-than 1, and the exact per-layer budget of the seeded generator).
+than 1, and the exact per-layer budget of the seeded generator; for the
+Gumbel-Sigmoid sample: hand-derived decisions and relaxation values, and
+agreement with a library sigmoid; for the straight-through backward: central
+finite differences of the relaxed forward loss, and exact integer cases).
 """
 from __future__ import annotations
 
@@ -360,3 +368,59 @@ def linear_packed_groups(x_bits: np.ndarray, p: PackedGroups) -> np.ndarray:
             u = int(p.block_row[j])
             y[:, p.g_out * u: p.g_out * (u + 1)] += xv @ tiles[j].T
     return y
+
+
+# ---------------------------------------------------------------------------
+# Sec. 2.2: Gumbel-Sigmoid relaxation with a straight-through estimator (the
+# training-side masked linear).  The paper names the relaxation (temperature
+# T = 0.4 in Table 7) and the estimator without printing formulas; the
+# standard form is used.  A sample draws two independent standard Gumbel
+# variables per selector; their difference L is a standard logistic variable,
+# passed in as `noise`.
+#   forward:  B = [sigmoid((l + L) / tau) > 1/2] = [l + L > 0]  (binary, used
+#             in W_hat = W (.) (B (x) 1) as in Eq. 1)
+#   backward: dB/dl is replaced by d sigmoid((l + L) / tau) / dl
+#             = s (1 - s) / tau with s = sigmoid((l + L) / tau)
+# ---------------------------------------------------------------------------
+
+def gumbel_select(logits: np.ndarray, noise: np.ndarray, tau: float) -> Tuple[np.ndarray, np.ndarray]:
+    """Binary selectors and their relaxation for one Gumbel-Sigmoid sample.
+
+    l + L is formed in float32 (the sum both the oracle and the kernel decide
+    on); B = [l + L > 0] (NaN prunes); s = sigmoid((l + L) / tau) in float64.
+    Returns (B uint8, s float64), both of the logits' shape."""
+    if not tau > 0:
+        raise ValueError("tau must be positive")
+    z32 = np.asarray(logits, dtype=np.float32) + np.asarray(noise, dtype=np.float32)
+    B = (z32.astype(np.float64) > 0.0).astype(np.uint8)
+    z = z32.astype(np.float64) / float(tau)
+    with np.errstate(over="ignore"):
+        s = 1.0 / (1.0 + np.exp(-z))
+    return B, s
+
+
+def group_weight_grad(x_bits: np.ndarray, W_bits: np.ndarray, dy: np.ndarray, g_out: int = 1,
+                      g_in: int = G_IN) -> np.ndarray:
+    """dL/dB for every group (kept or pruned): with y = x W_hat^T, dL/dW_hat = dy^T x,
+    and W_hat = W (.) (B (x) 1) gives dL/dB[u, v] = sum over the group's cells of
+    W[r, k] (dy^T x)[r, k].  dy: float [T, out]."""
+    x = _bf16_to_f64(x_bits)
+    W = _bf16_to_f64(W_bits)
+    dWhat = np.asarray(dy, dtype=np.float64).T @ x
+    P = W * dWhat
+    out, inp = W.shape
+    Go, Gi = group_grid(out, inp, g_out, g_in)
+    return P.reshape(Go, g_out, Gi, g_in).sum(axis=(1, 3))
+
+
+def masked_linear_backward(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray, dy: np.ndarray,
+                           soft: np.ndarray, tau: float, g_out: int = 1,
+                           g_in: int = G_IN) -> Tuple[np.ndarray, np.ndarray]:
+    """Straight-through backward of y = x W_hat^T: the selector-logit gradient
+    dL/dl = dL/dB * s (1 - s) / tau and the input gradient dL/dx = dy W_hat
+    (W is frozen, so there is no weight gradient).  Returns (dlogits, dx)."""
+    G = group_weight_grad(x_bits, W_bits, dy, g_out, g_in)
+    s = np.asarray(soft, dtype=np.float64)
+    dlogits = G * s * (1.0 - s) / float(tau)
+    dx = np.asarray(dy, dtype=np.float64) @ masked_weight(W_bits, B, g_out, g_in)
+    return dlogits, dx

@@ -497,3 +497,98 @@ def test_kept_groups_matches_the_allocated_budget():
         assert orc.kept_groups(B) == int(ks[i])
         total += orc.kept_groups(B)
     assert total == int(ks[0] + ks[4] + ks[6])
+
+
+# --------------------------------------------------------------------- Gumbel-Sigmoid + straight-through (Sec. 2.2)
+
+def test_golden_gumbel_select():
+    g = json.loads((GOLDEN / "gumbel_select.json").read_text())
+    B, s = orc.gumbel_select(np.asarray(g["logits"], np.float32), np.asarray(g["noise"], np.float32), g["tau"])
+    e = g["expected"]
+    assert B.tolist() == e["mask"]
+    for i, v in enumerate(e["sum"]):
+        if v == 0.0:
+            assert s[i] == e["soft_at_zero"]
+    for case in g["ln3_cases"]:
+        tau = abs(case["logit"] + case["noise"]) / math.log(3.0)
+        Bc, sc = orc.gumbel_select(np.float32([case["logit"]]), np.float32([case["noise"]]), tau)
+        assert int(Bc[0]) == case["mask"]
+        assert sc[0] == pytest.approx(case["soft"], abs=1e-15)
+
+
+@pytest.mark.parametrize("tau", [0.4, 1.0, 2.5])
+def test_gumbel_select_matches_library_sigmoid_and_threshold(tau):
+    from scipy.special import expit
+    rng = np.random.default_rng(5)
+    lg = rng.standard_normal(4000).astype(np.float32)
+    u = rng.random(4000)
+    noise = (np.log(u) - np.log1p(-u)).astype(np.float32)     # logistic = difference of two Gumbels
+    B, s = orc.gumbel_select(lg, noise, tau)
+    z = (lg + noise).astype(np.float64)
+    assert np.allclose(s, expit(z / tau), rtol=1e-14, atol=0)
+    assert np.array_equal(B, (z > 0).astype(np.uint8))
+    assert np.array_equal(B, (s > 0.5).astype(np.uint8))      # the threshold the paper describes
+    # without noise the sample is the evaluation-time export
+    assert np.array_equal(orc.gumbel_select(lg, np.zeros_like(lg), tau)[0], orc.select_groups(lg))
+
+
+def _relaxed_loss(x, W, lg, noise, tau, dy, g_in):
+    """sum(dy * y) with y = x (W (.) (s kron 1))^T, s = sigmoid((l + L)/tau): the
+    relaxed forward the straight-through backward differentiates (numpy, fp64)."""
+    s = 1.0 / (1.0 + np.exp(-(lg + noise) / tau))
+    M = np.repeat(s, g_in, axis=1)
+    return float(np.sum(dy * (x @ (W * M).T)))
+
+
+def test_straight_through_backward_against_finite_differences():
+    rng = np.random.default_rng(21)
+    out, inp, T, tau = 3, 512, 4, 0.4
+    xi = rng.integers(-3, 4, size=(T, inp))
+    Wi = rng.integers(-3, 4, size=(out, inp))
+    xb, Wb = bits_of(xi.astype(np.float32)), bits_of(Wi.astype(np.float32))
+    lg = (rng.integers(-8, 9, size=(out, inp // 256)) / 8.0).astype(np.float32)
+    noise = (rng.integers(-8, 9, size=lg.shape) / 8.0).astype(np.float32)
+    dy = rng.standard_normal((T, out))
+    B, s = orc.gumbel_select(lg, noise, tau)
+    dl, dx = orc.masked_linear_backward(xb, Wb, B, dy, s, tau)
+    x, W = xi.astype(np.float64), Wi.astype(np.float64)
+    h = 1e-6
+    for r in range(out):
+        for c in range(inp // 256):
+            lp, lm = lg.astype(np.float64), lg.astype(np.float64)
+            lp = lp.copy()
+            lm = lm.copy()
+            lp[r, c] += h
+            lm[r, c] -= h
+            fd = (_relaxed_loss(x, W, lp, noise.astype(np.float64), tau, dy, 256)
+                  - _relaxed_loss(x, W, lm, noise.astype(np.float64), tau, dy, 256)) / (2 * h)
+            assert dl[r, c] == pytest.approx(fd, rel=1e-6, abs=1e-6), (r, c)
+    # the input gradient uses the binary mask of the forward pass: exact in integers
+    Mi = np.repeat(B.astype(np.int64), 256, axis=1)
+    dyi = rng.integers(-3, 4, size=(T, out))
+    _, dx_int = orc.masked_linear_backward(xb, Wb, B, dyi.astype(np.float64), s, tau)
+    assert np.array_equal(dx_int, (dyi @ (Wi * Mi)).astype(np.float64))
+
+
+def test_group_weight_grad_exact_and_oriented():
+    # dL/dB[r, c] = sum_k W[r, 256c+k] sum_t dy[t, r] x[t, 256c+k], checked by int64 loops
+    rng = np.random.default_rng(22)
+    out, inp, T = 5, 768, 3
+    xi = rng.integers(-4, 5, size=(T, inp))
+    Wi = rng.integers(-4, 5, size=(out, inp))
+    dyi = rng.integers(-4, 5, size=(T, out))
+    G = orc.group_weight_grad(bits_of(xi.astype(np.float32)), bits_of(Wi.astype(np.float32)), dyi.astype(np.float64))
+    assert G.shape == (out, inp // 256)
+    for r in range(out):
+        for c in range(inp // 256):
+            ref = 0
+            for k in range(256 * c, 256 * c + 256):
+                ref += int(Wi[r, k]) * int(sum(int(dyi[t, r]) * int(xi[t, k]) for t in range(T)))
+            assert G[r, c] == float(ref)
+    # square groups: the 16x16 group sums reduce the same cell products
+    Gs = orc.group_weight_grad(bits_of(xi[:, :256].astype(np.float32)),
+                               bits_of(np.tile(Wi[:1, :256], (16, 1)).astype(np.float32)),
+                               np.tile(dyi[:, :1], (1, 16)).astype(np.float64), 16, 16)
+    assert Gs.shape == (1, 16)
+    cell = np.tile(Wi[:1, :256], (16, 1)) * (np.tile(dyi[:, :1], (1, 16)).T @ xi[:, :256])
+    assert np.array_equal(Gs, cell.reshape(1, 16, 16, 16).sum(axis=(1, 3)).astype(np.float64))
