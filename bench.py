@@ -785,8 +785,9 @@ def measure_block_7b(gs, torch, dev, stream, pool, hbm_peak, copies: int = 4):
     return {"workload": "llama2-7b block (7 projections), one batched launch per T", "per_T": rows}
 
 
-def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak, shapes=(16, 32, 64, 128)):
-    """The other group shapes (square g x g; Sec. 3.5 ablation, App. E) on the
+def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak,
+                         shapes=((1, 128), (16, 16), (32, 32), (64, 64), (128, 128))):
+    """The other group shapes (1x128 and square g x g; Sec. 3.5 ablation, App. E) on the
     LLaMA-2-7B block's seven projections, each keeping the same fraction of its
     groups as under the second configuration's 1x256 allocation (50 % overall):
     prefill at T = 2048 (one batched call per pass, kept TFLOP/s against the
@@ -796,18 +797,19 @@ def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak, shapes=(16
     ks = wl.keep_counts(w)
     n = len(w.layers)
     rows = []
-    for g in shapes:
-        masks = [pool.submit(wl.group_mask_shaped, w, i, int(ks[i]), g, g) for i in range(n)]
+    for go, gi in shapes:
+        masks = [pool.submit(wl.group_mask_shaped, w, i, int(ks[i]), go, gi) for i in range(n)]
         copies = [[], []]
         for i in range(n):
             W = wl.weight_device(w, i, device=dev)
             M = torch.from_numpy(masks[i].result()).to(dev)
             for c in range(2):
-                copies[c].append(gs.pack_groups(W, M, g, g))
+                copies[c].append(gs.pack_groups(W, M, go, gi))
             del W, M
         kept_tiles = sum(p.kept for p in copies[0])
-        kept_w = kept_tiles * g * g
-        row = {"group": f"{g}x{g}", "kept_weights": kept_w, "kept_fraction": kept_w / sum(L.out * L.inp for L in w.layers)}
+        kept_w = kept_tiles * go * gi
+        row = {"group": f"{go}x{gi}", "kept_weights": kept_w,
+               "kept_fraction": kept_w / sum(L.out * L.inp for L in w.layers)}
         for T in (1, 16, 2048):
             xs, ys = stack_inputs(torch, w, dev, T)
 
@@ -816,7 +818,9 @@ def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak, shapes=(16
             if T <= 16:
                 gr = [capture(torch, stream, lambda c=c: run(c)) for c in range(2)]
                 s = time_replays(torch, stream, gr, reps=100)
-                nb = 2.0 * kept_w + sum(4.0 * p.kept + 2.0 * T * (L.inp + L.out) for p, L in zip(copies[0], w.layers))
+                meta = (lambda p, L: 6.0 * (L.inp // gi) * ((L.out + 15) // 16)) if go == 1 else \
+                    (lambda p, L: 4.0 * p.kept)
+                nb = 2.0 * kept_w + sum(meta(p, L) + 2.0 * T * (L.inp + L.out) for p, L in zip(copies[0], w.layers))
                 row[f"decode_T{T}"] = {"us_per_block": s * 1e6, "GB/s": nb / s / 1e9,
                                        "frac_of_measured_hbm": nb / s / 1e9 / hbm_peak}
             else:

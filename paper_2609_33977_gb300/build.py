@@ -98,7 +98,7 @@ def build_library(force: bool = False, verbose: bool = False, extra_flags=None) 
     tmp = LIB.with_suffix(".so.tmp")
     libdir = _cuda_lib_dir(nvcc)
     cmd = [nvcc, "-shared", *ARCH, "-o", str(tmp), *map(str, objs), "-cudart", "shared",
-           f"-L{libdir}", "-Xlinker", f"-rpath,{libdir}"]
+           f"-L{libdir}", "-lcublas", "-Xlinker", f"-rpath,{libdir}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")

@@ -135,4 +135,11 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
 void sq_release(gs_packed* p);
 inline bool is_square(const gs_packed* p) { return p->g_out > 1; }
 
+// train.cu: Gumbel-Sigmoid sample and straight-through backward (Sec. 2.2)
+gs_status launch_gumbel(const float* logits, const float* noise, int64_t n, float tau, uint8_t* mask, float* soft,
+                        int64_t* kept, cudaStream_t s);
+size_t backward_workspace_bytes(const gs_packed* p, bool want_dx);
+gs_status launch_backward(const void* x, const void* W, const gs_packed* p, const void* dy, int64_t T,
+                          const float* soft, float tau, float* dlogits, void* dx, void* ws, cudaStream_t s);
+
 }  // namespace gs
