@@ -380,7 +380,10 @@ def linear_packed_groups(x_bits: np.ndarray, p: PackedGroups) -> np.ndarray:
 #   forward:  B = [sigmoid((l + L) / tau) > 1/2] = [l + L > 0]  (binary, used
 #             in W_hat = W (.) (B (x) 1) as in Eq. 1)
 #   backward: dB/dl is replaced by d sigmoid((l + L) / tau) / dl
-#             = s (1 - s) / tau with s = sigmoid((l + L) / tau)
+#             = s (1 - s) / tau with s = sigmoid((l + L) / tau); since
+#             1 - sigmoid(a) = sigmoid(-a), it is evaluated as
+#             sigmoid(a) sigmoid(-a) / tau, a = (l + L) / tau, which has no
+#             cancellation where s is near 0 or 1
 # ---------------------------------------------------------------------------
 
 def gumbel_select(logits: np.ndarray, noise: np.ndarray, tau: float) -> Tuple[np.ndarray, np.ndarray]:
@@ -399,6 +402,18 @@ def gumbel_select(logits: np.ndarray, noise: np.ndarray, tau: float) -> Tuple[np
     return B, s
 
 
+def gumbel_dsdl(logits: np.ndarray, noise: np.ndarray, tau: float) -> np.ndarray:
+    """The straight-through derivative ds/dl = sigmoid(a) sigmoid(-a) / tau,
+    a = (l + L) / tau, with l + L formed in float32 as in `gumbel_select`;
+    float64 of the logits' shape."""
+    if not tau > 0:
+        raise ValueError("tau must be positive")
+    z32 = np.asarray(logits, dtype=np.float32) + np.asarray(noise, dtype=np.float32)
+    a = z32.astype(np.float64) / float(tau)
+    with np.errstate(over="ignore"):
+        return (1.0 / (1.0 + np.exp(-a))) * (1.0 / (1.0 + np.exp(a))) / float(tau)
+
+
 def group_weight_grad(x_bits: np.ndarray, W_bits: np.ndarray, dy: np.ndarray, g_out: int = 1,
                       g_in: int = G_IN) -> np.ndarray:
     """dL/dB for every group (kept or pruned): with y = x W_hat^T, dL/dW_hat = dy^T x,
@@ -414,13 +429,13 @@ def group_weight_grad(x_bits: np.ndarray, W_bits: np.ndarray, dy: np.ndarray, g_
 
 
 def masked_linear_backward(x_bits: np.ndarray, W_bits: np.ndarray, B: np.ndarray, dy: np.ndarray,
-                           soft: np.ndarray, tau: float, g_out: int = 1,
+                           dsdl: np.ndarray, g_out: int = 1,
                            g_in: int = G_IN) -> Tuple[np.ndarray, np.ndarray]:
     """Straight-through backward of y = x W_hat^T: the selector-logit gradient
-    dL/dl = dL/dB * s (1 - s) / tau and the input gradient dL/dx = dy W_hat
-    (W is frozen, so there is no weight gradient).  Returns (dlogits, dx)."""
+    dL/dl = dL/dB * ds/dl (ds/dl from `gumbel_dsdl`) and the input gradient
+    dL/dx = dy W_hat (W is frozen, so there is no weight gradient).
+    Returns (dlogits, dx)."""
     G = group_weight_grad(x_bits, W_bits, dy, g_out, g_in)
-    s = np.asarray(soft, dtype=np.float64)
-    dlogits = G * s * (1.0 - s) / float(tau)
+    dlogits = G * np.asarray(dsdl, dtype=np.float64)
     dx = np.asarray(dy, dtype=np.float64) @ masked_weight(W_bits, B, g_out, g_in)
     return dlogits, dx

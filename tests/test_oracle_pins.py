@@ -550,7 +550,7 @@ def test_straight_through_backward_against_finite_differences():
     noise = (rng.integers(-8, 9, size=lg.shape) / 8.0).astype(np.float32)
     dy = rng.standard_normal((T, out))
     B, s = orc.gumbel_select(lg, noise, tau)
-    dl, dx = orc.masked_linear_backward(xb, Wb, B, dy, s, tau)
+    dl, dx = orc.masked_linear_backward(xb, Wb, B, dy, orc.gumbel_dsdl(lg, noise, tau))
     x, W = xi.astype(np.float64), Wi.astype(np.float64)
     h = 1e-6
     for r in range(out):
@@ -566,7 +566,7 @@ def test_straight_through_backward_against_finite_differences():
     # the input gradient uses the binary mask of the forward pass: exact in integers
     Mi = np.repeat(B.astype(np.int64), 256, axis=1)
     dyi = rng.integers(-3, 4, size=(T, out))
-    _, dx_int = orc.masked_linear_backward(xb, Wb, B, dyi.astype(np.float64), s, tau)
+    _, dx_int = orc.masked_linear_backward(xb, Wb, B, dyi.astype(np.float64), orc.gumbel_dsdl(lg, noise, tau))
     assert np.array_equal(dx_int, (dyi @ (Wi * Mi)).astype(np.float64))
 
 
@@ -592,3 +592,26 @@ def test_group_weight_grad_exact_and_oriented():
     assert Gs.shape == (1, 16)
     cell = np.tile(Wi[:1, :256], (16, 1)) * (np.tile(dyi[:, :1], (1, 16)).T @ xi[:, :256])
     assert np.array_equal(Gs, cell.reshape(1, 16, 16, 16).sum(axis=(1, 3)).astype(np.float64))
+
+
+@pytest.mark.parametrize("tau", [0.4, 1.0, 3.0])
+def test_gumbel_dsdl_is_the_sigmoid_derivative(tau):
+    from scipy.special import expit
+    rng = np.random.default_rng(31)
+    lg = (rng.standard_normal(2000) * 4).astype(np.float32)
+    noise = rng.standard_normal(2000).astype(np.float32)
+    d = orc.gumbel_dsdl(lg, noise, tau)
+    z = (lg + noise).astype(np.float64)
+    # central finite difference of sigmoid(z / tau) in z
+    h = 1e-5
+    fd = (expit((z + h) / tau) - expit((z - h) / tau)) / (2 * h)
+    assert np.allclose(d, fd, rtol=1e-6, atol=1e-12)
+    # closed forms: 1 / (4 tau) at z = 0, symmetric in z, and s (1 - s) / tau where that has no cancellation
+    assert orc.gumbel_dsdl(np.float32([0.0]), np.float32([0.0]), tau)[0] == 0.25 / tau
+    assert np.array_equal(d, orc.gumbel_dsdl(-lg, -noise, tau))
+    s = expit(z / tau)
+    mid = np.abs(z / tau) < 5
+    assert np.allclose(d[mid], (s * (1 - s) / tau)[mid], rtol=1e-12)
+    # far in the tails it keeps its relative precision (1 - s would have cancelled)
+    far = orc.gumbel_dsdl(np.float32([20.0]), np.float32([0.0]), 0.5)[0]
+    assert far == pytest.approx(math.exp(-40.0) / (1 + math.exp(-40.0)) ** 2 / 0.5, rel=1e-14)
