@@ -602,9 +602,11 @@ def test_gumbel_dsdl_is_the_sigmoid_derivative(tau):
     noise = rng.standard_normal(2000).astype(np.float32)
     d = orc.gumbel_dsdl(lg, noise, tau)
     z = (lg + noise).astype(np.float64)
-    # central finite difference of sigmoid(z / tau) in z
+    # central finite difference of sigmoid(z / tau) in z, taken on the lower
+    # tail (sigmoid(-a) for z > 0) where the two values do not cancel
     h = 1e-5
-    fd = (expit((z + h) / tau) - expit((z - h) / tau)) / (2 * h)
+    fd = np.where(z > 0, expit(-(z - h) / tau) - expit(-(z + h) / tau),
+                  expit((z + h) / tau) - expit((z - h) / tau)) / (2 * h)
     assert np.allclose(d, fd, rtol=1e-6, atol=1e-12)
     # closed forms: 1 / (4 tau) at z = 0, symmetric in z, and s (1 - s) / tau where that has no cancellation
     assert orc.gumbel_dsdl(np.float32([0.0]), np.float32([0.0]), tau)[0] == 0.25 / tau
