@@ -123,6 +123,11 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
       : "memory");
 }
 
+// bulk prefetch of [p, p + bytes) into L2 (bytes a multiple of 16)
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 // atomic add with acquire-release ordering at GPU scope; returns the old value
 __device__ __forceinline__ int atom_add_acq_rel_gpu(int32_t* p, int v) {
   int old;
@@ -295,6 +300,21 @@ __global__ void __launch_bounds__(kThreadsDec, 2) k_decode(const __grid_constant
 #pragma unroll
       for (int j = 0; j < kMaxCpu / 32; ++j)
         if (lane + 32 * j < U.nC) mrow[lane + 32 * j] = pre[j];
+      if (k == 0) {
+        // Before the grid-dependency wait the first unit's weight slices are
+        // also fetched into L2 (the ring takes only its first few chunks), so a
+        // CTA that starts while the previous grid is still finishing puts the
+        // idle HBM bandwidth of that grid's last units to use.
+        const uint16_t* tl = P.L[U.l].tiles;
+#pragma unroll
+        for (int j = 0; j < kMaxCpu / 32; ++j) {
+          if (lane + 32 * j < U.nC) {
+            const int4 mp = pre[j];
+            const uint32_t cnt = __popc((uint32_t)mp.y) + __popc((uint32_t)mp.z);
+            if (cnt) prefetch_l2_bulk(tl + (int64_t)mp.x * KW, cnt * (uint32_t)(2 * KW));
+          }
+        }
+      }
       if (lane == 0) unit_id[ms] = u;
       __threadfence_block();
       __syncwarp();
