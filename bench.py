@@ -540,6 +540,7 @@ def run_ours(args):
         extras["single_layer"] = measure_single_layer(gs, torch, dev, stream, hbm_peak)
         extras["block_7b"] = measure_block_7b(gs, torch, dev, stream, pool, hbm_peak)
         extras["group_shapes"] = measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak)
+        extras["train_op"] = measure_train_op(gs, torch, dev, stream, tpk, hbm_peak)
         try:
             extras["mask_export"] = measure_select(gs, torch, dev, stream, peaks)
         except Exception as e:   # reported in the line, never hidden
@@ -838,6 +839,57 @@ def measure_group_shapes(gs, torch, dev, stream, pool, tpk, hbm_peak,
                         "fractions", "shapes": rows}
 
 
+def measure_train_op(gs, torch, dev, stream, tpk, hbm_peak):
+    """The training-side op (Sec. 2.2): one Gumbel-Sigmoid sample over all selectors
+    of the 13B stack (logits + noise + ds/dl float32, mask uint8: 13 B per selector),
+    and the straight-through backward of one 13B down projection (5120 x 13824,
+    1x256 groups) at T = 2048 with and without the input gradient."""
+    w = wl.workload(4, 0.5)
+    n = w.total_groups
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    lg = torch.randn((n,), generator=g, device=dev)
+    u = torch.rand((n,), generator=g, device=dev).clamp_(1e-7, 1 - 1e-7)
+    noise = (torch.log(u) - torch.log1p(-u)).float()
+    s = time_calls(torch, stream, lambda: gs.gumbel_select(lg, noise, 0.4, stream=stream), reps=20, warm=3)
+    out = {"sample": {"selectors": n, "us_per_call": s * 1e6, "GB/s": 13.0 * n / s / 1e9,
+                      "frac_of_measured_hbm": 13.0 * n / s / 1e9 / hbm_peak}}
+    del lg, u, noise
+    o, i, T = 5120, 13824, 2048
+    W = (torch.randn((o, i), generator=g, device=dev) * 0.02).to(torch.bfloat16)
+    lgl = torch.randn((o, i // 256), generator=g, device=dev)
+    nz = torch.zeros_like(lgl)
+    mask, dsdl, _ = gs.gumbel_select(lgl, nz, 0.4)
+    p = gs.pack(W, mask)
+    x = torch.randn((T, i), generator=g, device=dev).to(torch.bfloat16)
+    dy = torch.randn((T, o), generator=g, device=dev).to(torch.bfloat16)
+    for want_dx in (False, True):
+        sb = time_calls(torch, stream, lambda: gs.masked_linear_backward(x, W, p, dy, dsdl, want_dx=want_dx,
+                                                                          stream=stream), reps=5, warm=2)
+        fl = 2.0 * T * o * i * (2 if want_dx else 1)
+        out["backward_dx" if want_dx else "backward"] = {"layer": f"{o}x{i}", "T": T, "ms": sb * 1e3,
+                                                         "dense_TFLOP/s": fl / sb / 1e12,
+                                                         "frac_of_burst_peak": fl / sb / 1e12 / tpk}
+    assert gs.device_status() == gs.GS_OK
+    del W, x, dy, p
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_train_op(args):
+    """The training-side op measurement alone; prints one JSON line."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_33977_gb300 import groupsparse as gs
+    peaks, _ = load_peaks()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device=dev)
+    print(json.dumps(measure_train_op(gs, torch, dev, stream, float(peaks.get("bf16_tflops", 1900.0)),
+                                      float(peaks.get("hbm_gbs", 6800.0)))), flush=True)
+    return 0
+
+
 def run_group_shapes(args):
     """The group-shape measurement alone; prints one JSON line."""
     import concurrent.futures as cf
@@ -993,6 +1045,8 @@ def main():
     ap.add_argument("--group", type=int, default=0, help="single-layer mode: square g x g groups (0 = 1x256)")
     ap.add_argument("--density", type=float, default=0.5)
     ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
+    ap.add_argument("--train-op", action="store_true",
+                    help="time only the Gumbel-Sigmoid sample and the straight-through backward")
     ap.add_argument("--group-shapes", action="store_true",
                     help="time only the square-group kernels on the 7B block")
     ap.add_argument("--mask-export", action="store_true",
@@ -1014,6 +1068,8 @@ def main():
         return run_mask_export(args)
     if args.group_shapes:
         return run_group_shapes(args)
+    if args.train_op:
+        return run_train_op(args)
     return run_ours(args)
 
 
