@@ -567,7 +567,9 @@ def run_ours(args):
                             f"(one per block per T)"},
         "roofline": {"kernel": "k_decode", "bound": "hbm", "achieved": achieved_gbs, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved_gbs / hbm_peak, "peak_source": f"{peaks_src} hbm_gbs",
-                     "bytes_per_step": bytes_per_step, "traffic": traffic,
+                     "bytes_per_step": bytes_per_step, "launches_per_step": launches_per_step,
+                     "algorithmic_bytes_per_launch": bytes_per_step / launches_per_step, "traffic": traffic,
+                     "traffic_source": "profiles/traffic.json: DRAM bytes of one block's launch (mean over T = 1, 16)",
                      "frac_of_8TBs_nominal": achieved_gbs / NOMINAL_HBM_GBS},
         "cpu_baseline": cpu,
         "e2e": e2e,

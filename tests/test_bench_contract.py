@@ -46,12 +46,14 @@ def test_bench_helpers():
     sys.path.insert(0, str(ROOT))
     import bench
     # the recorded DRAM traffic is reported only for the kernel source it was measured on
-    rec = json.loads((ROOT / "profiles" / "traffic.json").read_text())["k_decode"]["llama2-7b-block"]
-    got = bench.recorded_traffic("k_decode", "gs_decode.cu", "llama2-7b-block")
-    if rec["source_sha256_16"] == bench.kernel_source_hash("gs_decode.cu"):
-        assert got == rec["dram_bytes_per_launch"]
-    else:
-        assert got is None
+    recs = json.loads((ROOT / "profiles" / "traffic.json").read_text())["k_decode"]
+    for workload in ("llama2-7b-block", "llama2-13b-block"):
+        rec = recs[workload]
+        got = bench.recorded_traffic("k_decode", "gs_decode.cu", workload)
+        if rec["source_sha256_16"] == bench.kernel_source_hash("gs_decode.cu"):
+            assert got == rec["dram_bytes_per_launch"]
+        else:
+            assert got is None
     assert bench.recorded_traffic("k_decode", "gs_decode.cu", "no-such-workload") is None
     assert bench.recorded_traffic("no_such_kernel", "gs_decode.cu", "llama2-7b-block") is None
     # threads kept busy = process CPU time / wall time, at least one
