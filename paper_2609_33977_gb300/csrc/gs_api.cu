@@ -479,23 +479,23 @@ gs_status gs_preserved_rates(int32_t n, const int64_t* kept_host, const int64_t*
 }
 
 gs_status gs_gumbel_select(const float* logits_dev, const float* noise_dev, int64_t n, float tau, uint8_t* mask_dev,
-                           float* soft_dev, int64_t* kept_dev, void* stream) {
+                           float* dsdl_dev, int64_t* kept_dev, void* stream) {
   if (n < 0 || n >= (int64_t(1) << 36) || !(tau > 0.f) || !(tau < 3.0e38f)) return GS_ERR_INVALID_ARG;
   if (kept_dev && (reinterpret_cast<uintptr_t>(kept_dev) & 7u) != 0) return GS_ERR_INVALID_ARG;
   if (n > 0) {
     if (!logits_dev || !noise_dev || !mask_dev) return GS_ERR_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(logits_dev) & 3u) || (reinterpret_cast<uintptr_t>(noise_dev) & 3u) ||
-        (soft_dev && (reinterpret_cast<uintptr_t>(soft_dev) & 3u)))
+        (dsdl_dev && (reinterpret_cast<uintptr_t>(dsdl_dev) & 3u)))
       return GS_ERR_INVALID_ARG;
     // outputs must not overlap the inputs or each other
     const uintptr_t lo[4] = {reinterpret_cast<uintptr_t>(logits_dev), reinterpret_cast<uintptr_t>(noise_dev),
-                             reinterpret_cast<uintptr_t>(mask_dev), reinterpret_cast<uintptr_t>(soft_dev)};
-    const uintptr_t len[4] = {4 * (uintptr_t)n, 4 * (uintptr_t)n, (uintptr_t)n, soft_dev ? 4 * (uintptr_t)n : 0};
+                             reinterpret_cast<uintptr_t>(mask_dev), reinterpret_cast<uintptr_t>(dsdl_dev)};
+    const uintptr_t len[4] = {4 * (uintptr_t)n, 4 * (uintptr_t)n, (uintptr_t)n, dsdl_dev ? 4 * (uintptr_t)n : 0};
     for (int i = 2; i < 4; ++i)
       for (int j = 0; j < 4; ++j)
         if (i != j && len[i] && len[j] && lo[i] < lo[j] + len[j] && lo[j] < lo[i] + len[i]) return GS_ERR_INVALID_ARG;
   }
-  return launch_gumbel(logits_dev, noise_dev, n, tau, mask_dev, soft_dev, kept_dev, static_cast<cudaStream_t>(stream));
+  return launch_gumbel(logits_dev, noise_dev, n, tau, mask_dev, dsdl_dev, kept_dev, static_cast<cudaStream_t>(stream));
 }
 
 gs_status gs_masked_linear_backward_workspace(const gs_packed* p, int32_t want_dx, size_t* bytes) {
@@ -505,18 +505,18 @@ gs_status gs_masked_linear_backward_workspace(const gs_packed* p, int32_t want_d
 }
 
 gs_status gs_masked_linear_backward(const void* x_dev, const void* W_dev, const gs_packed* p, const void* dy_dev,
-                                    int64_t T, const float* soft_dev, float tau, float* dlogits_dev, void* dx_dev,
+                                    int64_t T, const float* dsdl_dev, float* dlogits_dev, void* dx_dev,
                                     void* workspace_dev, size_t workspace_bytes, void* stream) {
   if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
-  if (T <= 0 || T > INT32_MAX || !(tau > 0.f) || !(tau < 3.0e38f)) return GS_ERR_INVALID_ARG;
-  if (!x_dev || !W_dev || !dy_dev || !soft_dev || !dlogits_dev || !workspace_dev) return GS_ERR_INVALID_ARG;
+  if (T <= 0 || T > INT32_MAX) return GS_ERR_INVALID_ARG;
+  if (!x_dev || !W_dev || !dy_dev || !dsdl_dev || !dlogits_dev || !workspace_dev) return GS_ERR_INVALID_ARG;
   if (!aligned16(x_dev) || !aligned16(W_dev) || !aligned16(dy_dev) || !aligned16(workspace_dev) ||
-      (reinterpret_cast<uintptr_t>(soft_dev) & 3u) || (reinterpret_cast<uintptr_t>(dlogits_dev) & 3u) ||
+      (reinterpret_cast<uintptr_t>(dsdl_dev) & 3u) || (reinterpret_cast<uintptr_t>(dlogits_dev) & 3u) ||
       (dx_dev && !aligned16(dx_dev)))
     return GS_ERR_INVALID_ARG;
   if (p->out > INT32_MAX || p->in > INT32_MAX) return GS_ERR_UNSUPPORTED;
   if (workspace_bytes < backward_workspace_bytes(p, dx_dev != nullptr)) return GS_ERR_INVALID_ARG;
-  return launch_backward(x_dev, W_dev, p, dy_dev, T, soft_dev, tau, dlogits_dev, dx_dev, workspace_dev,
+  return launch_backward(x_dev, W_dev, p, dy_dev, T, dsdl_dev, dlogits_dev, dx_dev, workspace_dev,
                          static_cast<cudaStream_t>(stream));
 }
 

@@ -65,6 +65,7 @@ struct gs_packed {
   int32_t* gwoff;     // [G][nwin + 1]: first packed tile of column block v in window w (+ end)
   uint8_t* gwmask;    // [G][nwin]: bit i = block row (128/g) w + i kept in column block v
   alignas(64) unsigned char gmaps[8][128];   // W slice descriptors, box heights g, 2g, ..., 128 rows
+  alignas(64) unsigned char hmaps[8][128];   // CTA-pair halves: rows [r g/2, r g/2 + g/2) of 1..8 consecutive tiles
 };
 
 namespace gs {
@@ -76,6 +77,11 @@ bool encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t o
 // 2-D bf16 descriptor with a 32-, 64- or 128-byte swizzle (box_inner * 2 <= swizzle_bytes)
 bool encode_tmap_2d_bf16_swz(void* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
                              uint32_t box_outer, int swizzle_bytes);
+
+// rank-D bf16 descriptor (rank <= 5): dims innermost first, strides_bytes for
+// dims 1..rank-1, the given box and swizzle (box[0] * 2 <= swizzle_bytes)
+bool encode_tmap_nd_bf16(void* map, const void* base, int rank, const uint64_t* dims, const uint64_t* strides_bytes,
+                         const uint32_t* box, int swizzle_bytes);
 
 // 3-D "slab" bf16 descriptor over a row-major [rows][row_elems] matrix: a box
 // of box_rows rows x box_slabs 64-element slabs lands in shared memory as
@@ -136,10 +142,10 @@ void sq_release(gs_packed* p);
 inline bool is_square(const gs_packed* p) { return p->g_out > 1; }
 
 // train.cu: Gumbel-Sigmoid sample and straight-through backward (Sec. 2.2)
-gs_status launch_gumbel(const float* logits, const float* noise, int64_t n, float tau, uint8_t* mask, float* soft,
+gs_status launch_gumbel(const float* logits, const float* noise, int64_t n, float tau, uint8_t* mask, float* dsdl,
                         int64_t* kept, cudaStream_t s);
 size_t backward_workspace_bytes(const gs_packed* p, bool want_dx);
 gs_status launch_backward(const void* x, const void* W, const gs_packed* p, const void* dy, int64_t T,
-                          const float* soft, float tau, float* dlogits, void* dx, void* ws, cudaStream_t s);
+                          const float* dsdl, float* dlogits, void* dx, void* ws, cudaStream_t s);
 
 }  // namespace gs

@@ -24,6 +24,11 @@
 // For T < 128 the x boxes hold only T rows: the accumulator rows of the other
 // tokens then add up whatever the stage held before, and are never stored.
 //
+// Above 128 tokens a cluster of two CTAs owns a 256-token unit (one SM per 128
+// tokens, M = 256 MMAs issued by the leader, each CTA loading its own tokens'
+// x and one half of every tile's rows), which halves both the MMA instructions
+// and the W bytes each SM handles.
+//
 // Roles (one CTA per SM, persistent over units): warp 0 TMA producer, warp 1
 // TMEM allocator + single-thread MMA issuer, warps 2..5 epilogue (warp w reads
 // TMEM lanes 32 (w % 4) ..).  Two accumulator buffers let the epilogue of one
@@ -56,14 +61,17 @@ constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R 
 constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
 constexpr uint64_t kSqDrainLimitNs = 200000000ull;
 
-template <int G>
+template <int G, bool kPair>
 struct Sq {
   static constexpr int R = kSqWin / G;                  // block rows per window
   static constexpr int kSlabs = G > 64 ? 2 : 1;         // 64-column slabs per operand row
   static constexpr int kRowB = G >= 64 ? 128 : 2 * G;   // operand row bytes within a slab = swizzle width
-  static constexpr int kSlab = 128 * kRowB;             // one operand slab: 128 rows at the swizzle pitch
-  static constexpr int kRegion = kSlabs * kSlab;        // bytes per operand per stage
-  static constexpr int kStageBytes = 2 * kRegion;       // x box, then W slice
+  static constexpr int kSlab = 128 * kRowB;             // x slab: 128 token rows at the swizzle pitch
+  static constexpr int kRegion = kSlabs * kSlab;        // x bytes per stage
+  static constexpr int kWRows = kPair ? kSqWin / 2 : kSqWin;   // W rows a CTA holds per stage (pair: half of each tile)
+  static constexpr int kWSlab = kWRows * kRowB;
+  static constexpr int kWRegion = kSlabs * kWSlab;
+  static constexpr int kStageBytes = ((kRegion + kWRegion) + 1023) / 1024 * 1024;
   // as many stages as fit: a stage is one column block's copies, and the
   // copies of one stage wait for the MMAs of the stage before its last use,
   // so small groups need many stages in flight to cover the round trip
@@ -71,10 +79,11 @@ struct Sq {
   static constexpr uint32_t kSwz = G >= 64 ? 2u : (G == 32 ? 4u : 6u);   // UMMA layout: 128 / 64 / 32-byte swizzle
   static constexpr uint32_t kSBO = 8 * kRowB;           // bytes between 8-row core groups
   static constexpr int kKSteps = G / 16;
+  static constexpr int kTile = kPair ? 2 * kSqM : kSqM; // tokens per unit
   static constexpr int kSmem = kStages * kStageBytes + 2 * 32 * 8 + 1024;
   static_assert(R >= 1 && R <= kSqMaxMaps, "window holds 1..8 block rows");
   static_assert(kSmem <= 227 * 1024, "shared memory budget");
-  static_assert(kStageBytes % 1024 == 0, "stages keep 1024-byte alignment");
+  static_assert(kRegion % 1024 == 0, "the W region keeps 1024-byte alignment");
 };
 
 struct SqLayer {
@@ -135,9 +144,13 @@ __device__ __forceinline__ uint32_t sq_pack_bf16x2(float lo, float hi, bool keep
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-template <int G>
+// kPair: a cluster of two CTAs owns a 256-token unit; CTA r holds tokens
+// 128 r .. 128 r + 127 and rows [r g/2, r g/2 + g/2) of every tile, and the
+// leader's MMA thread issues M = 256 cta_group::2 MMAs whose accumulator lands
+// in both CTAs' TMEM.  Otherwise each CTA owns a 128-token unit.
+template <int G, bool kPair>
 __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ SqParams P) {
-  using C = Sq<G>;
+  using C = Sq<G, kPair>;
   extern __shared__ uint8_t sq_smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[C::kStages];
   __shared__ __align__(8) uint64_t empty_bar[C::kStages];
@@ -148,6 +161,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
   __shared__ int abort_s;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sq_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = kPair ? cluster_ctarank() : 0u;   // 0: leader (issues the pair's MMAs)
   uint2* ibuf = reinterpret_cast<uint2*>(smem + C::kStages * C::kStageBytes) + (warp < 2 ? warp : 0) * 32;
 
   if (threadIdx.x == 0) {
@@ -157,7 +171,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
     }
     for (int b = 0; b < kSqAccBufs; ++b) {
       mbar_init(&afull_bar[b], 1);
-      mbar_init(&aempty_bar[b], kSqEpiWarps);
+      mbar_init(&aempty_bar[b], (kPair ? 2 : 1) * kSqEpiWarps);   // the epilogue warps of the unit's CTAs
     }
     mbar_init(&drain_bar, 1);
     abort_s = 0;
@@ -168,25 +182,34 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
     }
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_s, kSqTmemCols);
-    tmem_relinquish();
+    if constexpr (kPair) {
+      tmem_alloc_pair(&tmem_base_s, kSqTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&tmem_base_s, kSqTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (kPair) cluster_sync_all();
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   volatile int* abort_flag = &abort_s;
   const int n_tiles = P.n_tiles;
+  const int owner = kPair ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;   // unit owners: CTA pairs or single CTAs
+  const int n_owners = kPair ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     uint32_t stage = 0, phase = 0;
     uint32_t armed = 0u, armed_par = 0u;
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int t = owner; t < n_tiles && ok; t += n_owners) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
+      const int tok0 = m * C::kTile + (int)rank * kSqM;
       for (int c0 = 0; c0 < L.Gin && ok; c0 += 32) {
         const int n_it = sq_items(L, w, c0, lane, ibuf);
         if (lane == 0) {
@@ -198,16 +221,33 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
               break;
             }
             uint8_t* sx = smem + stage * C::kStageBytes;
-            mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(P.x_rows * 2 * G) + (uint32_t)(n * G * 2 * G));
-            if constexpr (G > 64) {
-              // one box per 64-column slab, each into its own slab region (a two-slab
-              // box of fewer than 128 rows would pack the slabs back to back)
-              tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, m * kSqM, 2 * v);
-              tma_load_3d(sx + C::kSlab, &L.xmap, &full_bar[stage], 0, m * kSqM, 2 * v + 1);
-              tma_load_3d(sx + C::kRegion, &L.wmap[0], &full_bar[stage], 0, p0 * G, 0);
+            if constexpr (kPair) {
+              // both CTAs' copies complete on the leader's full barrier, which
+              // expects the bytes of both
+              if (rank == 0)
+                mbar_arrive_expect_tx(&full_bar[stage],
+                                      (uint32_t)(2 * P.x_rows * 2 * G) + (uint32_t)(n * G * 2 * G));
+              const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+              if constexpr (G > 64) {
+                tma_load_3d_pair(sx, &L.xmap, fb, 0, tok0, 2 * v);
+                tma_load_3d_pair(sx + C::kSlab, &L.xmap, fb, 0, tok0, 2 * v + 1);
+                tma_load_5d_pair(sx + C::kRegion, &L.wmap[0], fb, 0, 0, 0, (int)rank, p0);
+              } else {
+                tma_load_2d_pair(sx, &L.xmap, fb, v * G, tok0);
+                tma_load_4d_pair(sx + C::kRegion, &L.wmap[n - 1], fb, 0, 0, (int)rank, p0);
+              }
             } else {
-              tma_load_2d(sx, &L.xmap, &full_bar[stage], v * G, m * kSqM);
-              tma_load_2d(sx + C::kRegion, &L.wmap[n - 1], &full_bar[stage], 0, p0 * G);
+              mbar_arrive_expect_tx(&full_bar[stage], (uint32_t)(P.x_rows * 2 * G) + (uint32_t)(n * G * 2 * G));
+              if constexpr (G > 64) {
+                // one box per 64-column slab, each into its own slab region (a two-slab
+                // box of fewer than 128 rows would pack the slabs back to back)
+                tma_load_3d(sx, &L.xmap, &full_bar[stage], 0, tok0, 2 * v);
+                tma_load_3d(sx + C::kSlab, &L.xmap, &full_bar[stage], 0, tok0, 2 * v + 1);
+                tma_load_3d(sx + C::kRegion, &L.wmap[0], &full_bar[stage], 0, p0 * G, 0);
+              } else {
+                tma_load_2d(sx, &L.xmap, &full_bar[stage], v * G, tok0);
+                tma_load_2d(sx + C::kRegion, &L.wmap[n - 1], &full_bar[stage], 0, p0 * G);
+              }
             }
             armed |= 1u << stage;
             armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
@@ -220,7 +260,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       }
     }
-    if (lane == 0 && !ok) {
+    if (lane == 0 && !ok && rank == 0) {
       // let copies already in flight land before the CTA retires
       for (int s = 0; s < C::kStages; ++s) {
         if (!((armed >> s) & 1u)) continue;
@@ -230,19 +270,21 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
       }
     }
     __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 && rank == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader)
     uint32_t stage = 0, phase = 0;
     int buf = 0;
     uint32_t ae_ph = 0u;
     bool ok = true;
-    constexpr uint32_t idesc = idesc_bf16_f32(kSqM, G);
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    constexpr uint32_t idesc = idesc_bf16_f32(kPair ? 2 * kSqM : kSqM, G);
+    constexpr int kTileRows = kPair ? G / 2 : G;   // rows of each tile this CTA holds
+    for (int t = owner; t < n_tiles && ok; t += n_owners) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int w = (t - L.tile_begin) / L.n_m;
       if (lane == 0) {
-        ok = mbar_wait_bounded(&aempty_bar[buf], ((ae_ph >> buf) & 1u) ^ 1u, abort_flag, P.err, kSqWaitLimitNs,
-                               kDevErrTimeout);
+        const uint32_t par = ((ae_ph >> buf) & 1u) ^ 1u;
+        ok = kPair ? mbar_wait_bounded_cluster(&aempty_bar[buf], par, abort_flag, P.err, kSqWaitLimitNs, kDevErrTimeout)
+                   : mbar_wait_bounded(&aempty_bar[buf], par, abort_flag, P.err, kSqWaitLimitNs, kDevErrTimeout);
         ae_ph ^= 1u << buf;
         tc_fence_after();
       }
@@ -267,15 +309,20 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
               const uint32_t d = d0 + (uint32_t)(b * G);
 #pragma unroll
               for (int kk = 0; kk < C::kKSteps; ++kk) {
-                const uint32_t koff = (uint32_t)((kk >> 2) * C::kSlab + (kk & 3) * 32);
-                const uint64_t ad = sq_desc(sx + koff, C::kSBO, C::kSwz);
-                const uint64_t bd = sq_desc(sx + C::kRegion + (uint32_t)(i * G * C::kRowB) + koff, C::kSBO, C::kSwz);
-                mma_bf16_ss(d, ad, bd, idesc, (((seen >> b) & 1u) | (uint32_t)kk) != 0u ? 1u : 0u);
+                const uint32_t ka = (uint32_t)((kk >> 2) * C::kSlab + (kk & 3) * 32);
+                const uint32_t kb = (uint32_t)((kk >> 2) * C::kWSlab + (kk & 3) * 32);
+                const uint64_t ad = sq_desc(sx + ka, C::kSBO, C::kSwz);
+                const uint64_t bd =
+                    sq_desc(sx + C::kRegion + (uint32_t)(i * kTileRows * C::kRowB) + kb, C::kSBO, C::kSwz);
+                const uint32_t acc = (((seen >> b) & 1u) | (uint32_t)kk) != 0u ? 1u : 0u;
+                if constexpr (kPair) mma_bf16_ss_pair(d, ad, bd, idesc, acc);
+                else mma_bf16_ss(d, ad, bd, idesc, acc);
               }
               seen |= 1u << b;
               ++i;
             }
-            mma_commit(&empty_bar[stage]);
+            if constexpr (kPair) mma_commit_pair_mc(&empty_bar[stage], 0x3);
+            else mma_commit(&empty_bar[stage]);
             if (++stage == (uint32_t)C::kStages) {
               stage = 0;
               phase ^= 1u;
@@ -285,21 +332,26 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       }
       if (!ok) break;
-      if (lane == 0) mma_commit(&afull_bar[buf]);   // the unit's accumulator is complete once its MMAs are
+      // the unit's accumulator is complete once its MMAs are
+      if (lane == 0) {
+        if constexpr (kPair) mma_commit_pair_mc(&afull_bar[buf], 0x3);
+        else mma_commit(&afull_bar[buf]);
+      }
       buf ^= 1;
     }
     if (lane == 0) {
-      mma_commit(&drain_bar);
+      if constexpr (kPair) mma_commit_pair(&drain_bar);
+      else mma_commit(&drain_bar);
       mbar_wait_bounded(&drain_bar, 0u, nullptr, P.err, kSqWaitLimitNs, kDevErrTimeout);
     }
     __syncwarp();
-  } else {
+  } else if (warp >= 2) {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;   // TMEM lane quarter this warp may access
     int buf = 0;
     uint32_t af_ph = 0u;
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int t = owner; t < n_tiles && ok; t += n_owners) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -314,7 +366,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
       }
       af_ph ^= 1u << buf;
       tc_fence_after();
-      const int tok = m * kSqM + 32 * q + lane;
+      const int tok = m * C::kTile + (int)rank * kSqM + 32 * q + lane;
       uint16_t* yrow = L.y + (int64_t)tok * L.out;
 #pragma unroll 1
       for (int j = 0; j < kSqWin / 32; ++j) {
@@ -339,17 +391,29 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&aempty_bar[buf]);
+      if (lane == 0) {
+        if constexpr (kPair) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&aempty_bar[buf]), 0));
+        else mbar_arrive(&aempty_bar[buf]);
+      }
       buf ^= 1;
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  if (abort_s) {
+    // a role gave up: give copies the peer may still have in flight time to land
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 2000000ull) {
+    }
+  }
+  if constexpr (kPair) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kSqTmemCols);
+    if constexpr (kPair) tmem_dealloc_pair(tmem, kSqTmemCols);
+    else tmem_dealloc(tmem, kSqTmemCols);
   }
+  if constexpr (kPair) cluster_sync_all();
 }
 
 // ------------------------------------------------------------------ packing
@@ -442,41 +506,44 @@ int sq_sm_count() {
   return n;
 }
 
-template <int G>
+template <int G, bool kPair>
 cudaError_t sq_set_attr() {
   static std::once_flag once;
   static cudaError_t err = cudaSuccess;
   std::call_once(once, []() {
-    err = cudaFuncSetAttribute(k_sq<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sq<G>::kSmem);
+    err = cudaFuncSetAttribute(k_sq<G, kPair>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sq<G, kPair>::kSmem);
   });
   return err;
 }
 
-template <int G>
+// Above 128 tokens, CTA pairs own 256-token units; up to 128, single CTAs own
+// 128-token units (a pair unit would be half empty).
+template <int G, bool kPair>
 gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int* idx, int nb, int64_t T,
                     void* const* ys, int* err, cudaStream_t s) {
-  if (sq_set_attr<G>() != cudaSuccess) return GS_ERR_CUDA;
+  using C = Sq<G, kPair>;
+  if (sq_set_attr<G, kPair>() != cudaSuccess) return GS_ERR_CUDA;
   SqParams P;
   std::memset(&P, 0, sizeof(P));
   int64_t tiles = 0;
+  const uint32_t xr = (uint32_t)std::min<int64_t>(T, kSqM);
   for (int k = 0; k < nb; ++k) {
     const gs_packed* p = ps[idx[k]];
     SqLayer& L = P.L[k];
     bool ok;
-    const uint32_t xr = (uint32_t)std::min<int64_t>(T, kSqM);
     if (G > 64)
       ok = encode_tmap_slabs_bf16(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, xr, 1);
     else
-      ok = encode_tmap_2d_bf16_swz(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, G, xr, Sq<G>::kRowB);
+      ok = encode_tmap_2d_bf16_swz(&L.xmap, xs[idx[k]], (uint64_t)p->in, (uint64_t)T, G, xr, C::kRowB);
     if (!ok) return GS_ERR_CUDA;
-    for (int h = 0; h < Sq<G>::R; ++h) std::memcpy(&L.wmap[h], p->gmaps[h], sizeof(CUtensorMap));
+    for (int h = 0; h < C::R; ++h) std::memcpy(&L.wmap[h], kPair ? p->hmaps[h] : p->gmaps[h], sizeof(CUtensorMap));
     L.gwoff = p->gwoff;
     L.gwmask = p->gwmask;
     L.y = static_cast<uint16_t*>(ys[idx[k]]);
     L.out = (int32_t)p->out;
     L.Gin = p->G;
     L.nwin = p->nwin;
-    L.n_m = (int32_t)((T + kSqM - 1) / kSqM);
+    L.n_m = (int32_t)((T + C::kTile - 1) / C::kTile);
     L.tile_begin = (int32_t)tiles;
     tiles += (int64_t)L.n_m * L.nwin;
   }
@@ -484,12 +551,38 @@ gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int
   P.n_layers = nb;
   P.T = (int32_t)T;
   P.n_tiles = (int32_t)tiles;
-  P.x_rows = (int32_t)std::min<int64_t>(T, kSqM);
+  P.x_rows = (int32_t)xr;
   P.err = err;
-  const int grid = (int)std::min<int64_t>(tiles, sq_sm_count());
-  k_sq<G><<<grid, kSqThreads, Sq<G>::kSmem, s>>>(P);
+  cudaError_t e;
+  if constexpr (kPair) {
+    const int64_t pairs = std::min<int64_t>(tiles, sq_sm_count() / 2);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * pairs));
+    cfg.blockDim = dim3(kSqThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, k_sq<G, true>, P);
+  } else {
+    const int grid = (int)std::min<int64_t>(tiles, sq_sm_count());
+    k_sq<G, false><<<grid, kSqThreads, C::kSmem, s>>>(P);
+    e = cudaGetLastError();
+  }
   note_launch();
-  return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+  return e == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+}
+
+template <int G>
+gs_status sq_launch_any(const void* const* xs, const gs_packed* const* ps, const int* idx, int nb, int64_t T,
+                        void* const* ys, int* err, cudaStream_t s) {
+  return T > kSqM ? sq_launch<G, true>(xs, ps, idx, nb, T, ys, err, s)
+                  : sq_launch<G, false>(xs, ps, idx, nb, T, ys, err, s);
 }
 
 }  // namespace
@@ -550,6 +643,23 @@ gs_status sq_pack(const void* W, const uint8_t* mask, gs_packed* p, cudaStream_t
                                                        (uint32_t)((h + 1) * g), g >= 64 ? 128 : 2 * g);
       if (!ok) return GS_ERR_CUDA;
       std::memcpy(p->gmaps[h], &m, sizeof(m));
+      // CTA-pair halves: the tiles as [K][2 halves][g/2 rows][g] (g = 128: each row as
+      // two 64-wide slabs); a box takes one half of 1..8 consecutive tiles
+      const uint64_t gg = (uint64_t)g;
+      bool okh;
+      if (g > 64) {
+        const uint64_t dims[5] = {64, gg / 2, 2, 2, (uint64_t)kept};
+        const uint64_t str[4] = {2 * gg, 128, gg * gg, 2 * gg * gg};
+        const uint32_t box[5] = {64, (uint32_t)(g / 2), 2, 1, 1};
+        okh = encode_tmap_nd_bf16(&m, p->tiles, 5, dims, str, box, 128);
+      } else {
+        const uint64_t dims[4] = {gg, gg / 2, 2, (uint64_t)kept};
+        const uint64_t str[3] = {2 * gg, gg * gg, 2 * gg * gg};
+        const uint32_t box[4] = {(uint32_t)g, (uint32_t)(g / 2), 1, (uint32_t)(h + 1)};
+        okh = encode_tmap_nd_bf16(&m, p->tiles, 4, dims, str, box, g >= 64 ? 128 : 2 * g);
+      }
+      if (!okh) return GS_ERR_CUDA;
+      std::memcpy(p->hmaps[h], &m, sizeof(m));
     }
   }
   return GS_OK;
@@ -597,10 +707,10 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
       const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
       gs_status st;
       switch (gi) {
-        case 0: st = sq_launch<16>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
-        case 1: st = sq_launch<32>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
-        case 2: st = sq_launch<64>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
-        default: st = sq_launch<128>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        case 0: st = sq_launch_any<16>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        case 1: st = sq_launch_any<32>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        case 2: st = sq_launch_any<64>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
+        default: st = sq_launch_any<128>(xs, ps, o.data() + b0, nb, T, ys, err, s); break;
       }
       if (st != GS_OK) return st;
     }

@@ -4,10 +4,13 @@
 //
 //   sample:   z = l + L (L: logistic noise, the difference of two standard
 //             Gumbel draws, supplied by the caller), B = [z > 0] (the binary
-//             selectors of the forward pass), s = sigmoid(z / tau) (the
-//             relaxation the backward pass differentiates).
+//             selectors of the forward pass), and the derivative of the
+//             relaxation s = sigmoid(z / tau) that the backward pass uses,
+//             ds/dl = s (1 - s) / tau, written as t / (1 + t)^2 / tau with
+//             t = exp(-|z| / tau) so that it keeps its precision where s is
+//             near 0 or 1 (1 - s would cancel in float32).
 //   backward: dL/dW_hat = dy^T x, dL/dB[u, v] = sum over the group of
-//             W (.) dL/dW_hat, and the STE gives dL/dl = dL/dB s (1 - s) / tau;
+//             W (.) dL/dW_hat, and the STE gives dL/dl = dL/dB ds/dl;
 //             dL/dx = dy W_hat.
 //
 // The two products of the backward are plain dense GEMMs (dy^T x over all
@@ -27,25 +30,28 @@ constexpr int kGumbelThreads = 256;
 
 // one selector per thread (grid-stride); per-warp popcount, one 64-bit atomic per warp
 __global__ void k_gumbel(const float* __restrict__ logits, const float* __restrict__ noise, int64_t n, float tau,
-                         uint8_t* __restrict__ mask, float* __restrict__ soft, unsigned long long* __restrict__ kept) {
+                         uint8_t* __restrict__ mask, float* __restrict__ dsdl, unsigned long long* __restrict__ kept) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   unsigned int cnt = 0;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
     const float z = __fadd_rn(logits[i], noise[i]);
     const bool keep = z > 0.f;   // NaN prunes
     mask[i] = keep ? 1 : 0;
-    if (soft) soft[i] = 1.f / (1.f + expf(-__fdiv_rn(z, tau)));
+    if (dsdl) {
+      const float t = expf(-fabsf(__fdiv_rn(z, tau)));
+      const float d = 1.f + t;
+      dsdl[i] = __fdiv_rn(__fdiv_rn(t, d * d), tau);
+    }
     cnt += keep ? 1u : 0u;
   }
   const unsigned int w = __reduce_add_sync(0xffffffffu, cnt);
   if (kept && (threadIdx.x & 31) == 0 && w) atomicAdd(kept, (unsigned long long)w);
 }
 
-// dlogits[u, v] = s (1 - s) / tau * sum over group (u, v) of W (.) D, D = dy^T x
+// dlogits[u, v] = ds/dl[u, v] * sum over group (u, v) of W (.) D, D = dy^T x
 // (fp32 [out][in]); one warp per group, lanes over the group's cells four at a time
-__global__ void k_group_grad(const uint16_t* __restrict__ W, const float* __restrict__ D, const float* __restrict__ soft,
-                             int32_t out, int32_t in, int32_t g_out, int32_t g_in, float inv_tau,
-                             float* __restrict__ dlogits) {
+__global__ void k_group_grad(const uint16_t* __restrict__ W, const float* __restrict__ D, const float* __restrict__ dsdl,
+                             int32_t out, int32_t in, int32_t g_out, int32_t g_in, float* __restrict__ dlogits) {
   const int lane = threadIdx.x & 31;
   const int64_t Gin = in / g_in, n = (int64_t)(out / g_out) * Gin;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -65,10 +71,7 @@ __global__ void k_group_grad(const uint16_t* __restrict__ W, const float* __rest
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) {
-      const float s = soft[e];
-      dlogits[e] = acc * s * (1.f - s) * inv_tau;
-    }
+    if (lane == 0) dlogits[e] = acc * dsdl[e];
   }
 }
 
@@ -90,13 +93,13 @@ size_t round256(size_t b) { return (b + 255) & ~size_t(255); }
 
 }  // namespace
 
-gs_status launch_gumbel(const float* logits, const float* noise, int64_t n, float tau, uint8_t* mask, float* soft,
+gs_status launch_gumbel(const float* logits, const float* noise, int64_t n, float tau, uint8_t* mask, float* dsdl,
                         int64_t* kept, cudaStream_t s) {
   if (kept && cudaMemsetAsync(kept, 0, sizeof(int64_t), s) != cudaSuccess) return GS_ERR_CUDA;
   if (n == 0) return GS_OK;
   int64_t blocks = (n + kGumbelThreads - 1) / kGumbelThreads;
   if (blocks > 8 * 1024) blocks = 8 * 1024;
-  k_gumbel<<<(unsigned)blocks, kGumbelThreads, 0, s>>>(logits, noise, n, tau, mask, soft,
+  k_gumbel<<<(unsigned)blocks, kGumbelThreads, 0, s>>>(logits, noise, n, tau, mask, dsdl,
                                                        reinterpret_cast<unsigned long long*>(kept));
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
@@ -108,7 +111,7 @@ size_t backward_workspace_bytes(const gs_packed* p, bool want_dx) {
 }
 
 gs_status launch_backward(const void* x, const void* W, const gs_packed* p, const void* dy, int64_t T,
-                          const float* soft, float tau, float* dlogits, void* dx, void* ws, cudaStream_t s) {
+                          const float* dsdl, float* dlogits, void* dx, void* ws, cudaStream_t s) {
   const int64_t out = p->out, in = p->in;
   float* D = static_cast<float*>(ws);
   {
@@ -141,8 +144,8 @@ gs_status launch_backward(const void* x, const void* W, const gs_packed* p, cons
   const int64_t groups = (int64_t)(out / p->g_out) * (in / p->g_in);
   int64_t blocks = (groups + 7) / 8;
   if (blocks > (1 << 20)) blocks = 1 << 20;
-  k_group_grad<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const uint16_t*>(W), D, soft, (int32_t)out, (int32_t)in,
-                                                p->g_out, p->g_in, 1.f / tau, dlogits);
+  k_group_grad<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const uint16_t*>(W), D, dsdl, (int32_t)out, (int32_t)in,
+                                                p->g_out, p->g_in, dlogits);
   note_launch();
   return cudaGetLastError() == cudaSuccess ? GS_OK : GS_ERR_CUDA;
 }

@@ -50,8 +50,7 @@ def _load(path: Path = LIB_PATH) -> ctypes.CDLL:
     lib.gs_preserved_rates.argtypes = [i32, vp, vp, vp, i64, vp, vp, i32, vp, vp]
     lib.gs_gumbel_select.argtypes = [vp, vp, i64, ctypes.c_float, vp, vp, vp, vp]
     lib.gs_masked_linear_backward_workspace.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_size_t)]
-    lib.gs_masked_linear_backward.argtypes = [vp, vp, vp, vp, i64, vp, ctypes.c_float, vp, vp, vp, ctypes.c_size_t,
-                                              vp]
+    lib.gs_masked_linear_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, ctypes.c_size_t, vp]
     lib.gs_debug_fail_alloc.argtypes = [i64]
     lib.gs_debug_inject_wait.argtypes = [ctypes.c_int, ctypes.c_uint64]
     for fn in (lib.gs_pack, lib.gs_linear, lib.gs_linear_ex, lib.gs_linear_batched, lib.gs_unpack,
@@ -309,42 +308,42 @@ def preserved_report(kept: Sequence[int], shapes: Sequence[Sequence[int]],
 def gumbel_select(logits: torch.Tensor, noise: torch.Tensor, tau: float,
                   stream: Optional[torch.cuda.Stream] = None):
     """One Gumbel-Sigmoid sample of the selectors (Sec. 2.2): mask = [l + L > 0] (uint8),
-    soft = sigmoid((l + L) / tau) (float32) and the kept count (int64 [1]); L is the
-    caller's logistic noise, of the logits' shape."""
+    dsdl = d sigmoid((l + L) / tau) / dl (float32, the straight-through derivative) and the
+    kept count (int64 [1]); L is the caller's logistic noise, of the logits' shape."""
     _require_cuda(logits, torch.float32, "logits")
     _require_cuda(noise, torch.float32, "noise")
     if noise.shape != logits.shape:
         raise ValueError("noise must have the logits' shape")
     mask = torch.empty(logits.shape, dtype=torch.uint8, device=logits.device)
-    soft = torch.empty(logits.shape, dtype=torch.float32, device=logits.device)
+    dsdl = torch.empty(logits.shape, dtype=torch.float32, device=logits.device)
     kept = torch.empty((1,), dtype=torch.int64, device=logits.device)
     _check(lib.gs_gumbel_select(logits.data_ptr(), noise.data_ptr(), logits.numel(), float(tau), mask.data_ptr(),
-                                soft.data_ptr(), kept.data_ptr(), _stream_ptr(stream)), "gs_gumbel_select")
-    return mask, soft, kept
+                                dsdl.data_ptr(), kept.data_ptr(), _stream_ptr(stream)), "gs_gumbel_select")
+    return mask, dsdl, kept
 
 
-def masked_linear_backward(x: torch.Tensor, W: torch.Tensor, p: Packed, dy: torch.Tensor, soft: torch.Tensor,
-                           tau: float, want_dx: bool = True, stream: Optional[torch.cuda.Stream] = None):
+def masked_linear_backward(x: torch.Tensor, W: torch.Tensor, p: Packed, dy: torch.Tensor, dsdl: torch.Tensor,
+                           want_dx: bool = True, stream: Optional[torch.cuda.Stream] = None):
     """Straight-through backward of y = x W_hat^T (Sec. 2.2): (dlogits float32 of the
     mask's shape, dx bf16 [T, in] or None).  p is W packed with the sampled mask."""
     _require_cuda(x, torch.bfloat16, "x")
     _require_cuda(W, torch.bfloat16, "W")
     _require_cuda(dy, torch.bfloat16, "dy")
-    _require_cuda(soft, torch.float32, "soft")
+    _require_cuda(dsdl, torch.float32, "dsdl")
     T = x.shape[0]
     if tuple(W.shape) != (p.out, p.inp) or x.shape[1] != p.inp or tuple(dy.shape) != (T, p.out):
         raise ValueError("W must be [out, in], x [T, in] and dy [T, out]")
     shape = (p.out // p.g_out, p.inp // p.g_in)
-    if tuple(soft.shape) != shape:
-        raise ValueError(f"soft must be {shape}")
+    if tuple(dsdl.shape) != shape:
+        raise ValueError(f"dsdl must be {shape}")
     nbytes = ctypes.c_size_t()
     _check(lib.gs_masked_linear_backward_workspace(p.handle, 1 if want_dx else 0, ctypes.byref(nbytes)),
            "gs_masked_linear_backward_workspace")
     ws = torch.empty((nbytes.value,), dtype=torch.uint8, device=x.device)
     dl = torch.empty(shape, dtype=torch.float32, device=x.device)
     dx = torch.empty((T, p.inp), dtype=torch.bfloat16, device=x.device) if want_dx else None
-    _check(lib.gs_masked_linear_backward(x.data_ptr(), W.data_ptr(), p.handle, dy.data_ptr(), T, soft.data_ptr(),
-                                         float(tau), dl.data_ptr(), dx.data_ptr() if dx is not None else None,
+    _check(lib.gs_masked_linear_backward(x.data_ptr(), W.data_ptr(), p.handle, dy.data_ptr(), T, dsdl.data_ptr(),
+                                         dl.data_ptr(), dx.data_ptr() if dx is not None else None,
                                          ws.data_ptr(), nbytes.value, _stream_ptr(stream)),
            "gs_masked_linear_backward")
     return dl, dx
