@@ -295,23 +295,27 @@ gs_status gs_preserved_rates(int32_t n, const int64_t* kept_host, const int64_t*
  * Gumbel-Sigmoid relaxation with a straight-through estimator; the
  * temperature of Table 7 is 0.4).  The paper names the relaxation without
  * printing it; the standard form is used:
- *     z = l + L,   B = [z > 0] = [sigmoid(z / tau) > 1/2],   s = sigmoid(z / tau)
+ *     z = l + L,   B = [z > 0] = [sigmoid(z / tau) > 1/2],
+ *     ds/dl = s (1 - s) / tau  with  s = sigmoid(z / tau)
  * where L is standard logistic noise (the difference of two standard Gumbel
  * draws), which the caller draws.  B is the binary mask of the forward pass
- * (pack W with it: gs_pack / gs_pack_groups, then gs_linear); s is what the
- * backward pass (gs_masked_linear_backward) differentiates.  z is the float32
- * sum rounded to nearest; NaN prunes.
+ * (pack W with it: gs_pack / gs_pack_groups, then gs_linear); ds/dl is the
+ * derivative the straight-through estimator puts in place of dB/dl in the
+ * backward pass (gs_masked_linear_backward).  It is formed as
+ * t / (1 + t)^2 / tau with t = exp(-|z| / tau), which keeps its relative
+ * precision where s is near 0 or 1.  z is the float32 sum rounded to nearest;
+ * NaN prunes.
  *
  * logits_dev, noise_dev  float32 [n], device, 4-byte aligned, read only.
  * tau                    temperature, > 0 and finite.
  * mask_dev               uint8 [n], overwritten with 0 / 1.
- * soft_dev               float32 [n] or NULL, overwritten with s.
+ * dsdl_dev               float32 [n] or NULL, overwritten with ds/dl.
  * kept_dev               int64 or NULL, 8-byte aligned: the number of ones.
  * Outputs must not overlap the inputs or each other.  Asynchronous on stream.
  * Errors: INVALID_ARG, CUDA.
  */
 gs_status gs_gumbel_select(const float* logits_dev, const float* noise_dev, int64_t n, float tau, uint8_t* mask_dev,
-                           float* soft_dev, int64_t* kept_dev, void* stream);
+                           float* dsdl_dev, int64_t* kept_dev, void* stream);
 
 /*
  * gs_masked_linear_backward - the straight-through backward pass of the masked
@@ -319,7 +323,7 @@ gs_status gs_gumbel_select(const float* logits_dev, const float* noise_dev, int6
  * (Sec. 2.2; the pretrained weights are not updated):
  *     dL/dW_hat = dy^T x
  *     dL/dB[u][v] = sum over the cells (r, k) of group (u, v) of W[r][k] dL/dW_hat[r][k]
- *     dL/dl[u][v] = dL/dB[u][v] s (1 - s) / tau        (the estimator)
+ *     dL/dl[u][v] = dL/dB[u][v] ds/dl[u][v]             (the estimator)
  *     dL/dx = dy W_hat
  * Every group receives a logit gradient, pruned ones included.  The two
  * products are dense GEMMs done by cuBLAS (fp32 accumulation); the group
@@ -328,7 +332,7 @@ gs_status gs_gumbel_select(const float* logits_dev, const float* noise_dev, int6
  * x_dev       bf16 [T][in] (the forward input).      W_dev  bf16 [out][in] (dense, frozen).
  * p           handle of W packed with the sampled mask B (any supported group shape).
  * dy_dev      bf16 [T][out], the gradient of the loss with respect to y.
- * soft_dev    float32 [out/g_out][in/g_in]: s from gs_gumbel_select.
+ * dsdl_dev    float32 [out/g_out][in/g_in]: ds/dl from gs_gumbel_select.
  * dlogits_dev float32 [out/g_out][in/g_in], overwritten.
  * dx_dev      bf16 [T][in], overwritten, or NULL (no input gradient).
  * workspace   device scratch of gs_masked_linear_backward_workspace bytes
@@ -338,7 +342,7 @@ gs_status gs_gumbel_select(const float* logits_dev, const float* noise_dev, int6
  */
 gs_status gs_masked_linear_backward_workspace(const gs_packed* p, int32_t want_dx, size_t* bytes);
 gs_status gs_masked_linear_backward(const void* x_dev, const void* W_dev, const gs_packed* p, const void* dy_dev,
-                                    int64_t T, const float* soft_dev, float tau, float* dlogits_dev, void* dx_dev,
+                                    int64_t T, const float* dsdl_dev, float* dlogits_dev, void* dx_dev,
                                     void* workspace_dev, size_t workspace_bytes, void* stream);
 
 /*
