@@ -48,9 +48,12 @@ typedef enum gs_status {
 
 /* Kernel family for gs_linear_ex. */
 typedef enum gs_algo {
-  GS_ALGO_AUTO = 0,     /* pick by token count (decode for small T, else prefill)   */
+  GS_ALGO_AUTO = 0,     /* pick by token count and group shape                       */
   GS_ALGO_DECODE = 1,   /* CUDA-core/mma.sync streaming kernel (memory-bound)        */
-  GS_ALGO_PREFILL = 2   /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
+  GS_ALGO_PREFILL = 2,  /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
+  GS_ALGO_PREFILL_DENSE = 3  /* tcgen05 kernel over zero-filled 256-row windows: tensor
+                                work of the dense layer, no gather; 1 x 128 and 1 x 256
+                                groups; GS_ALGO_AUTO picks it for 1 x 128 at T >= 1024  */
 } gs_algo;
 
 typedef struct gs_packed gs_packed;   /* opaque, library-owned */

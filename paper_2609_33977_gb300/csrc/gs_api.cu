@@ -245,15 +245,22 @@ static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, v
                              gs_algo algo) {
   if (check_handle(p) != GS_OK) return GS_ERR_INVALID_ARG;
   if (T < 0 || T > INT32_MAX) return GS_ERR_INVALID_ARG;
-  if (algo != GS_ALGO_AUTO && algo != GS_ALGO_DECODE && algo != GS_ALGO_PREFILL) return GS_ERR_INVALID_ARG;
+  if (algo != GS_ALGO_AUTO && algo != GS_ALGO_DECODE && algo != GS_ALGO_PREFILL && algo != GS_ALGO_PREFILL_DENSE)
+    return GS_ERR_INVALID_ARG;
   if (T == 0) return GS_OK;
   if (!x_dev || !y_dev) return GS_ERR_INVALID_ARG;
   if (!aligned16(x_dev) || !aligned16(y_dev)) return GS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (is_square(p)) return sq_linear_batched(&x_dev, &p, 1, T, &y_dev, s);   // one kernel family for every T
-  if (algo == GS_ALGO_AUTO)
+  if (algo == GS_ALGO_AUTO) {
     algo = (T >= kPrefillMinTokens && p->G <= prefill_max_chunks()) ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
+    if (algo == GS_ALGO_PREFILL && prefill_prefers_dense(p, T)) algo = GS_ALGO_PREFILL_DENSE;
+  }
   if (algo == GS_ALGO_PREFILL) return launch_prefill(x_dev, p, T, y_dev, s);
+  if (algo == GS_ALGO_PREFILL_DENSE) {
+    if (p->kept == 0) return cudaMemsetAsync(y_dev, 0, (size_t)T * (size_t)p->out * 2, s) == cudaSuccess ? GS_OK : GS_ERR_CUDA;
+    return launch_prefill_dense(&x_dev, &p, 1, T, &y_dev, s);
+  }
   // decode family: token blocks of at most decode_max_tokens()
   const int64_t blk = decode_max_tokens();
   for (int64_t t0 = 0; t0 < T; t0 += blk) {
@@ -333,11 +340,16 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
   }
   if (T >= kPrefillMinTokens) {
     // layers the prefill kernel takes share batched launches; any other goes alone
-    std::vector<const void*> xp;
-    std::vector<const gs_packed*> pp;
-    std::vector<void*> yp;
+    // (layers the zero-filled kernel runs faster go there, batched the same way)
+    std::vector<const void*> xp, xd;
+    std::vector<const gs_packed*> pp, pd;
+    std::vector<void*> yp, yd;
     for (int i = 0; i < n; ++i) {
-      if (ps[i]->G <= prefill_max_chunks()) {
+      if (prefill_prefers_dense(ps[i], T)) {
+        xd.push_back(xs_dev[i]);
+        pd.push_back(ps[i]);
+        yd.push_back(ys_dev[i]);
+      } else if (ps[i]->G <= prefill_max_chunks()) {
         xp.push_back(xs_dev[i]);
         pp.push_back(ps[i]);
         yp.push_back(ys_dev[i]);
@@ -346,6 +358,11 @@ gs_status gs_linear_batched(int32_t n, const void* const* xs_dev, const gs_packe
         if (st != GS_OK) return st;
       }
     }
+    if (!pd.empty()) {
+      const gs_status st = launch_prefill_dense(xd.data(), pd.data(), (int)pd.size(), T, yd.data(), s);
+      if (st != GS_OK) return st;
+    }
+    if (pp.empty()) return GS_OK;
     return launch_prefill_batched(xp.data(), pp.data(), (int)pp.size(), T, yp.data(), s);
   }
   const int64_t blk = decode_max_tokens();

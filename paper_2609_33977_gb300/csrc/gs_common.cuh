@@ -131,6 +131,11 @@ gs_status launch_prefill(const void* x, const gs_packed* p, int64_t T, void* y, 
 gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T,
                                  void* const* ys, cudaStream_t s);
 int prefill_max_chunks();
+// prefill_dense.cu: zero-filled windows (1 x 128 / 1 x 256 layers with kept groups)
+gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
+                               cudaStream_t s);
+// whether the zero-filled kernel is the faster one for this layer and token count
+bool prefill_prefers_dense(const gs_packed* p, int64_t T);
 
 // groups.cu: square g x g groups
 bool sq_shape_supported(int g_out, int g_in);

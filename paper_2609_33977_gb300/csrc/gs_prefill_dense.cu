@@ -1,0 +1,530 @@
+// Prefill-regime group-sparse linear with zero-filled windows (1 x 256 and
+// 1 x 128 groups, Eq. 1), for layers whose kept fraction is high enough that
+// multiplying the pruned rows by zero costs less than gathering the kept ones.
+//
+// A unit of work is 256 tokens x a window of 256 output rows, owned by a
+// cluster of two CTAs: CTA r holds tokens 128 r .. 128 r + 127 and window rows
+// 128 r .. 128 r + 127.  For every chunk with a kept row in the window and every
+// 64-wide k slab of it, the producer warps place the window's rows in shared
+// memory at their row positions (a 16-byte cp.async per piece from the packed
+// tiles for a kept row; zeros for a pruned row), next to one TMA box of the
+// tokens' x slab, and the leader issues M = 256, N = 256 cta_group::2 MMAs that
+// accumulate the whole unit in TMEM.  Nothing is gathered or scattered: the
+// accumulator is read once per unit.  Packed weights are read from memory once
+// per unit (pruned groups move no bytes); the tensor work is that of the dense
+// window, i.e. 1 / density times the kept work.
+//
+// Roles (one CTA per SM, units persistent over the pairs): warps 0..3
+// producers (warp-cooperative 16-byte cp.async of the window's rows, zero-filled
+// for pruned rows; warp 0 lane 0 also issues the x boxes), warp 4 TMEM
+// allocator + single-thread MMA issuer (leader), warps 5..8 epilogue, warp 9
+// forwarder.  Producers never wait for their own copies: each thread's copies
+// of a stage signal a local barrier (cp.async.mbarrier.arrive), and the
+// forwarder, once all have landed, fences them to the async proxy and arrives
+// on the leader's full barrier.  Every wait is bounded.
+#include "gs_common.cuh"
+#include "gs_sm100.cuh"
+
+#include <cuda.h>
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+namespace gs {
+namespace {
+using namespace sm100;
+
+constexpr int kDM = 128;                          // tokens per CTA (TMEM lanes); a pair covers 256
+constexpr int kDW = 256;                          // output rows per window (N of each MMA)
+constexpr int kDHalf = kDW / 2;                   // window rows each CTA holds
+constexpr int kDSlabK = 64;                       // k per stage (one 128-byte swizzle row)
+constexpr int kDXBytes = kDM * kDSlabK * 2;       // 16 KB of x per stage
+constexpr int kDWBytes = kDHalf * kDSlabK * 2;    // 16 KB of W rows per stage
+constexpr int kDStageBytes = kDXBytes + kDWBytes;
+constexpr int kDStages = 6;
+constexpr int kDProdWarps = 4;                   // warps that copy W rows
+constexpr int kDMmaWarp = kDProdWarps;
+constexpr int kDEpiWarp0 = kDProdWarps + 1;
+constexpr int kDEpiWarps = 4;
+constexpr int kDFwdWarp = kDEpiWarp0 + kDEpiWarps;
+constexpr int kDThreads = (kDFwdWarp + 1) * 32;
+constexpr int kDAccBufs = 2;
+constexpr uint32_t kDTmemCols = kDAccBufs * kDW;  // 512
+constexpr int kDMaxLayers = 8;
+constexpr uint64_t kDWaitLimitNs = 2000000000ull;
+constexpr uint64_t kDDrainLimitNs = 200000000ull;
+constexpr int kDIbufBytes = 1024;                // per-warp chunk lists of d_items
+constexpr int kDSmem = kDStages * kDStageBytes + kDIbufBytes + 1024;
+static_assert(kDHalf % (kDProdWarps * 32) == 0, "producer warps split the CTA's window rows evenly");
+static_assert(kDSmem <= 227 * 1024, "shared memory budget");
+static_assert(kDStageBytes % 1024 == 0 && kDXBytes % 1024 == 0, "stages keep 1024-byte alignment");
+
+struct DLayer {
+  CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 1
+  const uint16_t* tiles;     // [kept][KW]
+  const int32_t* win_off16;  // [G][nw16 + 1]
+  const uint16_t* kmask16;   // [G][nw16]
+  uint16_t* y;
+  int32_t out, G, nw16, n_m, tile_begin;
+};
+struct DParams {
+  DLayer L[kDMaxLayers];
+  int32_t n_layers, T, n_tiles;
+  int* err;
+};
+
+__device__ __forceinline__ int d_layer_of(const DParams& P, int t) {
+  int l = 0;
+  while (l + 1 < P.n_layers && P.L[l + 1].tile_begin <= t) ++l;
+  return l;
+}
+
+// 16-byte copy global -> shared; src_bytes < 16 fills the rest with zeros (0: reads nothing)
+__device__ __forceinline__ void cp_async16_zfill(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+// arrive on a local mbarrier once all of this thread's earlier cp.async copies have landed
+// (without raising its expected count: the barrier counts the arriving threads)
+__device__ __forceinline__ void cp_async_arrive_noinc(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+__device__ __forceinline__ void fence_acq_rel_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_cta() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Chunks c0 .. c0 + 31 with at least one kept row in window w, in order, into buf.
+__device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane, int* buf) {
+  const int c = c0 + lane;
+  __syncwarp();   // every lane is done reading the previous batch
+  bool ne = false;
+  if (c < L.G) {
+    const int32_t* wo = L.win_off16 + (int64_t)c * (L.nw16 + 1);
+    const int lo = w * (kDW / kWin16), hi = min(lo + kDW / kWin16, L.nw16);
+    ne = wo[hi] > wo[lo];
+  }
+  const uint32_t ballot = __ballot_sync(0xffffffffu, ne);
+  if (ne) buf[__popc(ballot & ((1u << lane) - 1u))] = c;
+  __syncwarp();
+  return __popc(ballot);
+}
+
+__device__ __forceinline__ uint32_t d_pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+template <int KW>
+__global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_constant__ DParams P) {
+  constexpr int kSlabs = KW / kDSlabK;   // stages per chunk
+  extern __shared__ uint8_t d_smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kDStages];
+  __shared__ __align__(8) uint64_t wfull_bar[kDStages];
+  __shared__ __align__(8) uint64_t empty_bar[kDStages];
+  __shared__ __align__(8) uint64_t afull_bar[kDAccBufs];
+  __shared__ __align__(8) uint64_t aempty_bar[kDAccBufs];
+  __shared__ __align__(8) uint64_t drain_bar;
+  __shared__ uint32_t tmem_base_s;
+  __shared__ int abort_s;
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(d_smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs)
+  int* ibuf = reinterpret_cast<int*>(smem + kDStages * kDStageBytes) +
+              (warp <= kDMmaWarp ? warp : (warp == kDFwdWarp ? kDMmaWarp + 1 : 0)) * 32;
+  static_assert((kDMmaWarp + 2) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDStages; ++s) {
+      mbar_init(&full_bar[s], 2 + 1);                  // both CTAs' forwarders + the x byte count
+      mbar_init(&wfull_bar[s], kDProdWarps * 32);       // this CTA's producer threads' copies
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int b = 0; b < kDAccBufs; ++b) {
+      mbar_init(&afull_bar[b], 1);
+      mbar_init(&aempty_bar[b], 2 * kDEpiWarps);
+    }
+    mbar_init(&drain_bar, 1);
+    abort_s = 0;
+    fence_mbar_init();
+    for (int l = 0; l < P.n_layers; ++l) prefetch_tmap(&P.L[l].xmap);
+  }
+  if (warp == kDMmaWarp) {
+    tmem_alloc_pair(&tmem_base_s, kDTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  volatile int* abort_flag = &abort_s;
+  const int n_tiles = P.n_tiles;
+  const int pair = (int)(blockIdx.x >> 1), n_pairs = (int)(gridDim.x >> 1);
+
+  if (warp < kDProdWarps) {
+    // ------------------------------------------------------------ producers
+    // Warp v copies window rows v * kRows .. + kRows - 1 of this CTA's half,
+    // warp-cooperatively: copy i moves rows v * kRows + 4 i .. + 3, eight
+    // lanes per 128-byte row, so each instruction reads four whole lines.
+    // Lane l looks up the packed positions of rows v * kRows + 32 q + l.
+    constexpr int kRows = kDHalf / kDProdWarps;   // rows per producer warp
+    constexpr int kOwn = kRows / 32;              // rows whose metadata a lane loads
+    constexpr int kCopies = kRows / 4;            // 16-byte copies per lane per stage
+    uint32_t stage = 0, phase = 0;
+    uint32_t armed = 0u, armed_par = 0u;
+    bool ok = true;
+    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+      const DLayer& L = P.L[d_layer_of(P, u)];
+      const int lt = u - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      const int tok0 = m * 2 * kDM + (int)rank * kDM;
+      // metadata of this lane's rows in chunk c: the window's kept mask and first
+      // packed row (two independent loads, issued one item ahead of their use)
+      auto load_meta = [&](int c, uint32_t (&km)[kOwn], int (&wo)[kOwn]) {
+#pragma unroll
+        for (int q = 0; q < kOwn; ++q) {
+          const int h = (int)rank * kDHalf + warp * kRows + 32 * q + lane;   // row within the window
+          const int b16 = min(w * (kDW / kWin16) + (h >> 4), L.nw16 - 1);
+          km[q] = L.kmask16[(int64_t)c * L.nw16 + b16];
+          wo[q] = L.win_off16[(int64_t)c * (L.nw16 + 1) + b16];
+        }
+      };
+      for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
+        const int n_it = d_items(L, w, c0, lane, ibuf);
+        uint32_t km_n[kOwn];
+        int wo_n[kOwn];
+        if (n_it > 0) load_meta(ibuf[0], km_n, wo_n);
+        for (int it = 0; it < n_it && ok; ++it) {
+          const int c = ibuf[it];
+          // packed positions in chunk c of the rows this lane looks up (-1: pruned / beyond out)
+          int prow[kOwn];
+#pragma unroll
+          for (int q = 0; q < kOwn; ++q) {
+            const int h = (int)rank * kDHalf + warp * kRows + 32 * q + lane;
+            const int b16 = w * (kDW / kWin16) + (h >> 4), bit = h & 15;
+            const bool kept = b16 < L.nw16 && ((km_n[q] >> bit) & 1u);
+            prow[q] = kept ? wo_n[q] + __popc(km_n[q] & ((1u << bit) - 1u)) : -1;
+          }
+          if (it + 1 < n_it) load_meta(ibuf[it + 1], km_n, wo_n);
+          // the rows this lane copies: warp * kRows + 4 i + (lane >> 3)
+          int crow[kCopies];
+#pragma unroll
+          for (int i = 0; i < kCopies; ++i) {
+            const int r = 4 * i + (lane >> 3);   // row within the warp's block: owner lane r % 32, slot r / 32
+            crow[i] = __shfl_sync(0xffffffffu, prow[r >> 5], r & 31);
+          }
+          const int j = lane & 7;   // 16-byte piece of the row
+#pragma unroll 1
+          for (int sl = 0; sl < kSlabs && ok; ++sl) {
+            bool got = true;
+            if (lane == 0)
+              got = mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
+            if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
+              ok = false;
+              break;
+            }
+            uint8_t* sx = smem + stage * kDStageBytes;
+            if (warp == 0 && lane == 0) {
+              if (rank == 0) mbar_arrive_expect_tx(&full_bar[stage], 2u * kDXBytes);
+              tma_load_3d_pair(sx, &L.xmap, mapa_shared(smem_u32(&full_bar[stage]), 0), 0, tok0,
+                               c * kSlabs + sl);
+              armed |= 1u << stage;
+              armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+            }
+            const uint32_t wb = smem_u32(sx + kDXBytes);
+#pragma unroll
+            for (int i = 0; i < kCopies; ++i) {
+              const int rr = warp * kRows + 4 * i + (lane >> 3);
+              const uint32_t dst = wb + (uint32_t)rr * 128u + (uint32_t)((j ^ (rr & 7)) << 4);   // 128-byte swizzle
+              const bool kept = crow[i] >= 0;
+              // a pruned row reads nothing (source size 0) and is filled with zeros
+              const uint16_t* src = kept ? L.tiles + (int64_t)crow[i] * KW + sl * kDSlabK + 8 * j : L.tiles;
+              cp_async16_zfill(dst, src, kept ? 16u : 0u);
+            }
+            cp_async_arrive_noinc(&wfull_bar[stage]);   // fires once this thread's copies have landed
+            if (++stage == (uint32_t)kDStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+    }
+    cp_async_wait_all();
+    if (warp == 0 && lane == 0 && !ok && rank == 0) {
+      for (int s = 0; s < kDStages; ++s) {
+        if (!((armed >> s) & 1u)) continue;
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait_acq_cluster(&full_bar[s], (armed_par >> s) & 1u))
+          if (globaltimer_ns() - t0 > kDDrainLimitNs) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kDFwdWarp) {
+    // ------------------------------------------------------------ forwarder
+    // Once all of this CTA's producer threads' copies of a stage have landed,
+    // make them visible to the tensor cores (async proxy) and tell the leader.
+    uint32_t stage = 0, phase = 0;
+    bool ok = true;
+    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+      const DLayer& L = P.L[d_layer_of(P, u)];
+      const int w = (u - L.tile_begin) / L.n_m;
+      for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
+        const int n_st = d_items(L, w, c0, lane, ibuf) * kSlabs;
+        if (lane == 0) {
+          for (int k = 0; k < n_st && ok;) {
+            if (!mbar_wait_bounded(&wfull_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
+              ok = false;
+              break;
+            }
+            // take every following stage that has landed too, so that one
+            // release fence covers them all (a release per stage is slow)
+            int cnt = 1;
+            while (k + cnt < n_st && cnt < kDStages) {
+              const uint32_t s2 = (stage + (uint32_t)cnt) % kDStages;
+              const uint32_t p2 = phase ^ ((stage + (uint32_t)cnt) >= (uint32_t)kDStages ? 1u : 0u);
+              if (!mbar_try_wait(&wfull_bar[s2], p2)) break;
+              ++cnt;
+            }
+            fence_proxy_async_cta();
+            fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
+            for (int i = 0; i < cnt; ++i) {
+              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage]), 0));
+              if (++stage == (uint32_t)kDStages) {
+                stage = 0;
+                phase ^= 1u;
+              }
+            }
+            k += cnt;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      }
+    }
+  } else if (warp == kDMmaWarp && rank == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    uint32_t stage = 0, phase = 0;
+    int buf = 0;
+    uint32_t ae_ph = 0u;
+    bool ok = true;
+    constexpr uint32_t idesc = idesc_bf16_f32(2 * kDM, kDW);
+    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+      const DLayer& L = P.L[d_layer_of(P, u)];
+      const int w = (u - L.tile_begin) / L.n_m;
+      if (lane == 0) {
+        ok = mbar_wait_bounded_cluster(&aempty_bar[buf], ((ae_ph >> buf) & 1u) ^ 1u, abort_flag, P.err, kDWaitLimitNs,
+                                       kDevErrTimeout);
+        ae_ph ^= 1u << buf;
+        tc_fence_after();
+      }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      const uint32_t d = tmem + (uint32_t)(buf * kDW);
+      bool first = true;
+      for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
+        const int n_it = d_items(L, w, c0, lane, ibuf);
+        if (lane == 0) {
+          for (int it = 0; it < n_it * kSlabs && ok; ++it) {
+            if (!mbar_wait_bounded_cluster(&full_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs,
+                                           kDevErrTimeout)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sx = smem_u32(smem + stage * kDStageBytes);
+            const uint64_t ad = sdesc_sw128(sx), bd = sdesc_sw128(sx + kDXBytes);
+#pragma unroll
+            for (int kk = 0; kk < kDSlabK / 16; ++kk)
+              mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
+                               (first && kk == 0) ? 0u : 1u);
+            first = false;
+            mma_commit_pair_mc(&empty_bar[stage], 0x3);
+            if (++stage == (uint32_t)kDStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        first = __shfl_sync(0xffffffffu, first ? 1 : 0, 0) != 0;
+      }
+      if (!ok) break;
+      if (lane == 0) mma_commit_pair_mc(&afull_bar[buf], 0x3);
+      buf ^= 1;
+    }
+    if (lane == 0) {
+      mma_commit_pair(&drain_bar);
+      mbar_wait_bounded(&drain_bar, 0u, nullptr, P.err, kDWaitLimitNs, kDevErrTimeout);
+    }
+    __syncwarp();
+  } else if (warp >= kDEpiWarp0) {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;   // TMEM lane quarter this warp may access
+    int buf = 0;
+    uint32_t af_ph = 0u;
+    bool ok = true;
+    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+      const DLayer& L = P.L[d_layer_of(P, u)];
+      const int lt = u - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      // a window with no kept row in any chunk has no MMA: its rows are zero
+      bool any = false;
+      {
+        const int lo = w * (kDW / kWin16), hi = min(lo + kDW / kWin16, L.nw16);
+        for (int c = lane; c < L.G && !any; c += 32) {
+          const int32_t* wo = L.win_off16 + (int64_t)c * (L.nw16 + 1);
+          any = wo[hi] > wo[lo];
+        }
+        any = __any_sync(0xffffffffu, any);
+      }
+      const bool got =
+          mbar_wait_bounded(&afull_bar[buf], (af_ph >> buf) & 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
+      if (!__all_sync(0xffffffffu, got)) {   // the TMEM loads below need the whole warp
+        ok = false;
+        break;
+      }
+      af_ph ^= 1u << buf;
+      tc_fence_after();
+      const int tok = m * 2 * kDM + (int)rank * kDM + 32 * q + lane;
+      uint16_t* yrow = L.y + (int64_t)tok * L.out;
+      const bool vec_ok = (L.out & 7) == 0;
+#pragma unroll 1
+      for (int j = 0; j < kDW / 32; ++j) {
+        uint32_t v[32];
+        tmem_ld_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kDW + 32 * j), v);
+        tmem_wait_ld();
+        reg_fence(v);
+        const int r0 = w * kDW + 32 * j;
+        if (tok < P.T) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int rb = r0 + 8 * k;
+            const float* f = reinterpret_cast<const float*>(v + 8 * k);
+            if (vec_ok && rb + 8 <= L.out) {
+              *reinterpret_cast<uint4*>(yrow + rb) =
+                  any ? make_uint4(d_pack_bf16x2(f[0], f[1]), d_pack_bf16x2(f[2], f[3]), d_pack_bf16x2(f[4], f[5]),
+                                   d_pack_bf16x2(f[6], f[7]))
+                      : make_uint4(0u, 0u, 0u, 0u);
+            } else {
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+                if (rb + e < L.out) yrow[rb + e] = any ? __bfloat16_as_ushort(__float2bfloat16_rn(f[e])) : 0;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&aempty_bar[buf]), 0));
+      buf ^= 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (abort_s) {
+    // a role gave up: give copies the peer may still have in flight time to land
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 2000000ull) {
+    }
+  }
+  cluster_sync_all();
+  if (warp == kDMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, kDTmemCols);
+  }
+  cluster_sync_all();
+}
+
+int d_sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int KW>
+cudaError_t d_set_attr() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, []() {
+    err = cudaFuncSetAttribute(k_prefill_dense<KW>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDSmem);
+  });
+  return err;
+}
+
+}  // namespace
+
+// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes): with
+// 1 x 128 groups this kernel takes 0.76-0.85x the time of the gathering one at
+// T = 2048 and 0.95x on the 13824 x 5120 layer at T = 512, but more at T <= 512
+// on smaller layers; with 1 x 256 groups it is never faster (0.99-1.6x).  Both
+// kernels' times hardly depend on the density.
+bool prefill_prefers_dense(const gs_packed* p, int64_t T) { return p->g_in == 128 && p->kept > 0 && T >= 1024; }
+
+gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
+                               cudaStream_t s) {
+  if (T <= 0 || n <= 0) return GS_OK;
+  const int kw = ps[0]->g_in;
+  for (int i = 0; i < n; ++i)
+    if (ps[i]->g_in != kw || ps[i]->g_out != 1 || ps[i]->kept == 0) return GS_ERR_UNSUPPORTED;
+  if (kw != 256 && kw != 128) return GS_ERR_UNSUPPORTED;
+  if ((kw == 256 ? d_set_attr<256>() : d_set_attr<128>()) != cudaSuccess) return GS_ERR_CUDA;
+  int* err = device_error_flag();
+  if (!err) return GS_ERR_CUDA;
+  // most tensor work per unit (the window's chunks with a kept row) first
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return ps[a]->in > ps[b]->in; });
+  const int64_t max_pairs = d_sm_count() / 2;
+  for (int b0 = 0; b0 < n; b0 += kDMaxLayers) {
+    const int nb = std::min(kDMaxLayers, n - b0);
+    DParams P;
+    std::memset(&P, 0, sizeof(P));
+    int64_t tiles = 0;
+    for (int k = 0; k < nb; ++k) {
+      const int i = order[b0 + k];
+      const gs_packed* p = ps[i];
+      DLayer& L = P.L[k];
+      if (!encode_tmap_slabs_bf16(&L.xmap, xs[i], (uint64_t)p->in, (uint64_t)T, kDM, 1)) return GS_ERR_CUDA;
+      L.tiles = p->tiles;
+      L.win_off16 = p->win_off16;
+      L.kmask16 = p->kmask16;
+      L.y = static_cast<uint16_t*>(ys[i]);
+      L.out = (int32_t)p->out;
+      L.G = p->G;
+      L.nw16 = p->nw16;
+      L.n_m = (int32_t)((T + 2 * kDM - 1) / (2 * kDM));
+      L.tile_begin = (int32_t)tiles;
+      tiles += (int64_t)L.n_m * ((p->out + kDW - 1) / kDW);
+    }
+    if (tiles > INT32_MAX) return GS_ERR_UNSUPPORTED;
+    P.n_layers = nb;
+    P.T = (int32_t)T;
+    P.n_tiles = (int32_t)tiles;
+    P.err = err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * std::min<int64_t>(tiles, max_pairs)));
+    cfg.blockDim = dim3(kDThreads);
+    cfg.dynamicSmemBytes = kDSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = kw == 256 ? cudaLaunchKernelEx(&cfg, k_prefill_dense<256>, P)
+                                    : cudaLaunchKernelEx(&cfg, k_prefill_dense<128>, P);
+    note_launch();
+    if (e != cudaSuccess) return GS_ERR_CUDA;
+  }
+  return GS_OK;
+}
+
+}  // namespace gs

@@ -18,7 +18,7 @@ _PKG = Path(__file__).resolve().parent
 LIB_PATH = _PKG / "libgroupsparse.so"
 
 GS_OK, GS_ERR_INVALID_ARG, GS_ERR_UNSUPPORTED, GS_ERR_OOM, GS_ERR_CUDA, GS_ERR_DEVICE_TIMEOUT = range(6)
-ALGO_AUTO, ALGO_DECODE, ALGO_PREFILL = 0, 1, 2
+ALGO_AUTO, ALGO_DECODE, ALGO_PREFILL, ALGO_PREFILL_DENSE = 0, 1, 2, 3
 
 _c_i64p = ctypes.POINTER(ctypes.c_int64)
 _c_i32p = ctypes.POINTER(ctypes.c_int32)

@@ -200,7 +200,8 @@ def test_narrow_rows_linear(gs, T):
         xb = wl.random_activation_bits(T, inp, seed=T + seed)
         x = to_dev(xb)
         toks = None if T <= 300 else sample_tokens(T, seed)
-        for algo in ((gs.ALGO_DECODE, gs.ALGO_PREFILL) if T <= 300 else (gs.ALGO_PREFILL,)):
+        algos = (gs.ALGO_PREFILL, gs.ALGO_PREFILL_DENSE)
+        for algo in ((gs.ALGO_DECODE,) + algos if T <= 300 else algos):
             y = to_bits(gs.linear(x, p, algo=algo))
             if toks is None:
                 yr, A = orc.linear(xb, Wb, B, 1, 128)
@@ -220,7 +221,7 @@ def test_narrow_rows_batched_with_other_shapes(gs):
         B = wl.random_mask(1024 // go, 2048 // gi, 0.5, seed=90 + i)
         p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), go, gi)
         layers.append((Wb, B, p, go, gi))
-    for T in (3, 16, 200):
+    for T in (3, 16, 200, 1024):   # 1024: the 1 x 128 layers take the zero-filled prefill kernel
         xbs = [wl.random_activation_bits(T, 2048, seed=100 + i + T) for i in range(len(layers))]
         ys = [torch.empty((T, 1024), dtype=torch.bfloat16, device="cuda") for _ in layers]
         gs.linear_batched_into([to_dev(b) for b in xbs], [l[2] for l in layers], ys)

@@ -98,6 +98,18 @@ def test_prefill_parity(gs, out, inp, d, seed):
     assert gs.device_status() == gs.GS_OK
 
 
+@pytest.mark.parametrize("out,inp,d,seed", PREFILL_SHAPES)
+def test_prefill_dense_parity(gs, out, inp, d, seed):
+    """The zero-filled-window kernel: pruned rows multiply as zeros, so y keeps the same bound."""
+    Wb, B = layer(out, inp, d, seed)
+    p = packed(gs, Wb, B)
+    for T in PREFILL_T:
+        xb = wl.random_activation_bits(T, inp, seed=seed * 100 + T + 9)
+        y = gs.linear(to_dev(xb), p, algo=gs.ALGO_PREFILL_DENSE)
+        assert_within_bound(to_bits(y), xb, Wb, B, what=f"prefill-dense {out}x{inp} d={d} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
 def test_auto_dispatch_and_empty_batch(gs):
     import torch
     Wb, B = layer(1024, 1024, 0.5, 4)
