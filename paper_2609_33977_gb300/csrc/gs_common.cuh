@@ -64,6 +64,7 @@ struct gs_packed {
   int32_t nwin;       // square groups: ceil(out / 128) windows of 128 output rows
   int32_t* gwoff;     // [G][nwin + 1]: first packed tile of column block v in window w (+ end)
   uint8_t* gwmask;    // [G][nwin]: bit i = block row (128/g) w + i kept in column block v
+  int32_t* gtidx;     // [Gout][G]: packed tile of group (u, v), -1 if pruned (decode-regime lookups)
   alignas(64) unsigned char gmaps[8][128];   // W slice descriptors, box heights g, 2g, ..., 128 rows
   alignas(64) unsigned char hmaps[8][128];   // CTA-pair halves: rows [r g/2, r g/2 + g/2) of 1..8 consecutive tiles
 };
@@ -144,6 +145,10 @@ gs_status sq_unpack(const gs_packed* p, void* W_hat, cudaStream_t s);
 gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
                             cudaStream_t s);
 void sq_release(gs_packed* p);
+// sq_decode.cu: square groups, T <= sq_decode_max_tokens(): layers ps[idx[0..n)] (same g, kept > 0, n <= 8)
+int sq_decode_max_tokens();
+gs_status sq_decode_batched(const void* const* xs, const gs_packed* const* ps, const int* idx, int n, int T,
+                            void* const* ys, cudaStream_t s);
 inline bool is_square(const gs_packed* p) { return p->g_out > 1; }
 
 // train.cu: Gumbel-Sigmoid sample and straight-through backward (Sec. 2.2)

@@ -444,17 +444,22 @@ __device__ __forceinline__ uint4 sq_ld16(const void* p) {
 __global__ void k_sq_compact(const uint16_t* __restrict__ W, const uint8_t* __restrict__ mask, int32_t g,
                              int32_t in, int32_t Gout, int32_t Gin, int32_t R, int32_t nwin,
                              const int32_t* __restrict__ gwoff, const uint8_t* __restrict__ gwmask,
-                             int32_t* __restrict__ row_idx, uint16_t* __restrict__ tiles) {
+                             int32_t* __restrict__ row_idx, uint16_t* __restrict__ tiles,
+                             int32_t* __restrict__ gtidx) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int per_row = g / 8;   // 16-byte pieces per block row
   for (int64_t e = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < (int64_t)Gout * Gin;
        e += warps) {
     const int u = (int)(e / Gin), v = (int)(e % Gin);
-    if (mask[e] == 0) continue;
+    if (mask[e] == 0) {
+      if (lane == 0) gtidx[e] = -1;
+      continue;
+    }
     const int w = u / R, i = u % R;
     const uint32_t mk = gwmask[(int64_t)v * nwin + w];
     const int64_t j = gwoff[(int64_t)v * (nwin + 1) + w] + __popc(mk & ((1u << i) - 1u));
+    if (lane == 0) gtidx[e] = (int32_t)j;
     uint16_t* dst = tiles + j * (int64_t)g * g;
     for (int c = lane; c < g * per_row; c += 32) {
       const int r = c / per_row, k8 = c % per_row;
@@ -628,11 +633,12 @@ gs_status sq_pack(const void* W, const uint8_t* mask, gs_packed* p, cudaStream_t
   const size_t tile_elems = (size_t)g * (size_t)g;
   if ((st = alloc((void**)&p->row_idx, sizeof(int32_t) * (size_t)kept)) != GS_OK) return st;
   if ((st = alloc((void**)&p->tiles, 2 * tile_elems * (size_t)kept)) != GS_OK) return st;
+  if ((st = alloc((void**)&p->gtidx, sizeof(int32_t) * (size_t)(Gout * Gin))) != GS_OK) return st;
   p->device_bytes = total;
   if (kept > 0) {
     k_sq_compact<<<sq_grid_for(Gout * Gin), 256, 0, s>>>(static_cast<const uint16_t*>(W), mask, g, (int32_t)p->in,
                                                          (int32_t)Gout, (int32_t)Gin, R, (int32_t)nwin, p->gwoff,
-                                                         p->gwmask, p->row_idx, p->tiles);
+                                                         p->gwmask, p->row_idx, p->tiles, p->gtidx);
     note_launch();
     if (cudaGetLastError() != cudaSuccess) return GS_ERR_CUDA;
     // W slice descriptors: the tiles as a [K g][g] matrix (g = 128: 64-wide slabs)
@@ -677,8 +683,10 @@ gs_status sq_unpack(const gs_packed* p, void* W_hat, cudaStream_t s) {
 void sq_release(gs_packed* p) {
   if (p->gwoff) cudaFree(p->gwoff);
   if (p->gwmask) cudaFree(p->gwmask);
+  if (p->gtidx) cudaFree(p->gtidx);
   p->gwoff = nullptr;
   p->gwmask = nullptr;
+  p->gtidx = nullptr;
 }
 
 gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
@@ -703,6 +711,31 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
     std::stable_sort(o.begin(), o.end(), [&](int a, int b) {
       return (double)ps[a]->kept / ps[a]->nwin > (double)ps[b]->kept / ps[b]->nwin;
     });
+    // Decode regime: the tile-streaming kernel, one launch per 16 tokens, heaviest
+    // rows (widest input) first.  Its time grows with the 16-token blocks while
+    // the tensor-core kernel's stays flat up to 128 tokens; on the LLaMA-2 7B
+    // block shapes at d = 0.5 the blocks cost less up to 128 / 64 / 32 / 16
+    // tokens for g = 16 / 32 / 64 / 128.
+    const int g = 16 << gi;
+    if (T <= (int64_t)(2048 / g)) {
+      std::stable_sort(o.begin(), o.end(), [&](int a, int b) { return ps[a]->in > ps[b]->in; });
+      const int blk = sq_decode_max_tokens();
+      std::vector<const void*> xb(n);
+      std::vector<void*> yb(n);
+      for (int64_t t0 = 0; t0 < T; t0 += blk) {
+        const int tb = (int)std::min<int64_t>(blk, T - t0);
+        for (int i : o) {
+          xb[i] = static_cast<const uint16_t*>(xs[i]) + t0 * ps[i]->in;
+          yb[i] = static_cast<uint16_t*>(ys[i]) + t0 * ps[i]->out;
+        }
+        for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
+          const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
+          const gs_status st = sq_decode_batched(xb.data(), ps, o.data() + b0, nb, tb, yb.data(), s);
+          if (st != GS_OK) return st;
+        }
+      }
+      continue;
+    }
     for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
       const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
       gs_status st;

@@ -65,7 +65,7 @@ def test_pack_and_unpack_are_bit_exact(gs, g, out, inp, d, seed):
 
 
 @pytest.mark.parametrize("g", [16, 32, 64, 128])
-@pytest.mark.parametrize("T", [1, 3, 16, 64, 128, 129, 300])
+@pytest.mark.parametrize("T", [1, 3, 8, 9, 16, 17, 64, 128, 129, 300])
 def test_linear_small_layers(gs, g, T):
     for out, inp, d, seed in [(256, 512, 0.5, 11), (384, 1024, 0.3, 12), (128, 128, 1.0, 13)]:
         Wb, B, p = make(gs, out, inp, g, d, seed)
@@ -95,18 +95,19 @@ def test_outliers_zero_rows_and_empty_layers(gs):
     B = wl.random_mask(out // g, inp // g, 0.5, seed=32)
     B[0:4, :] = 0                        # block rows 0..3 = the whole first 128-row window
     B[9, :] = 0                          # one block row pruned everywhere
-    xb = wl.random_activation_bits(40, inp, seed=33)
-    xf = wl.bf16_bits_to_f32(xb)
-    xf[:, ::97] *= 20.0
-    xb = wl.f32_to_bf16_bits(xf)
     p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), g, g)
-    y = to_bits(gs.linear(to_dev(xb), p))
-    check_y(y, xb, Wb, B, g, what="pruned window")
-    assert not y[:, :128].any()
     p0 = gs.pack_groups(to_dev(Wb), torch.zeros((out // g, inp // g), dtype=torch.uint8, device="cuda"), g, g)
     assert p0.kept == 0
-    y0 = gs.linear(to_dev(xb), p0)
-    assert not to_bits(y0).any()
+    for T in (5, 40):   # the decode-regime and the tensor-core kernels
+        xb = wl.random_activation_bits(T, inp, seed=33)
+        xf = wl.bf16_bits_to_f32(xb)
+        xf[:, ::97] *= 20.0
+        xb = wl.f32_to_bf16_bits(xf)
+        y = to_bits(gs.linear(to_dev(xb), p))
+        check_y(y, xb, Wb, B, g, what=f"pruned window T={T}")
+        assert not y[:, :128].any() and not y[:, 9 * g:10 * g].any()
+        y0 = gs.linear(to_dev(xb), p0)
+        assert not to_bits(y0).any()
 
 
 def test_batched_mixes_shapes(gs):
