@@ -133,8 +133,9 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
                                  void* const* ys, cudaStream_t s);
 int prefill_max_chunks();
 // prefill_dense.cu: zero-filled windows (1 x 128 / 1 x 256 layers with kept groups)
+// (layers ps[idx[k]], k < n, when idx is given; else ps[0..n))
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
-                               cudaStream_t s);
+                               cudaStream_t s, const int* idx = nullptr);
 // whether the zero-filled kernel is the faster one for this layer and token count
 bool prefill_prefers_dense(const gs_packed* p, int64_t T);
 

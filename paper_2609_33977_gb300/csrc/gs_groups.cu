@@ -57,6 +57,7 @@ constexpr uint32_t kSqTmemCols = kSqAccBufs * kSqWin;
 constexpr int kSqEpiWarps = 4;
 constexpr int kSqThreads = (2 + kSqEpiWarps) * 32;
 constexpr int kSqMaxLayers = 8;
+constexpr int kSqDenseMaxG = 32;          // above the decode regime, g <= this takes the zero-filled kernel
 constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R <= 8)
 constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
 constexpr uint64_t kSqDrainLimitNs = 200000000ull;
@@ -734,6 +735,13 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
           if (st != GS_OK) return st;
         }
       }
+      continue;
+    }
+    // Small tiles: the zero-filled-window tensor-core kernel (dense-layer tensor
+    // work, no per-column-block handshake) is the faster one
+    if (g <= kSqDenseMaxG) {
+      const gs_status st = launch_prefill_dense(xs, ps, (int)o.size(), T, ys, s, o.data());
+      if (st != GS_OK) return st;
       continue;
     }
     for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {

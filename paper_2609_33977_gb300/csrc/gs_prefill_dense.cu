@@ -62,11 +62,13 @@ static_assert(kDStageBytes % 1024 == 0 && kDXBytes % 1024 == 0, "stages keep 102
 
 struct DLayer {
   CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 1
-  const uint16_t* tiles;     // [kept][KW]
-  const int32_t* win_off16;  // [G][nw16 + 1]
-  const uint16_t* kmask16;   // [G][nw16]
+  const uint16_t* tiles;     // 1 x KW: [kept][KW]; square g x g: [kept][g][g]
+  const int32_t* win_off16;  // 1 x KW: [G][nw16 + 1]
+  const uint16_t* kmask16;   // 1 x KW: [G][nw16]
+  const int32_t* gtidx;      // square: [out / g][in / g] packed tile of each group, -1 if pruned
   uint16_t* y;
-  int32_t out, G, nw16, n_m, tile_begin;
+  int32_t out, G, nw16, n_m, tile_begin;   // G: chunks of KW columns (square: 64-column slabs)
+  int32_t Gin;               // square: in / g
 };
 struct DParams {
   DLayer L[kDMaxLayers];
@@ -95,15 +97,21 @@ __device__ __forceinline__ void fence_proxy_async_cta() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Chunks c0 .. c0 + 31 with at least one kept row in window w, in order, into buf.
+// Chunks c0 .. c0 + 31 with at least one kept row in window w, in order, into
+// buf (square groups: every 64-column slab)
+template <int SQ>
 __device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane, int* buf) {
   const int c = c0 + lane;
   __syncwarp();   // every lane is done reading the previous batch
   bool ne = false;
   if (c < L.G) {
-    const int32_t* wo = L.win_off16 + (int64_t)c * (L.nw16 + 1);
-    const int lo = w * (kDW / kWin16), hi = min(lo + kDW / kWin16, L.nw16);
-    ne = wo[hi] > wo[lo];
+    if constexpr (SQ > 0) {
+      ne = true;
+    } else {
+      const int32_t* wo = L.win_off16 + (int64_t)c * (L.nw16 + 1);
+      const int lo = w * (kDW / kWin16), hi = min(lo + kDW / kWin16, L.nw16);
+      ne = wo[hi] > wo[lo];
+    }
   }
   const uint32_t ballot = __ballot_sync(0xffffffffu, ne);
   if (ne) buf[__popc(ballot & ((1u << lane) - 1u))] = c;
@@ -116,7 +124,9 @@ __device__ __forceinline__ uint32_t d_pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-template <int KW>
+// KW: chunk width (1 x KW groups; 64 for square groups, one slab per item);
+// SQ: 0, or g for square g x g groups
+template <int KW, int SQ>
 __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_constant__ DParams P) {
   constexpr int kSlabs = KW / kDSlabK;   // stages per chunk
   extern __shared__ uint8_t d_smem_raw[];
@@ -179,8 +189,9 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       const int lt = u - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
       const int tok0 = m * 2 * kDM + (int)rank * kDM;
-      // metadata of this lane's rows in chunk c: the window's kept mask and first
-      // packed row (two independent loads, issued one item ahead of their use)
+      const int j = lane & 7;   // 16-byte piece of a row this lane copies
+      // 1 x KW: metadata of this lane's rows in chunk c, the window's kept mask
+      // and first packed row (two independent loads, issued one item ahead of use)
       auto load_meta = [&](int c, uint32_t (&km)[kOwn], int (&wo)[kOwn]) {
 #pragma unroll
         for (int q = 0; q < kOwn; ++q) {
@@ -190,31 +201,56 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
           wo[q] = L.win_off16[(int64_t)c * (L.nw16 + 1) + b16];
         }
       };
+      // square: packed tile of each piece this lane copies in slab c (its row's
+      // block row, its columns' block column), issued one item ahead of use
+      auto load_tiles = [&](int c, int (&tv)[kCopies]) {
+#pragma unroll
+        for (int i = 0; i < kCopies; ++i) {
+          const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
+          const int k = c * kDSlabK + 8 * j;
+          tv[i] = row < L.out ? L.gtidx[(int64_t)(row / (SQ > 0 ? SQ : 1)) * L.Gin + k / (SQ > 0 ? SQ : 1)] : -1;
+        }
+      };
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
-        const int n_it = d_items(L, w, c0, lane, ibuf);
+        const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         uint32_t km_n[kOwn];
         int wo_n[kOwn];
-        if (n_it > 0) load_meta(ibuf[0], km_n, wo_n);
+        int tv_n[kCopies];
+        if (n_it > 0) {
+          if constexpr (SQ > 0) load_tiles(ibuf[0], tv_n);
+          else load_meta(ibuf[0], km_n, wo_n);
+        }
         for (int it = 0; it < n_it && ok; ++it) {
           const int c = ibuf[it];
-          // packed positions in chunk c of the rows this lane looks up (-1: pruned / beyond out)
-          int prow[kOwn];
+          // element offset of each piece this lane copies (slab 0 of the item), -1: zeros
+          int64_t soff[kCopies];
+          if constexpr (SQ > 0) {
 #pragma unroll
-          for (int q = 0; q < kOwn; ++q) {
-            const int h = (int)rank * kDHalf + warp * kRows + 32 * q + lane;
-            const int b16 = w * (kDW / kWin16) + (h >> 4), bit = h & 15;
-            const bool kept = b16 < L.nw16 && ((km_n[q] >> bit) & 1u);
-            prow[q] = kept ? wo_n[q] + __popc(km_n[q] & ((1u << bit) - 1u)) : -1;
-          }
-          if (it + 1 < n_it) load_meta(ibuf[it + 1], km_n, wo_n);
-          // the rows this lane copies: warp * kRows + 4 i + (lane >> 3)
-          int crow[kCopies];
+            for (int i = 0; i < kCopies; ++i) {
+              const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
+              const int k = c * kDSlabK + 8 * j;
+              soff[i] = tv_n[i] >= 0 ? ((int64_t)tv_n[i] * SQ + row % SQ) * SQ + k % SQ : -1;
+            }
+            if (it + 1 < n_it) load_tiles(ibuf[it + 1], tv_n);
+          } else {
+            // packed positions in chunk c of the rows this lane looks up (-1: pruned / beyond out)
+            int prow[kOwn];
 #pragma unroll
-          for (int i = 0; i < kCopies; ++i) {
-            const int r = 4 * i + (lane >> 3);   // row within the warp's block: owner lane r % 32, slot r / 32
-            crow[i] = __shfl_sync(0xffffffffu, prow[r >> 5], r & 31);
+            for (int q = 0; q < kOwn; ++q) {
+              const int h = (int)rank * kDHalf + warp * kRows + 32 * q + lane;
+              const int b16 = w * (kDW / kWin16) + (h >> 4), bit = h & 15;
+              const bool kept = b16 < L.nw16 && ((km_n[q] >> bit) & 1u);
+              prow[q] = kept ? wo_n[q] + __popc(km_n[q] & ((1u << bit) - 1u)) : -1;
+            }
+            if (it + 1 < n_it) load_meta(ibuf[it + 1], km_n, wo_n);
+            // the rows this lane copies: warp * kRows + 4 i + (lane >> 3)
+#pragma unroll
+            for (int i = 0; i < kCopies; ++i) {
+              const int r = 4 * i + (lane >> 3);   // row within the warp's block: owner lane r % 32, slot r / 32
+              const int pr = __shfl_sync(0xffffffffu, prow[r >> 5], r & 31);
+              soff[i] = pr >= 0 ? (int64_t)pr * KW + 8 * j : -1;
+            }
           }
-          const int j = lane & 7;   // 16-byte piece of the row
 #pragma unroll 1
           for (int sl = 0; sl < kSlabs && ok; ++sl) {
             bool got = true;
@@ -237,9 +273,9 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             for (int i = 0; i < kCopies; ++i) {
               const int rr = warp * kRows + 4 * i + (lane >> 3);
               const uint32_t dst = wb + (uint32_t)rr * 128u + (uint32_t)((j ^ (rr & 7)) << 4);   // 128-byte swizzle
-              const bool kept = crow[i] >= 0;
+              const bool kept = soff[i] >= 0;
               // a pruned row reads nothing (source size 0) and is filled with zeros
-              const uint16_t* src = kept ? L.tiles + (int64_t)crow[i] * KW + sl * kDSlabK + 8 * j : L.tiles;
+              const uint16_t* src = kept ? L.tiles + soff[i] + sl * kDSlabK : L.tiles;
               cp_async16_zfill(dst, src, kept ? 16u : 0u);
             }
             cp_async_arrive_noinc(&wfull_bar[stage]);   // fires once this thread's copies have landed
@@ -271,7 +307,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int w = (u - L.tile_begin) / L.n_m;
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
-        const int n_st = d_items(L, w, c0, lane, ibuf) * kSlabs;
+        const int n_st = d_items<SQ>(L, w, c0, lane, ibuf) * kSlabs;
         if (lane == 0) {
           for (int k = 0; k < n_st && ok;) {
             if (!mbar_wait_bounded(&wfull_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
@@ -322,7 +358,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       const uint32_t d = tmem + (uint32_t)(buf * kDW);
       bool first = true;
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
-        const int n_it = d_items(L, w, c0, lane, ibuf);
+        const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         if (lane == 0) {
           for (int it = 0; it < n_it * kSlabs && ok; ++it) {
             if (!mbar_wait_bounded_cluster(&full_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs,
@@ -368,8 +404,8 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       const int lt = u - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
       // a window with no kept row in any chunk has no MMA: its rows are zero
-      bool any = false;
-      {
+      bool any = SQ > 0;   // square groups: every slab has MMAs
+      if constexpr (SQ == 0) {
         const int lo = w * (kDW / kWin16), hi = min(lo + kDW / kWin16, L.nw16);
         for (int c = lane; c < L.G && !any; c += 32) {
           const int32_t* wo = L.win_off16 + (int64_t)c * (L.nw16 + 1);
@@ -447,14 +483,21 @@ int d_sm_count() {
   return n;
 }
 
-template <int KW>
+template <int KW, int SQ>
 cudaError_t d_set_attr() {
   static std::once_flag once;
   static cudaError_t err = cudaSuccess;
   std::call_once(once, []() {
-    err = cudaFuncSetAttribute(k_prefill_dense<KW>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDSmem);
+    err = cudaFuncSetAttribute(k_prefill_dense<KW, SQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDSmem);
   });
   return err;
+}
+
+template <int KW, int SQ>
+cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
+  const cudaError_t e = d_set_attr<KW, SQ>();
+  if (e != cudaSuccess) return e;
+  return cudaLaunchKernelEx(&cfg, k_prefill_dense<KW, SQ>, P);
 }
 
 }  // namespace
@@ -467,18 +510,20 @@ cudaError_t d_set_attr() {
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) { return p->g_in == 128 && p->kept > 0 && T >= 1024; }
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
-                               cudaStream_t s) {
+                               cudaStream_t s, const int* idx) {
   if (T <= 0 || n <= 0) return GS_OK;
-  const int kw = ps[0]->g_in;
-  for (int i = 0; i < n; ++i)
-    if (ps[i]->g_in != kw || ps[i]->g_out != 1 || ps[i]->kept == 0) return GS_ERR_UNSUPPORTED;
-  if (kw != 256 && kw != 128) return GS_ERR_UNSUPPORTED;
-  if ((kw == 256 ? d_set_attr<256>() : d_set_attr<128>()) != cudaSuccess) return GS_ERR_CUDA;
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = idx ? idx[i] : i;
+  const int kw = ps[order[0]]->g_in, go = ps[order[0]]->g_out;
+  for (int i : order)
+    if (ps[i]->g_in != kw || ps[i]->g_out != go || ps[i]->kept == 0) return GS_ERR_UNSUPPORTED;
+  const int sq = go > 1 ? go : 0;   // square g x g groups
+  if (sq ? (sq != kw || (sq != 16 && sq != 32 && sq != 64)) : (kw != 256 && kw != 128)) return GS_ERR_UNSUPPORTED;
+  for (int i : order)
+    if (sq && !ps[i]->gtidx) return GS_ERR_UNSUPPORTED;
   int* err = device_error_flag();
   if (!err) return GS_ERR_CUDA;
-  // most tensor work per unit (the window's chunks with a kept row) first
-  std::vector<int> order(n);
-  for (int i = 0; i < n; ++i) order[i] = i;
+  // most tensor work per unit (the widest input) first
   std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return ps[a]->in > ps[b]->in; });
   const int64_t max_pairs = d_sm_count() / 2;
   for (int b0 = 0; b0 < n; b0 += kDMaxLayers) {
@@ -492,12 +537,19 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
       DLayer& L = P.L[k];
       if (!encode_tmap_slabs_bf16(&L.xmap, xs[i], (uint64_t)p->in, (uint64_t)T, kDM, 1)) return GS_ERR_CUDA;
       L.tiles = p->tiles;
-      L.win_off16 = p->win_off16;
-      L.kmask16 = p->kmask16;
       L.y = static_cast<uint16_t*>(ys[i]);
       L.out = (int32_t)p->out;
-      L.G = p->G;
-      L.nw16 = p->nw16;
+      if (sq) {
+        if (p->in % kDSlabK != 0) return GS_ERR_UNSUPPORTED;
+        L.gtidx = p->gtidx;
+        L.Gin = p->G;
+        L.G = (int32_t)(p->in / kDSlabK);
+      } else {
+        L.win_off16 = p->win_off16;
+        L.kmask16 = p->kmask16;
+        L.G = p->G;
+        L.nw16 = p->nw16;
+      }
       L.n_m = (int32_t)((T + 2 * kDM - 1) / (2 * kDM));
       L.tile_begin = (int32_t)tiles;
       tiles += (int64_t)L.n_m * ((p->out + kDW - 1) / kDW);
@@ -519,8 +571,11 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = kw == 256 ? cudaLaunchKernelEx(&cfg, k_prefill_dense<256>, P)
-                                    : cudaLaunchKernelEx(&cfg, k_prefill_dense<128>, P);
+    const cudaError_t e = sq == 16   ? d_launch<kDSlabK, 16>(cfg, P)
+                          : sq == 32 ? d_launch<kDSlabK, 32>(cfg, P)
+                          : sq == 64 ? d_launch<kDSlabK, 64>(cfg, P)
+                          : kw == 256 ? d_launch<256, 0>(cfg, P)
+                                      : d_launch<128, 0>(cfg, P);
     note_launch();
     if (e != cudaSuccess) return GS_ERR_CUDA;
   }
