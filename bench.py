@@ -994,14 +994,16 @@ def run_layer(args):
     g.manual_seed(1234)
     W = (torch.randn((out, inp), generator=g, device=dev) * 0.02).to(torch.bfloat16)
     gsz = args.group
+    gin = args.group_in
     if gsz:
         B = (torch.rand((out // gsz, inp // gsz), generator=g, device=dev) < args.density).to(torch.uint8)
     else:
-        B = (torch.rand((out, inp // 256), generator=g, device=dev) < args.density).to(torch.uint8)
+        B = (torch.rand((out, inp // gin), generator=g, device=dev) < args.density).to(torch.uint8)
     x = torch.randn((T, inp), generator=g, device=dev).to(torch.bfloat16)
-    p = gs.pack_groups(W, B, gsz, gsz) if gsz else gs.pack(W, B)
+    p = gs.pack_groups(W, B, gsz, gsz) if gsz else gs.pack_groups(W, B, 1, gin)
     y = torch.empty((T, out), dtype=torch.bfloat16, device=dev)
-    algo = {"auto": gs.ALGO_AUTO, "decode": gs.ALGO_DECODE, "prefill": gs.ALGO_PREFILL}[args.algo]
+    algo = {"auto": gs.ALGO_AUTO, "decode": gs.ALGO_DECODE, "prefill": gs.ALGO_PREFILL,
+            "prefill_dense": gs.ALGO_PREFILL_DENSE}[args.algo]
     for _ in range(args.warmup):
         gs.linear_into(x, p, y, algo=algo)
     torch.cuda.synchronize()
@@ -1018,12 +1020,12 @@ def run_layer(args):
         kept_w = kept * gsz * gsz
         nbytes = 2 * kept_w + 4 * kept + 2 * T * inp + 2 * T * out
     else:
-        kept_w = 256 * kept
-        G, nw16 = inp // 256, (out + 15) // 16
+        kept_w = gin * kept
+        G, nw16 = inp // gin, (out + 15) // 16
         nbytes = 2 * kept_w + 6 * G * nw16 + 2 * T * inp + 2 * T * out
     flops = 2.0 * T * kept_w
     assert gs.device_status() == gs.GS_OK
-    print(json.dumps({"layer": f"{out}x{inp}", "group": f"{gsz}x{gsz}" if gsz else "1x256", "T": T,
+    print(json.dumps({"layer": f"{out}x{inp}", "group": f"{gsz}x{gsz}" if gsz else f"1x{gin}", "T": T,
                       "density": args.density, "algo": args.algo, "kept": kept,
                       "us": s * 1e6, "GB/s": nbytes / s / 1e9, "TFLOP/s": flops / s / 1e12}), flush=True)
     return 0
@@ -1046,7 +1048,9 @@ def main():
     ap.add_argument("--tokens", type=int, default=16)
     ap.add_argument("--group", type=int, default=0, help="single-layer mode: square g x g groups (0 = 1x256)")
     ap.add_argument("--density", type=float, default=0.5)
-    ap.add_argument("--algo", choices=["auto", "decode", "prefill"], default="auto")
+    ap.add_argument("--algo", choices=["auto", "decode", "prefill", "prefill_dense"], default="auto")
+    ap.add_argument("--group-in", type=int, default=256, choices=[128, 256],
+                    help="single-layer mode with --group 0: 1 x group_in groups")
     ap.add_argument("--train-op", action="store_true",
                     help="time only the Gumbel-Sigmoid sample and the straight-through backward")
     ap.add_argument("--group-shapes", action="store_true",
