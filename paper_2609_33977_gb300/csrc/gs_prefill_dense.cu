@@ -16,9 +16,11 @@
 //
 // Roles (one CTA per SM, units persistent over the pairs): warps 0..3
 // producers (warp-cooperative 16-byte cp.async of the window's rows, zero-filled
-// for pruned rows; warp 0 lane 0 also issues the x boxes), warp 4 TMEM
-// allocator + single-thread MMA issuer (leader), warps 5..8 epilogue, warp 9
-// forwarder.  Producers never wait for their own copies: each thread's copies
+// for pruned rows), warp 4 TMEM allocator + single-thread MMA issuer (leader),
+// warps 5..8 epilogue, warp 9 forwarder, warp 10 x producer (TMA).  W slots
+// and x slots are two rings: the W ring (nine 16 KB slots) runs three times as
+// deep as the x ring (three), because a W slot's round trip (copies landing,
+// fences, arrival at the leader) is about three times a TMA's.  Producers never wait for their own copies: each thread's copies
 // of a stage signal a local barrier (cp.async.mbarrier.arrive), and the
 // forwarder, once all have landed, fences them to the async proxy and arrives
 // on the leader's full barrier.  Every wait is bounded.
@@ -41,24 +43,30 @@ constexpr int kDHalf = kDW / 2;                   // window rows each CTA holds
 constexpr int kDSlabK = 64;                       // k per stage (one 128-byte swizzle row)
 constexpr int kDXBytes = kDM * kDSlabK * 2;       // 16 KB of x per stage
 constexpr int kDWBytes = kDHalf * kDSlabK * 2;    // 16 KB of W rows per stage
-constexpr int kDStageBytes = kDXBytes + kDWBytes;
-constexpr int kDStages = 6;
+// Two rings: W slots (the long round trip: copies landing, forwarder fences,
+// arrival at the leader) run three times as deep as x slots (TMA); measured
+// 9 / 3 ahead of 8 / 4, 7 / 5 and 10 / 2.
+constexpr int kDWStages = 9;
+constexpr int kDXStages = 3;
+constexpr int kDXRing = kDXStages * kDXBytes;     // 64 KB at offset 0
+constexpr int kDWRing = kDWStages * kDWBytes;     // 128 KB after it
 constexpr int kDProdWarps = 4;                   // warps that copy W rows
 constexpr int kDMmaWarp = kDProdWarps;
 constexpr int kDEpiWarp0 = kDProdWarps + 1;
 constexpr int kDEpiWarps = 4;
 constexpr int kDFwdWarp = kDEpiWarp0 + kDEpiWarps;
-constexpr int kDThreads = (kDFwdWarp + 1) * 32;
+constexpr int kDXWarp = kDFwdWarp + 1;            // x TMA producer
+constexpr int kDThreads = (kDXWarp + 1) * 32;
 constexpr int kDAccBufs = 2;
 constexpr uint32_t kDTmemCols = kDAccBufs * kDW;  // 512
 constexpr int kDMaxLayers = 8;
 constexpr uint64_t kDWaitLimitNs = 2000000000ull;
 constexpr uint64_t kDDrainLimitNs = 200000000ull;
 constexpr int kDIbufBytes = 1024;                // per-warp chunk lists of d_items
-constexpr int kDSmem = kDStages * kDStageBytes + kDIbufBytes + 1024;
+constexpr int kDSmem = kDXRing + kDWRing + kDIbufBytes + 1024;
 static_assert(kDHalf % (kDProdWarps * 32) == 0, "producer warps split the CTA's window rows evenly");
 static_assert(kDSmem <= 227 * 1024, "shared memory budget");
-static_assert(kDStageBytes % 1024 == 0 && kDXBytes % 1024 == 0, "stages keep 1024-byte alignment");
+static_assert(kDWBytes % 1024 == 0 && kDXBytes % 1024 == 0, "slots keep 1024-byte alignment");
 
 struct DLayer {
   CUtensorMap xmap;          // x as (64, T, in/64) slabs, box 64 x 128 x 1
@@ -130,9 +138,11 @@ template <int KW, int SQ>
 __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_constant__ DParams P) {
   constexpr int kSlabs = KW / kDSlabK;   // stages per chunk
   extern __shared__ uint8_t d_smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kDStages];
-  __shared__ __align__(8) uint64_t wfull_bar[kDStages];
-  __shared__ __align__(8) uint64_t empty_bar[kDStages];
+  __shared__ __align__(8) uint64_t xfull_bar[kDXStages];    // leader: both CTAs' x bytes
+  __shared__ __align__(8) uint64_t xempty_bar[kDXStages];
+  __shared__ __align__(8) uint64_t wfull_bar[kDWStages];    // local: this CTA's producer threads' copies
+  __shared__ __align__(8) uint64_t wready_bar[kDWStages];   // leader: both CTAs' forwarders
+  __shared__ __align__(8) uint64_t wempty_bar[kDWStages];
   __shared__ __align__(8) uint64_t afull_bar[kDAccBufs];
   __shared__ __align__(8) uint64_t aempty_bar[kDAccBufs];
   __shared__ __align__(8) uint64_t drain_bar;
@@ -141,15 +151,19 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(d_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs)
-  int* ibuf = reinterpret_cast<int*>(smem + kDStages * kDStageBytes) +
-              (warp <= kDMmaWarp ? warp : (warp == kDFwdWarp ? kDMmaWarp + 1 : 0)) * 32;
-  static_assert((kDMmaWarp + 2) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
+  int* ibuf = reinterpret_cast<int*>(smem + kDXRing + kDWRing) +
+              (warp <= kDMmaWarp ? warp : warp == kDFwdWarp ? kDMmaWarp + 1 : warp == kDXWarp ? kDMmaWarp + 2 : 0) * 32;
+  static_assert((kDMmaWarp + 3) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kDStages; ++s) {
-      mbar_init(&full_bar[s], 2 + 1);                  // both CTAs' forwarders + the x byte count
-      mbar_init(&wfull_bar[s], kDProdWarps * 32);       // this CTA's producer threads' copies
-      mbar_init(&empty_bar[s], 1);
+    for (int s = 0; s < kDXStages; ++s) {
+      mbar_init(&xfull_bar[s], 1);   // the leader's expect-tx of both CTAs' x bytes
+      mbar_init(&xempty_bar[s], 1);
+    }
+    for (int s = 0; s < kDWStages; ++s) {
+      mbar_init(&wfull_bar[s], kDProdWarps * 32);
+      mbar_init(&wready_bar[s], 2);
+      mbar_init(&wempty_bar[s], 1);
     }
     for (int b = 0; b < kDAccBufs; ++b) {
       mbar_init(&afull_bar[b], 1);
@@ -182,13 +196,10 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     constexpr int kOwn = kRows / 32;              // rows whose metadata a lane loads
     constexpr int kCopies = kRows / 4;            // 16-byte copies per lane per stage
     uint32_t stage = 0, phase = 0;
-    uint32_t armed = 0u, armed_par = 0u;
     bool ok = true;
     for (int u = pair; u < n_tiles && ok; u += n_pairs) {
       const DLayer& L = P.L[d_layer_of(P, u)];
-      const int lt = u - L.tile_begin;
-      const int m = lt % L.n_m, w = lt / L.n_m;
-      const int tok0 = m * 2 * kDM + (int)rank * kDM;
+      const int w = (u - L.tile_begin) / L.n_m;
       const int j = lane & 7;   // 16-byte piece of a row this lane copies
       // 1 x KW: metadata of this lane's rows in chunk c, the window's kept mask
       // and first packed row (two independent loads, issued one item ahead of use)
@@ -255,20 +266,12 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
           for (int sl = 0; sl < kSlabs && ok; ++sl) {
             bool got = true;
             if (lane == 0)
-              got = mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
+              got = mbar_wait_bounded(&wempty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
             if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
               ok = false;
               break;
             }
-            uint8_t* sx = smem + stage * kDStageBytes;
-            if (warp == 0 && lane == 0) {
-              if (rank == 0) mbar_arrive_expect_tx(&full_bar[stage], 2u * kDXBytes);
-              tma_load_3d_pair(sx, &L.xmap, mapa_shared(smem_u32(&full_bar[stage]), 0), 0, tok0,
-                               c * kSlabs + sl);
-              armed |= 1u << stage;
-              armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
-            }
-            const uint32_t wb = smem_u32(sx + kDXBytes);
+            const uint32_t wb = smem_u32(smem + kDXRing + stage * kDWBytes);
 #pragma unroll
             for (int i = 0; i < kCopies; ++i) {
               const int rr = warp * kRows + 4 * i + (lane >> 3);
@@ -279,7 +282,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
               cp_async16_zfill(dst, src, kept ? 16u : 0u);
             }
             cp_async_arrive_noinc(&wfull_bar[stage]);   // fires once this thread's copies have landed
-            if (++stage == (uint32_t)kDStages) {
+            if (++stage == (uint32_t)kDWStages) {
               stage = 0;
               phase ^= 1u;
             }
@@ -288,11 +291,49 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       }
     }
     cp_async_wait_all();
-    if (warp == 0 && lane == 0 && !ok && rank == 0) {
-      for (int s = 0; s < kDStages; ++s) {
+    __syncwarp();
+  } else if (warp == kDXWarp) {
+    // ------------------------------------------------------------ x producer
+    uint32_t stage = 0, phase = 0;
+    uint32_t armed = 0u, armed_par = 0u;
+    bool ok = true;
+    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+      const DLayer& L = P.L[d_layer_of(P, u)];
+      const int lt = u - L.tile_begin;
+      const int m = lt % L.n_m, w = lt / L.n_m;
+      const int tok0 = m * 2 * kDM + (int)rank * kDM;
+      for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
+        const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
+        if (lane == 0) {
+          for (int it = 0; it < n_it && ok; ++it) {
+            const int c = ibuf[it];
+            for (int sl = 0; sl < kSlabs && ok; ++sl) {
+              if (!mbar_wait_bounded(&xempty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs,
+                                     kDevErrTimeout)) {
+                ok = false;
+                break;
+              }
+              if (rank == 0) mbar_arrive_expect_tx(&xfull_bar[stage], 2u * kDXBytes);
+              tma_load_3d_pair(smem + stage * kDXBytes, &L.xmap, mapa_shared(smem_u32(&xfull_bar[stage]), 0), 0,
+                               tok0, c * kSlabs + sl);
+              armed |= 1u << stage;
+              armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
+              if (++stage == (uint32_t)kDXStages) {
+                stage = 0;
+                phase ^= 1u;
+              }
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      }
+    }
+    if (lane == 0 && !ok && rank == 0) {
+      // let the x copies in flight land before the CTA winds down
+      for (int s = 0; s < kDXStages; ++s) {
         if (!((armed >> s) & 1u)) continue;
         const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait_acq_cluster(&full_bar[s], (armed_par >> s) & 1u))
+        while (!mbar_try_wait_acq_cluster(&xfull_bar[s], (armed_par >> s) & 1u))
           if (globaltimer_ns() - t0 > kDDrainLimitNs) break;
       }
     }
@@ -317,17 +358,17 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             // take every following stage that has landed too, so that one
             // release fence covers them all (a release per stage is slow)
             int cnt = 1;
-            while (k + cnt < n_st && cnt < kDStages) {
-              const uint32_t s2 = (stage + (uint32_t)cnt) % kDStages;
-              const uint32_t p2 = phase ^ ((stage + (uint32_t)cnt) >= (uint32_t)kDStages ? 1u : 0u);
+            while (k + cnt < n_st && cnt < kDWStages) {
+              const uint32_t s2 = (stage + (uint32_t)cnt) % kDWStages;
+              const uint32_t p2 = phase ^ ((stage + (uint32_t)cnt) >= (uint32_t)kDWStages ? 1u : 0u);
               if (!mbar_try_wait(&wfull_bar[s2], p2)) break;
               ++cnt;
             }
             fence_proxy_async_cta();
             fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
             for (int i = 0; i < cnt; ++i) {
-              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage]), 0));
-              if (++stage == (uint32_t)kDStages) {
+              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&wready_bar[stage]), 0));
+              if (++stage == (uint32_t)kDWStages) {
                 stage = 0;
                 phase ^= 1u;
               }
@@ -340,7 +381,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     }
   } else if (warp == kDMmaWarp && rank == 0) {
     // ------------------------------------------------------------ MMA issuer (leader)
-    uint32_t stage = 0, phase = 0;
+    uint32_t ws = 0, wph = 0, xs = 0, xph = 0;   // W and x ring positions
     int buf = 0;
     uint32_t ae_ph = 0u;
     bool ok = true;
@@ -361,23 +402,28 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
         const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         if (lane == 0) {
           for (int it = 0; it < n_it * kSlabs && ok; ++it) {
-            if (!mbar_wait_bounded_cluster(&full_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs,
-                                           kDevErrTimeout)) {
+            if (!mbar_wait_bounded_cluster(&wready_bar[ws], wph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout) ||
+                !mbar_wait_bounded_cluster(&xfull_bar[xs], xph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sx = smem_u32(smem + stage * kDStageBytes);
-            const uint64_t ad = sdesc_sw128(sx), bd = sdesc_sw128(sx + kDXBytes);
+            const uint64_t ad = sdesc_sw128(smem_u32(smem + xs * kDXBytes));
+            const uint64_t bd = sdesc_sw128(smem_u32(smem + kDXRing + ws * kDWBytes));
 #pragma unroll
             for (int kk = 0; kk < kDSlabK / 16; ++kk)
               mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
                                (first && kk == 0) ? 0u : 1u);
             first = false;
-            mma_commit_pair_mc(&empty_bar[stage], 0x3);
-            if (++stage == (uint32_t)kDStages) {
-              stage = 0;
-              phase ^= 1u;
+            mma_commit_pair_mc(&wempty_bar[ws], 0x3);
+            mma_commit_pair_mc(&xempty_bar[xs], 0x3);
+            if (++ws == (uint32_t)kDWStages) {
+              ws = 0;
+              wph ^= 1u;
+            }
+            if (++xs == (uint32_t)kDXStages) {
+              xs = 0;
+              xph ^= 1u;
             }
           }
         }
@@ -502,12 +548,16 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 
 }  // namespace
 
-// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes): with
-// 1 x 128 groups this kernel takes 0.76-0.85x the time of the gathering one at
-// T = 2048 and 0.95x on the 13824 x 5120 layer at T = 512, but more at T <= 512
-// on smaller layers; with 1 x 256 groups it is never faster (0.99-1.6x).  Both
-// kernels' times hardly depend on the density.
-bool prefill_prefers_dense(const gs_packed* p, int64_t T) { return p->g_in == 128 && p->kept > 0 && T >= 1024; }
+// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes, T = 2048):
+// with 1 x 128 groups this kernel takes 0.71-0.79x the gathering kernel's time
+// (0.88x on the 13824 x 5120 layer at T = 512, more on smaller layers at
+// T <= 512); with 1 x 256 groups 0.91-0.96x on the MLP up / gate shapes
+// (out > 2 in) and 1.01-1.03x on the square and down shapes.  Both kernels'
+// times hardly depend on the density.
+bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
+  if (p->kept == 0 || T < 1024) return false;
+  return p->g_in == 128 || (p->g_in == 256 && p->out >= 2 * p->in);
+}
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
                                cudaStream_t s, const int* idx) {
