@@ -738,11 +738,16 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
       continue;
     }
     // Small tiles: the zero-filled-window tensor-core kernel (dense-layer tensor
-    // work, no per-column-block handshake) is the faster one
+    // work, no per-column-block handshake) is the faster one; it takes the
+    // layers whose input is whole 64-column slabs, the others stay below
     if (g <= kSqDenseMaxG) {
-      const gs_status st = launch_prefill_dense(xs, ps, (int)o.size(), T, ys, s, o.data());
-      if (st != GS_OK) return st;
-      continue;
+      std::vector<int> dense, rest;
+      for (int i : o) (ps[i]->in % 64 == 0 ? dense : rest).push_back(i);
+      if (!dense.empty()) {
+        const gs_status st = launch_prefill_dense(xs, ps, (int)dense.size(), T, ys, s, dense.data());
+        if (st != GS_OK) return st;
+      }
+      o = rest;
     }
     for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
       const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);

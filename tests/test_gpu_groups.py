@@ -74,6 +74,21 @@ def test_linear_small_layers(gs, g, T):
         check_y(to_bits(y), xb, Wb, B, g, what=f"g={g} {out}x{inp} T={T}")
 
 
+@pytest.mark.parametrize("g", [16, 32])
+@pytest.mark.parametrize("T", [1, 40, 300])
+def test_linear_input_not_whole_slabs(gs, g, T):
+    # in = 3 g is not a multiple of 64 columns: these layers stay on the tile-operand kernel above
+    # the decode regime, beside a layer of the same g that takes the zero-filled kernel
+    import torch
+    layers = [make(gs, 4 * g, 3 * g, g, 0.6, 80 + g), make(gs, 256, 256, g, 0.5, 81 + g)]
+    xbs = [wl.random_activation_bits(T, Wb.shape[1], seed=82 + T) for Wb, _, _ in layers]
+    ys = [torch.empty((T, Wb.shape[0]), dtype=torch.bfloat16, device="cuda") for Wb, _, _ in layers]
+    gs.linear_batched_into([to_dev(b) for b in xbs], [p for _, _, p in layers], ys)
+    for (Wb, B, _), xb, y in zip(layers, xbs, ys):
+        check_y(to_bits(y), xb, Wb, B, g, what=f"g={g} {Wb.shape} T={T}")
+    assert gs.device_status() == gs.GS_OK
+
+
 @pytest.mark.parametrize("g", [16, 32, 64, 128])
 @pytest.mark.parametrize("T", [1, 16, 2048])
 def test_linear_llama_block_shapes(gs, g, T):
