@@ -53,8 +53,7 @@ typedef enum gs_algo {
   GS_ALGO_PREFILL = 2,  /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
   GS_ALGO_PREFILL_DENSE = 3  /* tcgen05 kernel over zero-filled 256-row windows: tensor
                                 work of the dense layer, no gather; 1 x 128 and 1 x 256
-                                groups; GS_ALGO_AUTO picks it at T >= 1024 for 1 x 128
-                                and for 1 x 256 layers with out >= 2 in                */
+                                groups; GS_ALGO_AUTO picks it for T >= 1024           */
 } gs_algo;
 
 typedef struct gs_packed gs_packed;   /* opaque, library-owned */

@@ -20,7 +20,12 @@
 // warps 5..8 epilogue, warp 9 forwarder, warp 10 x producer (TMA).  W slots
 // and x slots are two rings: the W ring (nine 16 KB slots) runs three times as
 // deep as the x ring (three), because a W slot's round trip (copies landing,
-// fences, arrival at the leader) is about three times a TMA's.  Producers never wait for their own copies: each thread's copies
+// fences, arrival at the leader) is about three times a TMA's.  Stage k's
+// readiness (both forwarders, both CTAs' x bytes) and completion are one
+// barrier each, indexed by its W slot: the single MMA-issuing thread spends
+// most of a stage on its own instructions (about 40 ns per MMA, 50 per commit
+// and 60 per wait), so one wait and one commit per stage instead of two each
+// is worth ~9 % on the 13824 x 5120 layer.  Producers never wait for their own copies: each thread's copies
 // of a stage signal a local barrier (cp.async.mbarrier.arrive), and the
 // forwarder, once all have landed, fences them to the async proxy and arrives
 // on the leader's full barrier.  Every wait is bounded.
@@ -138,11 +143,11 @@ template <int KW, int SQ>
 __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_constant__ DParams P) {
   constexpr int kSlabs = KW / kDSlabK;   // stages per chunk
   extern __shared__ uint8_t d_smem_raw[];
-  __shared__ __align__(8) uint64_t xfull_bar[kDXStages];    // leader: both CTAs' x bytes
-  __shared__ __align__(8) uint64_t xempty_bar[kDXStages];
+  // Stage k uses W slot k % kDWStages and x slot k % kDXStages; one barrier of
+  // each kind per W slot, so the MMA thread waits once and commits once a stage.
+  __shared__ __align__(8) uint64_t full_bar[kDWStages];     // leader: both forwarders + both CTAs' x bytes
+  __shared__ __align__(8) uint64_t done_bar[kDWStages];     // the stage's MMAs completed (both CTAs)
   __shared__ __align__(8) uint64_t wfull_bar[kDWStages];    // local: this CTA's producer threads' copies
-  __shared__ __align__(8) uint64_t wready_bar[kDWStages];   // leader: both CTAs' forwarders
-  __shared__ __align__(8) uint64_t wempty_bar[kDWStages];
   __shared__ __align__(8) uint64_t afull_bar[kDAccBufs];
   __shared__ __align__(8) uint64_t aempty_bar[kDAccBufs];
   __shared__ __align__(8) uint64_t drain_bar;
@@ -156,14 +161,10 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   static_assert((kDMmaWarp + 3) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kDXStages; ++s) {
-      mbar_init(&xfull_bar[s], 1);   // the leader's expect-tx of both CTAs' x bytes
-      mbar_init(&xempty_bar[s], 1);
-    }
     for (int s = 0; s < kDWStages; ++s) {
+      mbar_init(&full_bar[s], 2 + 1);   // both CTAs' forwarders + the leader's expect-tx of the x bytes
+      mbar_init(&done_bar[s], 1);
       mbar_init(&wfull_bar[s], kDProdWarps * 32);
-      mbar_init(&wready_bar[s], 2);
-      mbar_init(&wempty_bar[s], 1);
     }
     for (int b = 0; b < kDAccBufs; ++b) {
       mbar_init(&afull_bar[b], 1);
@@ -266,7 +267,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
           for (int sl = 0; sl < kSlabs && ok; ++sl) {
             bool got = true;
             if (lane == 0)
-              got = mbar_wait_bounded(&wempty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
+              got = mbar_wait_bounded(&done_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
             if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
               ok = false;
               break;
@@ -294,7 +295,9 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     __syncwarp();
   } else if (warp == kDXWarp) {
     // ------------------------------------------------------------ x producer
-    uint32_t stage = 0, phase = 0;
+    // Stage k's x box goes to x slot k % kDXStages once stage k - kDXStages is
+    // done, and completes on the leader's full barrier of W slot k % kDWStages.
+    uint32_t k = 0;
     uint32_t armed = 0u, armed_par = 0u;
     bool ok = true;
     for (int u = pair; u < n_tiles && ok; u += n_pairs) {
@@ -307,21 +310,21 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
         if (lane == 0) {
           for (int it = 0; it < n_it && ok; ++it) {
             const int c = ibuf[it];
-            for (int sl = 0; sl < kSlabs && ok; ++sl) {
-              if (!mbar_wait_bounded(&xempty_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs,
-                                     kDevErrTimeout)) {
-                ok = false;
-                break;
+            for (int sl = 0; sl < kSlabs && ok; ++sl, ++k) {
+              if (k >= (uint32_t)kDXStages) {
+                const uint32_t kp = k - kDXStages;   // the stage whose x slot this one reuses
+                if (!mbar_wait_bounded(&done_bar[kp % kDWStages], (kp / kDWStages) & 1u, abort_flag, P.err,
+                                       kDWaitLimitNs, kDevErrTimeout)) {
+                  ok = false;
+                  break;
+                }
               }
-              if (rank == 0) mbar_arrive_expect_tx(&xfull_bar[stage], 2u * kDXBytes);
-              tma_load_3d_pair(smem + stage * kDXBytes, &L.xmap, mapa_shared(smem_u32(&xfull_bar[stage]), 0), 0,
-                               tok0, c * kSlabs + sl);
-              armed |= 1u << stage;
-              armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
-              if (++stage == (uint32_t)kDXStages) {
-                stage = 0;
-                phase ^= 1u;
-              }
+              const uint32_t fs = k % kDWStages;
+              if (rank == 0) mbar_arrive_expect_tx(&full_bar[fs], 2u * kDXBytes);
+              tma_load_3d_pair(smem + (k % kDXStages) * kDXBytes, &L.xmap, mapa_shared(smem_u32(&full_bar[fs]), 0),
+                               0, tok0, c * kSlabs + sl);
+              armed |= 1u << fs;
+              armed_par = (armed_par & ~(1u << fs)) | (((k / kDWStages) & 1u) << fs);
             }
           }
         }
@@ -330,10 +333,10 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     }
     if (lane == 0 && !ok && rank == 0) {
       // let the x copies in flight land before the CTA winds down
-      for (int s = 0; s < kDXStages; ++s) {
+      for (int s = 0; s < kDWStages; ++s) {
         if (!((armed >> s) & 1u)) continue;
         const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait_acq_cluster(&xfull_bar[s], (armed_par >> s) & 1u))
+        while (!mbar_try_wait_acq_cluster(&full_bar[s], (armed_par >> s) & 1u))
           if (globaltimer_ns() - t0 > kDDrainLimitNs) break;
       }
     }
@@ -367,7 +370,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             fence_proxy_async_cta();
             fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
             for (int i = 0; i < cnt; ++i) {
-              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&wready_bar[stage]), 0));
+              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage]), 0));
               if (++stage == (uint32_t)kDWStages) {
                 stage = 0;
                 phase ^= 1u;
@@ -381,7 +384,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     }
   } else if (warp == kDMmaWarp && rank == 0) {
     // ------------------------------------------------------------ MMA issuer (leader)
-    uint32_t ws = 0, wph = 0, xs = 0, xph = 0;   // W and x ring positions
+    uint32_t ws = 0, wph = 0, xs = 0;   // W slot (and its barriers' phase), x slot
     int buf = 0;
     uint32_t ae_ph = 0u;
     bool ok = true;
@@ -402,8 +405,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
         const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         if (lane == 0) {
           for (int it = 0; it < n_it * kSlabs && ok; ++it) {
-            if (!mbar_wait_bounded_cluster(&wready_bar[ws], wph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout) ||
-                !mbar_wait_bounded_cluster(&xfull_bar[xs], xph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
+            if (!mbar_wait_bounded_cluster(&full_bar[ws], wph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
               ok = false;
               break;
             }
@@ -415,16 +417,12 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
               mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
                                (first && kk == 0) ? 0u : 1u);
             first = false;
-            mma_commit_pair_mc(&wempty_bar[ws], 0x3);
-            mma_commit_pair_mc(&xempty_bar[xs], 0x3);
+            mma_commit_pair_mc(&done_bar[ws], 0x3);
             if (++ws == (uint32_t)kDWStages) {
               ws = 0;
               wph ^= 1u;
             }
-            if (++xs == (uint32_t)kDXStages) {
-              xs = 0;
-              xph ^= 1u;
-            }
+            if (++xs == (uint32_t)kDXStages) xs = 0;
           }
         }
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -548,15 +546,13 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 
 }  // namespace
 
-// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes, T = 2048):
-// with 1 x 128 groups this kernel takes 0.71-0.79x the gathering kernel's time
-// (0.88x on the 13824 x 5120 layer at T = 512, more on smaller layers at
-// T <= 512); with 1 x 256 groups 0.91-0.96x on the MLP up / gate shapes
-// (out > 2 in) and 1.01-1.03x on the square and down shapes.  Both kernels'
-// times hardly depend on the density.
+// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes): at
+// T = 2048 this kernel takes 0.70-0.80x the gathering kernel's time with
+// 1 x 128 groups and 0.83-0.93x with 1 x 256 groups; at T = 512 0.88x (1 x 128)
+// and 0.99x (1 x 256) on the 13824 x 5120 layer, more on smaller ones.  Both
+// kernels' times hardly depend on the density.
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
-  if (p->kept == 0 || T < 1024) return false;
-  return p->g_in == 128 || (p->g_in == 256 && p->out >= 2 * p->in);
+  return p->kept > 0 && T >= 1024 && (p->g_in == 128 || p->g_in == 256);
 }
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
