@@ -739,10 +739,10 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
     }
     // Small tiles: the zero-filled-window tensor-core kernel (dense-layer tensor
     // work, no per-column-block handshake) is the faster one; it takes the
-    // layers whose input is whole 64-column slabs, the others stay below
+    // layers whose input is whole 128-column items, the others stay below
     if (g <= kSqDenseMaxG) {
       std::vector<int> dense, rest;
-      for (int i : o) (ps[i]->in % 64 == 0 ? dense : rest).push_back(i);
+      for (int i : o) (ps[i]->in % 128 == 0 ? dense : rest).push_back(i);
       if (!dense.empty()) {
         const gs_status st = launch_prefill_dense(xs, ps, (int)dense.size(), T, ys, s, dense.data());
         if (st != GS_OK) return st;

@@ -18,14 +18,17 @@
 // producers (warp-cooperative 16-byte cp.async of the window's rows, zero-filled
 // for pruned rows), warp 4 TMEM allocator + single-thread MMA issuer (leader),
 // warps 5..8 epilogue, warp 9 forwarder, warp 10 x producer (TMA).  W slots
-// and x slots are two rings: the W ring (nine 16 KB slots) runs three times as
-// deep as the x ring (three), because a W slot's round trip (copies landing,
-// fences, arrival at the leader) is about three times a TMA's.  Stage k's
-// readiness (both forwarders, both CTAs' x bytes) and completion are one
-// barrier each, indexed by its W slot: the single MMA-issuing thread spends
+// and x slots are two rings: the W ring (ten 16 KB slots) runs deeper than
+// the x ring (four), because a W slot's round trip (copies landing,
+// fences, arrival at the leader) is about three times a TMA's.  Two
+// consecutive stages share one readiness barrier (both forwarders, both CTAs'
+// x bytes) and one completion barrier: the single MMA-issuing thread spends
 // most of a stage on its own instructions (about 40 ns per MMA, 50 per commit
-// and 60 per wait), so one wait and one commit per stage instead of two each
-// is worth ~9 % on the 13824 x 5120 layer.  Producers never wait for their own copies: each thread's copies
+// and 60 per wait), so one wait and one commit per stage pair (eight MMAs)
+// instead of two of each per stage took the 13824 x 5120 layer from 1120 to
+// ~1220 dense-equivalent TFLOP/s (1 x 256) and 1 x 128 groups from 0.283 to
+// 0.232 ms.  Every item therefore has an even number of stages (square groups
+// use 128-column items, two slabs with their own tile lookups).  Producers never wait for their own copies: each thread's copies
 // of a stage signal a local barrier (cp.async.mbarrier.arrive), and the
 // forwarder, once all have landed, fences them to the async proxy and arrives
 // on the leader's full barrier.  Every wait is bounded.
@@ -49,10 +52,12 @@ constexpr int kDSlabK = 64;                       // k per stage (one 128-byte s
 constexpr int kDXBytes = kDM * kDSlabK * 2;       // 16 KB of x per stage
 constexpr int kDWBytes = kDHalf * kDSlabK * 2;    // 16 KB of W rows per stage
 // Two rings: W slots (the long round trip: copies landing, forwarder fences,
-// arrival at the leader) run three times as deep as x slots (TMA); measured
-// 9 / 3 ahead of 8 / 4, 7 / 5 and 10 / 2.
-constexpr int kDWStages = 9;
-constexpr int kDXStages = 3;
+// arrival at the leader) run deeper than x slots (TMA); with single stages 9 / 3
+// measured ahead of 8 / 4, 7 / 5 and 10 / 2; with stage pairs both counts are
+// even and the shared memory (224 KB) is used up.
+constexpr int kDWStages = 10;                    // 160 KB
+constexpr int kDXStages = 4;                     // 64 KB
+constexpr int kDSuper = kDWStages / 2;          // pairs of consecutive stages share their barriers
 constexpr int kDXRing = kDXStages * kDXBytes;     // 64 KB at offset 0
 constexpr int kDWRing = kDWStages * kDWBytes;     // 128 KB after it
 constexpr int kDProdWarps = 4;                   // warps that copy W rows
@@ -111,7 +116,7 @@ __device__ __forceinline__ void fence_proxy_async_cta() {
 }
 
 // Chunks c0 .. c0 + 31 with at least one kept row in window w, in order, into
-// buf (square groups: every 64-column slab)
+// buf (square groups: every 128-column item)
 template <int SQ>
 __device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane, int* buf) {
   const int c = c0 + lane;
@@ -137,16 +142,17 @@ __device__ __forceinline__ uint32_t d_pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// KW: chunk width (1 x KW groups; 64 for square groups, one slab per item);
+// KW: chunk width (1 x KW groups; 128 for square groups: items of two slabs);
 // SQ: 0, or g for square g x g groups
 template <int KW, int SQ>
 __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_constant__ DParams P) {
   constexpr int kSlabs = KW / kDSlabK;   // stages per chunk
+  static_assert(kSlabs % 2 == 0 && kDWStages % 2 == 0 && kDXStages % 2 == 0, "stages go in pairs");
   extern __shared__ uint8_t d_smem_raw[];
   // Stage k uses W slot k % kDWStages and x slot k % kDXStages; one barrier of
   // each kind per W slot, so the MMA thread waits once and commits once a stage.
-  __shared__ __align__(8) uint64_t full_bar[kDWStages];     // leader: both forwarders + both CTAs' x bytes
-  __shared__ __align__(8) uint64_t done_bar[kDWStages];     // the stage's MMAs completed (both CTAs)
+  __shared__ __align__(8) uint64_t full_bar[kDSuper];       // leader: both forwarders + both CTAs' x bytes, two stages
+  __shared__ __align__(8) uint64_t done_bar[kDSuper];       // the two stages' MMAs completed (both CTAs)
   __shared__ __align__(8) uint64_t wfull_bar[kDWStages];    // local: this CTA's producer threads' copies
   __shared__ __align__(8) uint64_t afull_bar[kDAccBufs];
   __shared__ __align__(8) uint64_t aempty_bar[kDAccBufs];
@@ -161,11 +167,11 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   static_assert((kDMmaWarp + 3) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kDWStages; ++s) {
-      mbar_init(&full_bar[s], 2 + 1);   // both CTAs' forwarders + the leader's expect-tx of the x bytes
+    for (int s = 0; s < kDSuper; ++s) {
+      mbar_init(&full_bar[s], 2 * (2 + 1));   // per stage: both CTAs' forwarders + the leader's expect-tx
       mbar_init(&done_bar[s], 1);
-      mbar_init(&wfull_bar[s], kDProdWarps * 32);
     }
+    for (int s = 0; s < kDWStages; ++s) mbar_init(&wfull_bar[s], kDProdWarps * 32);
     for (int b = 0; b < kDAccBufs; ++b) {
       mbar_init(&afull_bar[b], 1);
       mbar_init(&aempty_bar[b], 2 * kDEpiWarps);
@@ -213,36 +219,42 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
           wo[q] = L.win_off16[(int64_t)c * (L.nw16 + 1) + b16];
         }
       };
-      // square: packed tile of each piece this lane copies in slab c (its row's
-      // block row, its columns' block column), issued one item ahead of use
-      auto load_tiles = [&](int c, int (&tv)[kCopies]) {
+      // square: packed tile of each piece this lane copies in each slab of item c
+      // (its row's block row, its columns' block column), loaded one item ahead
+      constexpr int kTS = SQ > 0 ? kSlabs : 1;   // slabs with their own tile lookups
+      auto load_tiles = [&](int c, int (&tv)[kTS][kCopies]) {
 #pragma unroll
-        for (int i = 0; i < kCopies; ++i) {
-          const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
-          const int k = c * kDSlabK + 8 * j;
-          tv[i] = row < L.out ? L.gtidx[(int64_t)(row / (SQ > 0 ? SQ : 1)) * L.Gin + k / (SQ > 0 ? SQ : 1)] : -1;
-        }
+        for (int sl = 0; sl < kTS; ++sl)
+#pragma unroll
+          for (int i = 0; i < kCopies; ++i) {
+            const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
+            const int k = c * KW + sl * kDSlabK + 8 * j;
+            tv[sl][i] = row < L.out ? L.gtidx[(int64_t)(row / (SQ > 0 ? SQ : 1)) * L.Gin + k / (SQ > 0 ? SQ : 1)] : -1;
+          }
       };
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
         const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         uint32_t km_n[kOwn];
         int wo_n[kOwn];
-        int tv_n[kCopies];
+        int tv_n[kTS][kCopies];
         if (n_it > 0) {
           if constexpr (SQ > 0) load_tiles(ibuf[0], tv_n);
           else load_meta(ibuf[0], km_n, wo_n);
         }
         for (int it = 0; it < n_it && ok; ++it) {
           const int c = ibuf[it];
-          // element offset of each piece this lane copies (slab 0 of the item), -1: zeros
-          int64_t soff[kCopies];
+          // element offset of each piece this lane copies (1 x KW: slab 0 of the
+          // item, the others follow at 64-element steps; square: per slab), -1: zeros
+          int64_t soff[kTS][kCopies];
           if constexpr (SQ > 0) {
 #pragma unroll
-            for (int i = 0; i < kCopies; ++i) {
-              const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
-              const int k = c * kDSlabK + 8 * j;
-              soff[i] = tv_n[i] >= 0 ? ((int64_t)tv_n[i] * SQ + row % SQ) * SQ + k % SQ : -1;
-            }
+            for (int sl = 0; sl < kTS; ++sl)
+#pragma unroll
+              for (int i = 0; i < kCopies; ++i) {
+                const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
+                const int k = c * KW + sl * kDSlabK + 8 * j;
+                soff[sl][i] = tv_n[sl][i] >= 0 ? ((int64_t)tv_n[sl][i] * SQ + row % SQ) * SQ + k % SQ : -1;
+              }
             if (it + 1 < n_it) load_tiles(ibuf[it + 1], tv_n);
           } else {
             // packed positions in chunk c of the rows this lane looks up (-1: pruned / beyond out)
@@ -260,14 +272,15 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             for (int i = 0; i < kCopies; ++i) {
               const int r = 4 * i + (lane >> 3);   // row within the warp's block: owner lane r % 32, slot r / 32
               const int pr = __shfl_sync(0xffffffffu, prow[r >> 5], r & 31);
-              soff[i] = pr >= 0 ? (int64_t)pr * KW + 8 * j : -1;
+              soff[0][i] = pr >= 0 ? (int64_t)pr * KW + 8 * j : -1;
             }
           }
-#pragma unroll 1
-          for (int sl = 0; sl < kSlabs && ok; ++sl) {
+#pragma unroll
+          for (int sl = 0; sl < kSlabs; ++sl) {
+            if (!ok) break;
             bool got = true;
             if (lane == 0)
-              got = mbar_wait_bounded(&done_bar[stage], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
+              got = mbar_wait_bounded(&done_bar[stage / 2], phase ^ 1u, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout);
             if (!__shfl_sync(0xffffffffu, got ? 1 : 0, 0)) {
               ok = false;
               break;
@@ -277,9 +290,10 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             for (int i = 0; i < kCopies; ++i) {
               const int rr = warp * kRows + 4 * i + (lane >> 3);
               const uint32_t dst = wb + (uint32_t)rr * 128u + (uint32_t)((j ^ (rr & 7)) << 4);   // 128-byte swizzle
-              const bool kept = soff[i] >= 0;
+              const int64_t so = soff[SQ > 0 ? sl : 0][i];
+              const bool kept = so >= 0;
               // a pruned row reads nothing (source size 0) and is filled with zeros
-              const uint16_t* src = kept ? L.tiles + soff[i] + sl * kDSlabK : L.tiles;
+              const uint16_t* src = kept ? L.tiles + so + (SQ > 0 ? 0 : sl * kDSlabK) : L.tiles;
               cp_async16_zfill(dst, src, kept ? 16u : 0u);
             }
             cp_async_arrive_noinc(&wfull_bar[stage]);   // fires once this thread's copies have landed
@@ -312,19 +326,19 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             const int c = ibuf[it];
             for (int sl = 0; sl < kSlabs && ok; ++sl, ++k) {
               if (k >= (uint32_t)kDXStages) {
-                const uint32_t kp = k - kDXStages;   // the stage whose x slot this one reuses
-                if (!mbar_wait_bounded(&done_bar[kp % kDWStages], (kp / kDWStages) & 1u, abort_flag, P.err,
+                const uint32_t pp = (k - kDXStages) / 2;   // the stage pair whose x slot this one reuses
+                if (!mbar_wait_bounded(&done_bar[pp % kDSuper], (pp / kDSuper) & 1u, abort_flag, P.err,
                                        kDWaitLimitNs, kDevErrTimeout)) {
                   ok = false;
                   break;
                 }
               }
-              const uint32_t fs = k % kDWStages;
+              const uint32_t fs = (k / 2) % kDSuper;
               if (rank == 0) mbar_arrive_expect_tx(&full_bar[fs], 2u * kDXBytes);
               tma_load_3d_pair(smem + (k % kDXStages) * kDXBytes, &L.xmap, mapa_shared(smem_u32(&full_bar[fs]), 0),
                                0, tok0, c * kSlabs + sl);
               armed |= 1u << fs;
-              armed_par = (armed_par & ~(1u << fs)) | (((k / kDWStages) & 1u) << fs);
+              armed_par = (armed_par & ~(1u << fs)) | (((k / 2 / kDSuper) & 1u) << fs);
             }
           }
         }
@@ -333,7 +347,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     }
     if (lane == 0 && !ok && rank == 0) {
       // let the x copies in flight land before the CTA winds down
-      for (int s = 0; s < kDWStages; ++s) {
+      for (int s = 0; s < kDSuper; ++s) {
         if (!((armed >> s) & 1u)) continue;
         const uint64_t t0 = globaltimer_ns();
         while (!mbar_try_wait_acq_cluster(&full_bar[s], (armed_par >> s) & 1u))
@@ -370,7 +384,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             fence_proxy_async_cta();
             fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
             for (int i = 0; i < cnt; ++i) {
-              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage]), 0));
+              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage / 2]), 0));
               if (++stage == (uint32_t)kDWStages) {
                 stage = 0;
                 phase ^= 1u;
@@ -404,25 +418,31 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
         const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         if (lane == 0) {
-          for (int it = 0; it < n_it * kSlabs && ok; ++it) {
-            if (!mbar_wait_bounded_cluster(&full_bar[ws], wph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
+          // stages two at a time (every item has an even number of them)
+          for (int it = 0; it < n_it * kSlabs && ok; it += 2) {
+            if (!mbar_wait_bounded_cluster(&full_bar[ws / 2], wph, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint64_t ad = sdesc_sw128(smem_u32(smem + xs * kDXBytes));
-            const uint64_t bd = sdesc_sw128(smem_u32(smem + kDXRing + ws * kDWBytes));
 #pragma unroll
-            for (int kk = 0; kk < kDSlabK / 16; ++kk)
-              mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
-                               (first && kk == 0) ? 0u : 1u);
+            for (int h = 0; h < 2; ++h) {
+              const uint64_t ad = sdesc_sw128(smem_u32(smem + (xs + h) * kDXBytes));
+              const uint64_t bd = sdesc_sw128(smem_u32(smem + kDXRing + (ws + h) * kDWBytes));
+#pragma unroll
+              for (int kk = 0; kk < kDSlabK / 16; ++kk)
+                mma_bf16_ss_pair(d, ad + (uint64_t)(2 * kk), bd + (uint64_t)(2 * kk), idesc,
+                                 (first && h == 0 && kk == 0) ? 0u : 1u);
+            }
             first = false;
-            mma_commit_pair_mc(&done_bar[ws], 0x3);
-            if (++ws == (uint32_t)kDWStages) {
+            mma_commit_pair_mc(&done_bar[ws / 2], 0x3);
+            ws += 2;
+            if (ws == (uint32_t)kDWStages) {
               ws = 0;
               wph ^= 1u;
             }
-            if (++xs == (uint32_t)kDXStages) xs = 0;
+            xs += 2;
+            if (xs == (uint32_t)kDXStages) xs = 0;
           }
         }
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
@@ -586,10 +606,10 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
       L.y = static_cast<uint16_t*>(ys[i]);
       L.out = (int32_t)p->out;
       if (sq) {
-        if (p->in % kDSlabK != 0) return GS_ERR_UNSUPPORTED;
+        if (p->in % 128 != 0) return GS_ERR_UNSUPPORTED;
         L.gtidx = p->gtidx;
         L.Gin = p->G;
-        L.G = (int32_t)(p->in / kDSlabK);
+        L.G = (int32_t)(p->in / 128);   // 128-column items (two 64-column stages)
       } else {
         L.win_off16 = p->win_off16;
         L.kmask16 = p->kmask16;
@@ -617,9 +637,9 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = sq == 16   ? d_launch<kDSlabK, 16>(cfg, P)
-                          : sq == 32 ? d_launch<kDSlabK, 32>(cfg, P)
-                          : sq == 64 ? d_launch<kDSlabK, 64>(cfg, P)
+    const cudaError_t e = sq == 16   ? d_launch<128, 16>(cfg, P)
+                          : sq == 32 ? d_launch<128, 32>(cfg, P)
+                          : sq == 64 ? d_launch<128, 64>(cfg, P)
                           : kw == 256 ? d_launch<256, 0>(cfg, P)
                                       : d_launch<128, 0>(cfg, P);
     note_launch();
