@@ -17,7 +17,8 @@
 // Roles (one CTA per SM, units persistent over the pairs): warps 0..3
 // producers (warp-cooperative 16-byte cp.async of the window's rows, zero-filled
 // for pruned rows), warp 4 TMEM allocator + single-thread MMA issuer (leader),
-// warps 5..8 epilogue, warp 9 forwarder, warp 10 x producer (TMA).  W slots
+// warps 5..8 epilogue, warps 9 and 11 forwarders (alternate stage pairs),
+// warp 10 x producer (TMA).  W slots
 // and x slots are two rings: the W ring (ten 16 KB slots) runs deeper than
 // the x ring (four), because a W slot's round trip (copies landing,
 // fences, arrival at the leader) is about three times a TMA's.  Two
@@ -27,7 +28,8 @@
 // and 60 per wait), so one wait and one commit per stage pair (eight MMAs)
 // instead of two of each per stage took the 13824 x 5120 layer from 1120 to
 // ~1220 dense-equivalent TFLOP/s (1 x 256) and 1 x 128 groups from 0.283 to
-// 0.232 ms.  Every item therefore has an even number of stages (square groups
+// 0.232 ms; a second forwarder (the fences of one batch take about a
+// microsecond, which one forwarder could no longer hide) then took it to 1440.  Every item therefore has an even number of stages (square groups
 // use 128-column items, two slabs with their own tile lookups).  Producers never wait for their own copies: each thread's copies
 // of a stage signal a local barrier (cp.async.mbarrier.arrive), and the
 // forwarder, once all have landed, fences them to the async proxy and arrives
@@ -66,7 +68,8 @@ constexpr int kDEpiWarp0 = kDProdWarps + 1;
 constexpr int kDEpiWarps = 4;
 constexpr int kDFwdWarp = kDEpiWarp0 + kDEpiWarps;
 constexpr int kDXWarp = kDFwdWarp + 1;            // x TMA producer
-constexpr int kDThreads = (kDXWarp + 1) * 32;
+constexpr int kDFwdWarp2 = kDXWarp + 1;           // second forwarder (odd stage pairs)
+constexpr int kDThreads = (kDFwdWarp2 + 1) * 32;
 constexpr int kDAccBufs = 2;
 constexpr uint32_t kDTmemCols = kDAccBufs * kDW;  // 512
 constexpr int kDMaxLayers = 8;
@@ -162,9 +165,12 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(d_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs)
-  int* ibuf = reinterpret_cast<int*>(smem + kDXRing + kDWRing) +
-              (warp <= kDMmaWarp ? warp : warp == kDFwdWarp ? kDMmaWarp + 1 : warp == kDXWarp ? kDMmaWarp + 2 : 0) * 32;
-  static_assert((kDMmaWarp + 3) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
+  const int ib_slot = warp <= kDMmaWarp ? warp
+                      : warp == kDFwdWarp ? kDMmaWarp + 1
+                      : warp == kDXWarp   ? kDMmaWarp + 2
+                      : warp == kDFwdWarp2 ? kDMmaWarp + 3 : 0;
+  int* ibuf = reinterpret_cast<int*>(smem + kDXRing + kDWRing) + ib_slot * 32;
+  static_assert((kDMmaWarp + 4) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDSuper; ++s) {
@@ -355,45 +361,51 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       }
     }
     __syncwarp();
-  } else if (warp == kDFwdWarp) {
-    // ------------------------------------------------------------ forwarder
-    // Once all of this CTA's producer threads' copies of a stage have landed,
-    // make them visible to the tensor cores (async proxy) and tell the leader.
-    uint32_t stage = 0, phase = 0;
+  } else if (warp == kDFwdWarp || warp == kDFwdWarp2) {
+    // ------------------------------------------------------------ forwarders
+    // Once all of this CTA's producer threads' copies of a stage pair have
+    // landed, make them visible to the tensor cores (async proxy) and tell the
+    // leader.  Two forwarders take alternate stage pairs, so that their fences
+    // (about a microsecond per batch) overlap.
+    const uint32_t f = warp == kDFwdWarp ? 0u : 1u;
+    uint32_t K = 0;   // stages before the current batch
     bool ok = true;
     for (int u = pair; u < n_tiles && ok; u += n_pairs) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int w = (u - L.tile_begin) / L.n_m;
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
-        const int n_st = d_items<SQ>(L, w, c0, lane, ibuf) * kSlabs;
+        const int n_pr = d_items<SQ>(L, w, c0, lane, ibuf) * kSlabs / 2;   // stage pairs of the batch
         if (lane == 0) {
-          for (int k = 0; k < n_st && ok;) {
-            if (!mbar_wait_bounded(&wfull_bar[stage], phase, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
+          int cnt = 1;
+          for (int q = (int)(((K / 2) & 1u) == f ? 0u : 1u); q < n_pr && ok; q += 2 * cnt) {
+            const uint32_t p0 = K / 2 + (uint32_t)q;   // global pair index
+            const uint32_t s0 = (2 * p0) % kDWStages, ph0 = ((2 * p0) / kDWStages) & 1u;
+            if (!mbar_wait_bounded(&wfull_bar[s0], ph0, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout) ||
+                !mbar_wait_bounded(&wfull_bar[s0 + 1], ph0, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout)) {
               ok = false;
               break;
             }
-            // take every following stage that has landed too, so that one
-            // release fence covers them all (a release per stage is slow)
-            int cnt = 1;
-            while (k + cnt < n_st && cnt < kDWStages) {
-              const uint32_t s2 = (stage + (uint32_t)cnt) % kDWStages;
-              const uint32_t p2 = phase ^ ((stage + (uint32_t)cnt) >= (uint32_t)kDWStages ? 1u : 0u);
-              if (!mbar_try_wait(&wfull_bar[s2], p2)) break;
+            // take this forwarder's following pairs that have landed too, so that
+            // one release fence covers them all (a release per stage is slow)
+            cnt = 1;
+            while (q + 2 * cnt < n_pr && cnt < kDSuper / 2) {
+              const uint32_t p2 = p0 + 2 * (uint32_t)cnt;
+              const uint32_t s2 = (2 * p2) % kDWStages, ph2 = ((2 * p2) / kDWStages) & 1u;
+              if (!mbar_try_wait(&wfull_bar[s2], ph2) || !mbar_try_wait(&wfull_bar[s2 + 1], ph2)) break;
               ++cnt;
             }
             fence_proxy_async_cta();
             fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
             for (int i = 0; i < cnt; ++i) {
-              mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(&full_bar[stage / 2]), 0));
-              if (++stage == (uint32_t)kDWStages) {
-                stage = 0;
-                phase ^= 1u;
-              }
+              const uint32_t fs = (p0 + 2 * (uint32_t)i) % kDSuper;
+              const uint32_t fb = mapa_shared(smem_u32(&full_bar[fs]), 0);
+              mbar_arrive_cluster_relaxed(fb);   // one arrival per stage of the pair
+              mbar_arrive_cluster_relaxed(fb);
             }
-            k += cnt;
           }
         }
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        K += (uint32_t)(2 * n_pr);
       }
     }
   } else if (warp == kDMmaWarp && rank == 0) {
