@@ -57,7 +57,7 @@ constexpr uint32_t kSqTmemCols = kSqAccBufs * kSqWin;
 constexpr int kSqEpiWarps = 4;
 constexpr int kSqThreads = (2 + kSqEpiWarps) * 32;
 constexpr int kSqMaxLayers = 8;
-constexpr int kSqDenseMaxG = 32;          // above the decode regime, g <= this takes the zero-filled kernel
+constexpr int kSqDenseMaxG = 64;          // above the decode regime, g <= this takes the zero-filled kernel (7B block, T = 2048: 64x64 525 vs 476 TFLOP/s)
 constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R <= 8)
 constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
 constexpr uint64_t kSqDrainLimitNs = 200000000ull;

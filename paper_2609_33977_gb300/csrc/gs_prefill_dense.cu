@@ -17,8 +17,8 @@
 // Roles (one CTA per SM, units persistent over the pairs): warps 0..3
 // producers (warp-cooperative 16-byte cp.async of the window's rows, zero-filled
 // for pruned rows), warp 4 TMEM allocator + single-thread MMA issuer (leader),
-// warps 5..8 epilogue, warps 9 and 11 forwarders (alternate stage pairs),
-// warp 10 x producer (TMA).  W slots
+// warps 5..8 epilogue, warp 9 and warps 11.. forwarders (stage pairs taken in
+// turn), warp 10 x producer (TMA).  W slots
 // and x slots are two rings: the W ring (ten 16 KB slots) runs deeper than
 // the x ring (four), because a W slot's round trip (copies landing,
 // fences, arrival at the leader) is about three times a TMA's.  Two
@@ -68,8 +68,8 @@ constexpr int kDEpiWarp0 = kDProdWarps + 1;
 constexpr int kDEpiWarps = 4;
 constexpr int kDFwdWarp = kDEpiWarp0 + kDEpiWarps;
 constexpr int kDXWarp = kDFwdWarp + 1;            // x TMA producer
-constexpr int kDFwdWarp2 = kDXWarp + 1;           // second forwarder (odd stage pairs)
-constexpr int kDThreads = (kDFwdWarp2 + 1) * 32;
+constexpr int kDNumFwd = 2;                       // forwarders: warp kDFwdWarp, then kDXWarp + 1, ...
+constexpr int kDThreads = (kDXWarp + kDNumFwd) * 32;
 constexpr int kDAccBufs = 2;
 constexpr uint32_t kDTmemCols = kDAccBufs * kDW;  // 512
 constexpr int kDMaxLayers = 8;
@@ -121,7 +121,7 @@ __device__ __forceinline__ void fence_proxy_async_cta() {
 // Chunks c0 .. c0 + 31 with at least one kept row in window w, in order, into
 // buf (square groups: every 128-column item)
 template <int SQ>
-__device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane, int* buf) {
+__device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane, int16_t* buf) {
   const int c = c0 + lane;
   __syncwarp();   // every lane is done reading the previous batch
   bool ne = false;
@@ -135,7 +135,7 @@ __device__ __forceinline__ int d_items(const DLayer& L, int w, int c0, int lane,
     }
   }
   const uint32_t ballot = __ballot_sync(0xffffffffu, ne);
-  if (ne) buf[__popc(ballot & ((1u << lane) - 1u))] = c;
+  if (ne) buf[__popc(ballot & ((1u << lane) - 1u))] = (int16_t)c;
   __syncwarp();
   return __popc(ballot);
 }
@@ -165,12 +165,10 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(d_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();   // 0: leader (issues the pair's MMAs)
-  const int ib_slot = warp <= kDMmaWarp ? warp
-                      : warp == kDFwdWarp ? kDMmaWarp + 1
-                      : warp == kDXWarp   ? kDMmaWarp + 2
-                      : warp == kDFwdWarp2 ? kDMmaWarp + 3 : 0;
-  int* ibuf = reinterpret_cast<int*>(smem + kDXRing + kDWRing) + ib_slot * 32;
-  static_assert((kDMmaWarp + 4) * 32 * 4 <= kDIbufBytes, "chunk lists fit");
+  // chunk lists of d_items (producers, MMA issuer, x producer, forwarders)
+  const int ib_slot = warp <= kDMmaWarp ? warp : warp == kDFwdWarp ? kDMmaWarp + 1 : warp >= kDXWarp ? warp - kDXWarp + kDMmaWarp + 2 : 0;
+  int16_t* ibuf = reinterpret_cast<int16_t*>(smem + kDXRing + kDWRing) + ib_slot * 32;
+  static_assert((kDMmaWarp + 2 + kDNumFwd) * 32 * 2 <= kDIbufBytes, "chunk lists fit");
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDSuper; ++s) {
@@ -361,13 +359,13 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       }
     }
     __syncwarp();
-  } else if (warp == kDFwdWarp || warp == kDFwdWarp2) {
+  } else if (warp == kDFwdWarp || warp > kDXWarp) {
     // ------------------------------------------------------------ forwarders
     // Once all of this CTA's producer threads' copies of a stage pair have
     // landed, make them visible to the tensor cores (async proxy) and tell the
-    // leader.  Two forwarders take alternate stage pairs, so that their fences
-    // (about a microsecond per batch) overlap.
-    const uint32_t f = warp == kDFwdWarp ? 0u : 1u;
+    // leader.  The forwarders take the stage pairs in turn, so that their
+    // fences (about a microsecond per batch) overlap.
+    const uint32_t f = warp == kDFwdWarp ? 0u : (uint32_t)(warp - kDXWarp);   // takes pairs p with p % kDNumFwd == f
     uint32_t K = 0;   // stages before the current batch
     bool ok = true;
     for (int u = pair; u < n_tiles && ok; u += n_pairs) {
@@ -377,7 +375,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
         const int n_pr = d_items<SQ>(L, w, c0, lane, ibuf) * kSlabs / 2;   // stage pairs of the batch
         if (lane == 0) {
           int cnt = 1;
-          for (int q = (int)(((K / 2) & 1u) == f ? 0u : 1u); q < n_pr && ok; q += 2 * cnt) {
+          for (int q = (int)((f + kDNumFwd - (K / 2) % kDNumFwd) % kDNumFwd); q < n_pr && ok; q += kDNumFwd * cnt) {
             const uint32_t p0 = K / 2 + (uint32_t)q;   // global pair index
             const uint32_t s0 = (2 * p0) % kDWStages, ph0 = ((2 * p0) / kDWStages) & 1u;
             if (!mbar_wait_bounded(&wfull_bar[s0], ph0, abort_flag, P.err, kDWaitLimitNs, kDevErrTimeout) ||
@@ -388,8 +386,8 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             // take this forwarder's following pairs that have landed too, so that
             // one release fence covers them all (a release per stage is slow)
             cnt = 1;
-            while (q + 2 * cnt < n_pr && cnt < kDSuper / 2) {
-              const uint32_t p2 = p0 + 2 * (uint32_t)cnt;
+            while (q + kDNumFwd * cnt < n_pr && cnt * kDNumFwd < kDSuper) {
+              const uint32_t p2 = p0 + kDNumFwd * (uint32_t)cnt;
               const uint32_t s2 = (2 * p2) % kDWStages, ph2 = ((2 * p2) / kDWStages) & 1u;
               if (!mbar_try_wait(&wfull_bar[s2], ph2) || !mbar_try_wait(&wfull_bar[s2 + 1], ph2)) break;
               ++cnt;
@@ -397,7 +395,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
             fence_proxy_async_cta();
             fence_acq_rel_cluster();   // with the relaxed arrives below: a release of the copies to the leader
             for (int i = 0; i < cnt; ++i) {
-              const uint32_t fs = (p0 + 2 * (uint32_t)i) % kDSuper;
+              const uint32_t fs = (p0 + kDNumFwd * (uint32_t)i) % kDSuper;
               const uint32_t fb = mapa_shared(smem_u32(&full_bar[fs]), 0);
               mbar_arrive_cluster_relaxed(fb);   // one arrival per stage of the pair
               mbar_arrive_cluster_relaxed(fb);
@@ -578,13 +576,15 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 
 }  // namespace
 
-// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes): at
-// T = 2048 this kernel takes 0.70-0.80x the gathering kernel's time with
-// 1 x 128 groups and 0.83-0.93x with 1 x 256 groups; at T = 512 0.88x (1 x 128)
-// and 0.99x (1 x 256) on the 13824 x 5120 layer, more on smaller ones.  Both
-// kernels' times hardly depend on the density.
+// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes, time
+// relative to the gathering kernel): 1 x 128 groups 0.47-0.95x at every T from
+// 256 to 2048; 1 x 256 groups 0.66-0.92x from T = 768 up, while at T <= 512
+// only the 13824 x 5120 layer gains (0.73-0.85x) and the smaller ones lose
+// (1.12-1.24x: too few 256 x 256 units for the CTA pairs).  Both kernels' times
+// hardly depend on the density.
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
-  return p->kept > 0 && T >= 1024 && (p->g_in == 128 || p->g_in == 256);
+  if (p->kept == 0 || p->g_out != 1) return false;
+  return (p->g_in == 128 && T > 128) || (p->g_in == 256 && T >= 768);
 }
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
@@ -628,6 +628,7 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
         L.G = p->G;
         L.nw16 = p->nw16;
       }
+      if (L.G > 32767) return GS_ERR_UNSUPPORTED;   // chunk lists hold 16-bit indices
       L.n_m = (int32_t)((T + 2 * kDM - 1) / (2 * kDM));
       L.tile_begin = (int32_t)tiles;
       tiles += (int64_t)L.n_m * ((p->out + kDW - 1) / kDW);
