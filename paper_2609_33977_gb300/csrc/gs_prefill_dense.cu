@@ -226,21 +226,24 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
       // square: packed tile of each piece this lane copies in each slab of item c
       // (its row's block row, its columns' block column), loaded one item ahead
       constexpr int kTS = SQ > 0 ? kSlabs : 1;   // slabs with their own tile lookups
-      auto load_tiles = [&](int c, int (&tv)[kTS][kCopies]) {
+      // a warp's 32 rows lie in one block row (g >= 32) or two (g = 16): one
+      // lookup per block row and slab; copy i uses block row kU * i / kCopies
+      constexpr int kU = SQ == 16 ? 2 : 1;
+      auto load_tiles = [&](int c, int (&tv)[kTS][kU]) {
 #pragma unroll
         for (int sl = 0; sl < kTS; ++sl)
 #pragma unroll
-          for (int i = 0; i < kCopies; ++i) {
-            const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
+          for (int q = 0; q < kU; ++q) {
+            const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 16 * q;   // first row of the block row part
             const int k = c * KW + sl * kDSlabK + 8 * j;
-            tv[sl][i] = row < L.out ? L.gtidx[(int64_t)(row / (SQ > 0 ? SQ : 1)) * L.Gin + k / (SQ > 0 ? SQ : 1)] : -1;
+            tv[sl][q] = row < L.out ? L.gtidx[(int64_t)(row / (SQ > 0 ? SQ : 1)) * L.Gin + k / (SQ > 0 ? SQ : 1)] : -1;
           }
       };
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
         const int n_it = d_items<SQ>(L, w, c0, lane, ibuf);
         uint32_t km_n[kOwn];
         int wo_n[kOwn];
-        int tv_n[kTS][kCopies];
+        int tv_n[kTS][kU];
         if (n_it > 0) {
           if constexpr (SQ > 0) load_tiles(ibuf[0], tv_n);
           else load_meta(ibuf[0], km_n, wo_n);
@@ -257,7 +260,8 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
               for (int i = 0; i < kCopies; ++i) {
                 const int row = w * kDW + (int)rank * kDHalf + warp * kRows + 4 * i + (lane >> 3);
                 const int k = c * KW + sl * kDSlabK + 8 * j;
-                soff[sl][i] = tv_n[sl][i] >= 0 ? ((int64_t)tv_n[sl][i] * SQ + row % SQ) * SQ + k % SQ : -1;
+                const int tq = tv_n[sl][kU * i / kCopies];
+                soff[sl][i] = tq >= 0 ? ((int64_t)tq * SQ + row % SQ) * SQ + k % SQ : -1;
               }
             if (it + 1 < n_it) load_tiles(ibuf[it + 1], tv_n);
           } else {
