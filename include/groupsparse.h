@@ -359,8 +359,9 @@ gs_status gs_masked_linear_backward(const void* x_dev, const void* W_dev, const 
  * allocated.
  *
  * gs_debug_inject_wait(family, limit_ns) - the next launch of that kernel
- * family (GS_ALGO_DECODE or GS_ALGO_PREFILL) makes its first CTA (the first
- * CTA pair for prefill) wait, before issuing any copy or tensor-core work, on
+ * family (GS_ALGO_DECODE, GS_ALGO_PREFILL or GS_ALGO_PREFILL_DENSE) makes its
+ * first CTA (the first CTA pair for the tensor-core kernels) wait, before
+ * issuing any copy or tensor-core work, on
  * a library word that nothing ever sets, for at most limit_ns (<= 1 s).  The
  * wait runs out, the kernel records GS_ERR_DEVICE_TIMEOUT and that CTA skips
  * its work; the other CTAs finish theirs.  One-shot; limit_ns = 0 disarms.

@@ -19,7 +19,7 @@ std::atomic<int64_t> g_launches{0};
 std::atomic<uint64_t> g_timeout_epoch{0};
 // test hooks: countdown to a failing allocation (0 = off), injected wait limits
 std::atomic<int64_t> g_fail_alloc_in{0};
-std::atomic<uint64_t> g_inject_ns[3] = {{0}, {0}, {0}};
+std::atomic<uint64_t> g_inject_ns[4] = {{0}, {0}, {0}, {0}};
 
 // Token count at and above which gs_linear uses the tensor-core kernel.
 constexpr int64_t kPrefillMinTokens = 33;
@@ -103,7 +103,7 @@ gs_status lib_malloc(void** ptr, size_t bytes) {
 }
 
 uint64_t take_injected_wait(int family) {
-  if (family < 1 || family > 2) return 0;
+  if (family < GS_ALGO_DECODE || family > GS_ALGO_PREFILL_DENSE) return 0;
   return g_inject_ns[family].exchange(0);
 }
 
@@ -544,7 +544,8 @@ gs_status gs_debug_fail_alloc(int64_t nth) {
 }
 
 gs_status gs_debug_inject_wait(gs_algo family, uint64_t limit_ns) {
-  if (family != GS_ALGO_DECODE && family != GS_ALGO_PREFILL) return GS_ERR_INVALID_ARG;
+  if (family != GS_ALGO_DECODE && family != GS_ALGO_PREFILL && family != GS_ALGO_PREFILL_DENSE)
+    return GS_ERR_INVALID_ARG;
   if (limit_ns > 1000000000ull) return GS_ERR_INVALID_ARG;
   g_inject_ns[family].store(limit_ns);
   return GS_OK;

@@ -102,7 +102,8 @@ uint64_t timeout_epoch();
 // make the n-th one fail); OOM on cudaErrorMemoryAllocation, else CUDA.
 gs_status lib_malloc(void** ptr, size_t bytes);
 // Test hook: limit of a wait on the never-set word to inject into the next
-// launch of a kernel family (GS_ALGO_DECODE / GS_ALGO_PREFILL); 0 = none.
+// launch of a kernel family (GS_ALGO_DECODE / GS_ALGO_PREFILL /
+// GS_ALGO_PREFILL_DENSE); 0 = none.
 // Reading it disarms it.
 uint64_t take_injected_wait(int family);
 

@@ -95,6 +95,7 @@ struct DParams {
   DLayer L[kDMaxLayers];
   int32_t n_layers, T, n_tiles;
   int* err;
+  uint64_t inject_ns;   // test hook: CTA pair 0 first waits this long on a word nothing sets (0 = off)
 };
 
 __device__ __forceinline__ int d_layer_of(const DParams& P, int t) {
@@ -197,7 +198,29 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
   const int n_tiles = P.n_tiles;
   const int pair = (int)(blockIdx.x >> 1), n_pairs = (int)(gridDim.x >> 1);
 
-  if (warp < kDProdWarps) {
+  if (P.inject_ns != 0 && pair == 0) {
+    // test hook: before any copy or MMA is issued, a bounded wait on a word
+    // that nothing sets runs out in each CTA of pair 0; the pair then records
+    // the timeout and skips its units (every role, both CTAs)
+    if (threadIdx.x == 0) {
+      const volatile int* never = P.err + 1;
+      const uint64_t t0 = globaltimer_ns();
+      while (*never == 0) {
+        if (globaltimer_ns() - t0 > P.inject_ns) {
+          atomicExch(P.err, kDevErrTimeout);
+          abort_s = 1;
+          break;
+        }
+        __nanosleep(1000);
+      }
+    }
+    __syncthreads();
+  }
+  const bool injected_abort = pair == 0 && abort_s != 0;
+
+  if (injected_abort) {
+    // nothing was issued: go straight to the TMEM release
+  } else if (warp < kDProdWarps) {
     // ------------------------------------------------------------ producers
     // Warp v copies window rows v * kRows .. + kRows - 1 of this CTA's half,
     // warp-cooperatively: copy i moves rows v * kRows + 4 i .. + 3, eight
@@ -642,6 +665,7 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
     P.T = (int32_t)T;
     P.n_tiles = (int32_t)tiles;
     P.err = err;
+    P.inject_ns = b0 == 0 ? take_injected_wait(GS_ALGO_PREFILL_DENSE) : 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(2 * std::min<int64_t>(tiles, max_pairs)));
     cfg.blockDim = dim3(kDThreads);

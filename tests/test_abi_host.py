@@ -156,3 +156,5 @@ def test_debug_hooks_validate_arguments(lib):
     assert lib.gs_debug_inject_wait(0, 1000) == INVALID          # AUTO is not a kernel family
     assert lib.gs_debug_inject_wait(1, 2_000_000_000) == INVALID  # above 1 s
     assert lib.gs_debug_inject_wait(1, 0) == 0 and lib.gs_debug_inject_wait(2, 0) == 0
+    assert lib.gs_debug_inject_wait(3, 0) == 0                 # the zero-filled prefill kernel
+    assert lib.gs_debug_inject_wait(4, 1000) == INVALID        # no such family

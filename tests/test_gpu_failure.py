@@ -89,6 +89,34 @@ def test_prefill_wait_timeout_then_recovery(gs, T):
     assert gs.device_status() == gs.GS_OK
 
 
+@pytest.mark.parametrize("g", [0, 16])
+def test_prefill_dense_wait_timeout_then_recovery(gs, g):
+    # the zero-filled-window kernel: CTA pair 0 skips its units, then a clean launch matches the oracle
+    import torch
+    T = 300
+    if g == 0:
+        Wb, B, p = make(gs, 4096, 4096, 0.5, 75)
+        gg = None
+    else:
+        Wb = wl.random_weight_bits(1024, 2048, seed=76)
+        B = wl.random_mask(1024 // g, 2048 // g, 0.5, seed=77)
+        p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), g, g)
+        gg = g
+    xb = wl.random_activation_bits(T, Wb.shape[1], seed=78 + g)
+    x = to_dev(xb)
+    algo = gs.ALGO_PREFILL_DENSE if g == 0 else gs.ALGO_AUTO   # square 16x16 at T = 300: the same kernel
+    gs.debug_inject_wait(gs.ALGO_PREFILL_DENSE, 1_000_000)
+    gs.linear(x, p, algo=algo)
+    assert gs.device_status() == gs.GS_ERR_DEVICE_TIMEOUT
+    y = to_bits(gs.linear(x, p, algo=algo))
+    if gg is None:
+        assert_within_bound(y, xb, Wb, B, what="zero-filled prefill after timeout")
+    else:
+        yr, A = orc.linear(xb, Wb, B, gg, gg)
+        assert np.all(np.abs(wl.bf16_bits_to_f32(y).astype(np.float64) - yr) <= 2.0 ** -7 * A + 1e-6)
+    assert gs.device_status() == gs.GS_OK
+
+
 def test_failed_allocation_returns_oom_and_frees_everything(gs):
     import torch
     out, inp = 2048, 4096
