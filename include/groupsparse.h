@@ -53,8 +53,9 @@ typedef enum gs_algo {
   GS_ALGO_PREFILL = 2,  /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
   GS_ALGO_PREFILL_DENSE = 3  /* tcgen05 kernel over zero-filled 256-row windows: tensor
                                 work of the dense layer, no gather; 1 x 128 and 1 x 256
-                                groups; GS_ALGO_AUTO picks it for T > 128 (1 x 128)
-                                and T >= 768 (1 x 256)                                 */
+                                groups; GS_ALGO_AUTO picks it for T > 128 (1 x 128;
+                                1 x 256: from T = 768, or when the layer holds enough
+                                256 x 256 units to fill the GPU)                       */
 } gs_algo;
 
 typedef struct gs_packed gs_packed;   /* opaque, library-owned */

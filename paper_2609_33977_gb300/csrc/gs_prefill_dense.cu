@@ -609,9 +609,18 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 // only the 13824 x 5120 layer gains (0.73-0.85x) and the smaller ones lose
 // (1.12-1.24x: too few 256 x 256 units for the CTA pairs).  Both kernels' times
 // hardly depend on the density.
+// Below T = 768 a 1 x 256 layer gains once its own 256 x 256 units fill the
+// CTA pairs (13824 x 5120 at T = 512: 108 units, 0.85x; 11008 x 4096: 86
+// units, 1.20x).  The choice depends on the layer and T only, so a batched call
+// gives each layer the result gs_linear gives it, bit for bit (a choice by the
+// launch's total units would have sped the LLaMA-2-13B stack at T = 512 from
+// 12.33 to 10.76 ms per pass, at the price of that guarantee).
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
-  if (p->kept == 0 || p->g_out != 1) return false;
-  return (p->g_in == 128 && T > 128) || (p->g_in == 256 && T >= 768);
+  if (p->kept == 0 || p->g_out != 1 || T <= 128) return false;
+  if (p->g_in == 128) return true;
+  if (p->g_in != 256) return false;
+  const int64_t units = ((T + 255) / 256) * ((p->out + 255) / 256);
+  return T >= 768 || units * 10 >= 13 * (d_sm_count() / 2);
 }
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
