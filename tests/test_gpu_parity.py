@@ -200,7 +200,7 @@ def test_decode_batched_many_layers(gs, n):
     assert gs.device_status() == gs.GS_OK
 
 
-@pytest.mark.parametrize("n,T", [(3, 200), (11, 300)])
+@pytest.mark.parametrize("n,T", [(3, 200), (11, 300), (7, 1024)])   # T = 1024: the zero-filled kernel
 def test_prefill_batched_matches_single(gs, n, T):
     """A batched prefill call (several layers with one T share launches of up
     to 8 layers) gives bit for bit the single-layer results and stays within
