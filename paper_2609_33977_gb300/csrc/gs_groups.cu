@@ -58,6 +58,7 @@ constexpr int kSqEpiWarps = 4;
 constexpr int kSqThreads = (2 + kSqEpiWarps) * 32;
 constexpr int kSqMaxLayers = 8;
 constexpr int kSqDenseMaxG = 64;          // above the decode regime, g <= this takes the zero-filled kernel (7B block, T = 2048: 64x64 525 vs 476 TFLOP/s)
+constexpr int kSqDecodeMaxTokensZf = 32;  // decode regime of the layers the zero-filled kernel takes
 constexpr int kSqMaxMaps = 8;             // W slice heights g, 2g, ..., R g (R <= 8)
 constexpr uint64_t kSqWaitLimitNs = 2000000000ull;
 constexpr uint64_t kSqDrainLimitNs = 200000000ull;
@@ -712,43 +713,48 @@ gs_status sq_linear_batched(const void* const* xs, const gs_packed* const* ps, i
     std::stable_sort(o.begin(), o.end(), [&](int a, int b) {
       return (double)ps[a]->kept / ps[a]->nwin > (double)ps[b]->kept / ps[b]->nwin;
     });
-    // Decode regime: the tile-streaming kernel, one launch per 16 tokens, heaviest
-    // rows (widest input) first.  Its time grows with the 16-token blocks while
-    // the tensor-core kernel's stays flat up to 128 tokens; on the LLaMA-2 7B
-    // block shapes at d = 0.5 the blocks cost less up to 128 / 64 / 32 / 16
-    // tokens for g = 16 / 32 / 64 / 128.
+    // Per layer, by its group size, input width and T only (so a batched call
+    // gives each layer what a single call gives it):
+    //  - decode regime: the tile-streaming kernel, one launch per 16 tokens.  Its
+    //    time grows with the 16-token blocks while the tensor-core kernels' stays
+    //    flat up to 128 tokens.  Over the five LLaMA-2 7B / 13B projection shapes
+    //    at d = 0.5 the zero-filled-window kernel (layers whose input is whole
+    //    128-column items, g <= 64) takes 1.3-1.5x its time at 32 tokens,
+    //    0.90-1.03x at 48 and 0.37-0.43x at 128; the square tensor-core kernel
+    //    (the other layers) breaks even at 128 / 64 / 32 / 16 tokens for
+    //    g = 16 / 32 / 64 / 128;
+    //  - above it, the zero-filled-window kernel where it applies (dense-layer
+    //    tensor work, no per-column-block handshake: the faster of the two at
+    //    small tiles), else the square tensor-core kernel.
     const int g = 16 << gi;
-    if (T <= (int64_t)(2048 / g)) {
-      std::stable_sort(o.begin(), o.end(), [&](int a, int b) { return ps[a]->in > ps[b]->in; });
+    std::vector<int> dec, dense, rest;
+    for (int i : o) {
+      const bool zf = g <= kSqDenseMaxG && ps[i]->in % 128 == 0;
+      (T <= (zf ? (int64_t)kSqDecodeMaxTokensZf : (int64_t)(2048 / g)) ? dec : zf ? dense : rest).push_back(i);
+    }
+    if (!dec.empty()) {
+      std::stable_sort(dec.begin(), dec.end(), [&](int a, int b) { return ps[a]->in > ps[b]->in; });   // heaviest rows first
       const int blk = sq_decode_max_tokens();
       std::vector<const void*> xb(n);
       std::vector<void*> yb(n);
       for (int64_t t0 = 0; t0 < T; t0 += blk) {
         const int tb = (int)std::min<int64_t>(blk, T - t0);
-        for (int i : o) {
+        for (int i : dec) {
           xb[i] = static_cast<const uint16_t*>(xs[i]) + t0 * ps[i]->in;
           yb[i] = static_cast<uint16_t*>(ys[i]) + t0 * ps[i]->out;
         }
-        for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
-          const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
-          const gs_status st = sq_decode_batched(xb.data(), ps, o.data() + b0, nb, tb, yb.data(), s);
+        for (size_t b0 = 0; b0 < dec.size(); b0 += kSqMaxLayers) {
+          const int nb = (int)std::min<size_t>(kSqMaxLayers, dec.size() - b0);
+          const gs_status st = sq_decode_batched(xb.data(), ps, dec.data() + b0, nb, tb, yb.data(), s);
           if (st != GS_OK) return st;
         }
       }
-      continue;
     }
-    // Small tiles: the zero-filled-window tensor-core kernel (dense-layer tensor
-    // work, no per-column-block handshake) is the faster one; it takes the
-    // layers whose input is whole 128-column items, the others stay below
-    if (g <= kSqDenseMaxG) {
-      std::vector<int> dense, rest;
-      for (int i : o) (ps[i]->in % 128 == 0 ? dense : rest).push_back(i);
-      if (!dense.empty()) {
-        const gs_status st = launch_prefill_dense(xs, ps, (int)dense.size(), T, ys, s, dense.data());
-        if (st != GS_OK) return st;
-      }
-      o = rest;
+    if (!dense.empty()) {
+      const gs_status st = launch_prefill_dense(xs, ps, (int)dense.size(), T, ys, s, dense.data());
+      if (st != GS_OK) return st;
     }
+    o = rest;
     for (size_t b0 = 0; b0 < o.size(); b0 += kSqMaxLayers) {
       const int nb = (int)std::min<size_t>(kSqMaxLayers, o.size() - b0);
       gs_status st;

@@ -89,11 +89,11 @@ def test_prefill_wait_timeout_then_recovery(gs, T):
     assert gs.device_status() == gs.GS_OK
 
 
-@pytest.mark.parametrize("g", [0, 16])
-def test_prefill_dense_wait_timeout_then_recovery(gs, g):
-    # the zero-filled-window kernel: CTA pair 0 skips its units, then a clean launch matches the oracle
+@pytest.mark.parametrize("g,T", [(0, 300), (0, 64), (16, 300), (32, 100)])
+def test_prefill_dense_wait_timeout_then_recovery(gs, g, T):
+    # the zero-filled-window kernel: CTA pair 0 skips its units (at T = 64 and
+    # 100 the one token tile's first window), then a clean launch matches the oracle
     import torch
-    T = 300
     if g == 0:
         Wb, B, p = make(gs, 4096, 4096, 0.5, 75)
         gg = None
@@ -104,7 +104,8 @@ def test_prefill_dense_wait_timeout_then_recovery(gs, g):
         gg = g
     xb = wl.random_activation_bits(T, Wb.shape[1], seed=78 + g)
     x = to_dev(xb)
-    algo = gs.ALGO_PREFILL_DENSE if g == 0 else gs.ALGO_AUTO   # square 16x16 at T = 300: the same kernel
+    # squares 16x16 at T = 300 and 32x32 at T = 100: the same kernel
+    algo = gs.ALGO_PREFILL_DENSE if g == 0 else gs.ALGO_AUTO
     gs.debug_inject_wait(gs.ALGO_PREFILL_DENSE, 1_000_000)
     gs.linear(x, p, algo=algo)
     assert gs.device_status() == gs.GS_ERR_DEVICE_TIMEOUT

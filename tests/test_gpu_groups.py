@@ -65,7 +65,7 @@ def test_pack_and_unpack_are_bit_exact(gs, g, out, inp, d, seed):
 
 
 @pytest.mark.parametrize("g", [16, 32, 64, 128])
-@pytest.mark.parametrize("T", [1, 3, 8, 9, 16, 17, 64, 128, 129, 300])
+@pytest.mark.parametrize("T", [1, 3, 8, 9, 16, 17, 32, 33, 48, 64, 128, 129, 300])
 def test_linear_small_layers(gs, g, T):
     for out, inp, d, seed in [(256, 512, 0.5, 11), (384, 1024, 0.3, 12), (128, 128, 1.0, 13)]:
         Wb, B, p = make(gs, out, inp, g, d, seed)
