@@ -253,8 +253,10 @@ static gs_status linear_impl(const void* x_dev, const gs_packed* p, int64_t T, v
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (is_square(p)) return sq_linear_batched(&x_dev, &p, 1, T, &y_dev, s);   // one kernel family for every T
   if (algo == GS_ALGO_AUTO) {
-    algo = (T >= kPrefillMinTokens && p->G <= prefill_max_chunks()) ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
-    if (algo == GS_ALGO_PREFILL && prefill_prefers_dense(p, T)) algo = GS_ALGO_PREFILL_DENSE;
+    // the same per-layer choice as gs_linear_batched makes
+    if (T < kPrefillMinTokens) algo = GS_ALGO_DECODE;
+    else if (prefill_prefers_dense(p, T)) algo = GS_ALGO_PREFILL_DENSE;
+    else algo = p->G <= prefill_max_chunks() ? GS_ALGO_PREFILL : GS_ALGO_DECODE;
   }
   if (algo == GS_ALGO_PREFILL) return launch_prefill(x_dev, p, T, y_dev, s);
   if (algo == GS_ALGO_PREFILL_DENSE) {

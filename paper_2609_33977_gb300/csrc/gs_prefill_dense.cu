@@ -615,10 +615,14 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 // gives each layer the result gs_linear gives it, bit for bit (a choice by the
 // launch's total units would have sped the LLaMA-2-13B stack at T = 512 from
 // 12.33 to 10.76 ms per pass, at the price of that guarantee).
+// 1 x 128 layers take it from 33 tokens on: over the five LLaMA-2 7B / 13B
+// projection shapes at T = 64 and 128 it takes 0.91-0.96x the gathering
+// kernel's time in nine of the ten cases (13824 x 5120 at T = 128: 1.02x),
+// while 1 x 256 layers there stay on the gathering kernel (1.15-1.24x).
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
-  if (p->kept == 0 || p->g_out != 1 || T <= 128) return false;
+  if (p->kept == 0 || p->g_out != 1) return false;
   if (p->g_in == 128) return true;
-  if (p->g_in != 256) return false;
+  if (p->g_in != 256 || T <= 128) return false;
   const int64_t units = ((T + 255) / 256) * ((p->out + 255) / 256);
   return T >= 768 || units * 10 >= 13 * (d_sm_count() / 2);
 }
