@@ -237,11 +237,15 @@ def test_narrow_rows_batched_with_other_shapes(gs):
         B = wl.random_mask(1024 // go, 2048 // gi, 0.5, seed=90 + i)
         p = gs.pack_groups(to_dev(Wb), torch.from_numpy(B).cuda(), go, gi)
         layers.append((Wb, B, p, go, gi))
-    for T in (3, 16, 200, 1024):   # 1024: the 1 x 128 layers take the zero-filled prefill kernel
+    # 64 and 200: the 1 x 128 layers take the zero-filled prefill kernel, the 1 x 256 layer the
+    # gathering one and the 32 x 32 layer the zero-filled one (above its decode regime)
+    for T in (3, 16, 64, 200, 1024):
         xbs = [wl.random_activation_bits(T, 2048, seed=100 + i + T) for i in range(len(layers))]
         ys = [torch.empty((T, 1024), dtype=torch.bfloat16, device="cuda") for _ in layers]
         gs.linear_batched_into([to_dev(b) for b in xbs], [l[2] for l in layers], ys)
         for (Wb, B, p, go, gi), xb, y in zip(layers, xbs, ys):
             yr, A = orc.linear(xb, Wb, B, go, gi)
             assert np.all(np.abs(bf16_to_f64(to_bits(y)) - yr) <= REL * A + ABS), (go, gi, T)
+            # a batched call gives each layer what a single call gives it, bit for bit
+            assert np.array_equal(to_bits(y), to_bits(gs.linear(to_dev(xb), p))), (go, gi, T)
     assert gs.device_status() == gs.GS_OK

@@ -110,6 +110,45 @@ def test_prefill_dense_parity(gs, out, inp, d, seed):
     assert gs.device_status() == gs.GS_OK
 
 
+@pytest.mark.parametrize("go,gi", [(1, 256), (1, 128), (32, 32)])
+def test_prefill_dense_large_ragged_layers(gs, go, gi):
+    """Zero-filled kernel on ~10K-row layers at T ~ 1K (80+ units, more than one per CTA pair):
+    every element against the oracle, ragged rows and tokens, an empty window between non-empty
+    ones, and a batched call beside a small layer equal to single calls bit for bit."""
+    import torch
+    from tests._gpu_util import REL, ABS, bf16_to_f64
+    inp = 512
+    cases = []
+    for out, d, seed in ((10240, 0.5, 61), (10304, 0.3, 62)):   # 10304: a 64-row last window
+        Wb = wl.random_weight_bits(out, inp, seed=seed)
+        B = wl.random_mask(out // go, inp // gi, d, seed=seed + 1000)
+        if go == 1:
+            B[512:768, :] = 0    # window 2 empty, windows 1 and 3 not
+        else:
+            B[512 // go:768 // go, :] = 0
+        p = gs.pack_groups(to_dev(Wb), torch.from_numpy(np.ascontiguousarray(B, dtype=np.uint8)).cuda(), go, gi)
+        cases.append((Wb, B, p))
+    for T in (1000, 1024):
+        for Wb, B, p in cases:
+            xb = wl.random_activation_bits(T, inp, seed=T + Wb.shape[0])
+            y = to_bits(gs.linear(to_dev(xb), p, algo=gs.ALGO_PREFILL_DENSE if go == 1 else gs.ALGO_AUTO))
+            yr, A = orc.linear(xb, Wb, B, go, gi)
+            err = np.abs(bf16_to_f64(y) - yr)
+            assert np.all(err <= REL * A + ABS), (go, gi, Wb.shape, T, float((err / (REL * A + ABS)).max()))
+    # batched: the large layer beside a small layer of the same group shape
+    Ws = wl.random_weight_bits(512, inp, seed=63)
+    Bs = wl.random_mask(512 // go, inp // gi, 0.5, seed=64)
+    ps = gs.pack_groups(to_dev(Ws), torch.from_numpy(Bs).cuda(), go, gi)
+    T = 1024
+    layers = [(cases[0][0], cases[0][2]), (Ws, ps)]
+    xbs = [wl.random_activation_bits(T, inp, seed=70 + i) for i in range(2)]
+    ys = [torch.empty((T, W.shape[0]), dtype=torch.bfloat16, device="cuda") for W, _ in layers]
+    gs.linear_batched_into([to_dev(b) for b in xbs], [p for _, p in layers], ys)   # AUTO: zero-filled kernel at T = 1024
+    for (W, p), xb, y in zip(layers, xbs, ys):
+        assert np.array_equal(to_bits(y), to_bits(gs.linear(to_dev(xb), p)))
+    assert gs.device_status() == gs.GS_OK
+
+
 def test_auto_dispatch_and_empty_batch(gs):
     import torch
     Wb, B = layer(1024, 1024, 0.5, 4)
