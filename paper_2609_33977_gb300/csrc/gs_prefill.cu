@@ -113,6 +113,7 @@ struct PrefillParams {
   int32_t n_layers, T, n_tiles;
   int* err;
   uint64_t inject_ns;        // test hook: tile owner 0 first waits this long on a word nothing sets (0 = off)
+  TileList tl;               // which owner takes which tiles
 };
 
 // layer of global tile t
@@ -297,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
     uint32_t stage = 0, phase = 0;
     uint32_t armed = 0u, armed_par = 0u;   // per stage: a copy was issued / the phase it completes
     bool ok = true;
-    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, pair, n_pairs, kt)) >= 0; ++kt) {
       const PrefillLayer& L = P.L[tile_layer(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -355,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
     int buf = 0;
     uint32_t se_ph = 0u;   // bit b: parity of scratch buffer b's next release
     bool ok = true;
-    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, pair, n_pairs, kt)) >= 0; ++kt) {
       const PrefillLayer& L = P.L[tile_layer(P, t)];
       const int w = (t - L.tile_begin) / L.n_m;
       const int n_items = load_tile_items(L, w, lane, items);
@@ -432,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_prefill(const __grid_constant__
     int buf = 0;
     uint32_t sf_ph = 0u;   // bit b: parity of scratch buffer b's next fill
     bool ok = true;
-    for (int t = pair; t < n_tiles && ok; t += n_pairs) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, pair, n_pairs, kt)) >= 0; ++kt) {
       const PrefillLayer& L = P.L[tile_layer(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -666,9 +667,17 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
     P.n_tiles = (int32_t)tiles;
     P.err = err;
     P.inject_ns = b0 == 0 ? take_injected_wait(GS_ALGO_PREFILL) : 0;
+    const int owners = (int)std::min<int64_t>(tiles, pair ? max_pairs : (int64_t)sm_count());
+    if (tiles <= kTileListMax) {
+      // a tile's time follows its chunk count (measured flat in density)
+      std::vector<int32_t> cost((size_t)tiles);
+      for (int k = 0; k < nb; ++k)
+        for (int64_t t = 0; t < (int64_t)P.L[k].n_m * P.L[k].n_w; ++t) cost[(size_t)(P.L[k].tile_begin + t)] = P.L[k].G;
+      plan_tiles(cost, owners, P.tl);
+    }
     cudaError_t e;
     if (pair) {
-      const int grid = 2 * (int)(tiles < max_pairs ? tiles : max_pairs);   // CTA pairs: clusters of two
+      const int grid = 2 * owners;   // CTA pairs: clusters of two
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3((unsigned)grid);
       cfg.blockDim = dim3(kThreads);
@@ -683,8 +692,7 @@ gs_status launch_prefill_batched(const void* const* xs, const gs_packed* const* 
       cfg.numAttrs = 1;
       e = kw == 256 ? cudaLaunchKernelEx(&cfg, k_prefill<true, 256>, P) : cudaLaunchKernelEx(&cfg, k_prefill<true, 128>, P);
     } else {
-      const int64_t max_ctas = sm_count();
-      const int grid = (int)(tiles < max_ctas ? tiles : max_ctas);
+      const int grid = owners;
       if (kw == 256) k_prefill<false, 256><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
       else k_prefill<false, 128><<<grid, kThreads, kSmemBytesSingle, s>>>(P);
       e = cudaGetLastError();

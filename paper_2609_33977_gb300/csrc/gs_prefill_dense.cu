@@ -96,6 +96,7 @@ struct DParams {
   int32_t n_layers, T, n_tiles;
   int* err;
   uint64_t inject_ns;   // test hook: CTA pair 0 first waits this long on a word nothing sets (0 = off)
+  TileList tl;          // which pair takes which units
 };
 
 __device__ __forceinline__ int d_layer_of(const DParams& P, int t) {
@@ -231,7 +232,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     constexpr int kCopies = kRows / 4;            // 16-byte copies per lane per stage
     uint32_t stage = 0, phase = 0;
     bool ok = true;
-    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+    for (int ku = 0, u; ok && (u = owner_tile(P.tl, n_tiles, pair, n_pairs, ku)) >= 0; ++ku) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int w = (u - L.tile_begin) / L.n_m;
       const int j = lane & 7;   // 16-byte piece of a row this lane copies
@@ -345,7 +346,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     uint32_t k = 0;
     uint32_t armed = 0u, armed_par = 0u;
     bool ok = true;
-    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+    for (int ku = 0, u; ok && (u = owner_tile(P.tl, n_tiles, pair, n_pairs, ku)) >= 0; ++ku) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int lt = u - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -395,7 +396,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     const uint32_t f = warp == kDFwdWarp ? 0u : (uint32_t)(warp - kDXWarp);   // takes pairs p with p % kDNumFwd == f
     uint32_t K = 0;   // stages before the current batch
     bool ok = true;
-    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+    for (int ku = 0, u; ok && (u = owner_tile(P.tl, n_tiles, pair, n_pairs, ku)) >= 0; ++ku) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int w = (u - L.tile_begin) / L.n_m;
       for (int c0 = 0; c0 < L.G && ok; c0 += 32) {
@@ -440,7 +441,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     uint32_t ae_ph = 0u;
     bool ok = true;
     constexpr uint32_t idesc = idesc_bf16_f32(2 * kDM, kDW);
-    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+    for (int ku = 0, u; ok && (u = owner_tile(P.tl, n_tiles, pair, n_pairs, ku)) >= 0; ++ku) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int w = (u - L.tile_begin) / L.n_m;
       if (lane == 0) {
@@ -500,7 +501,7 @@ __global__ void __launch_bounds__(kDThreads, 1) k_prefill_dense(const __grid_con
     int buf = 0;
     uint32_t af_ph = 0u;
     bool ok = true;
-    for (int u = pair; u < n_tiles && ok; u += n_pairs) {
+    for (int ku = 0, u; ok && (u = owner_tile(P.tl, n_tiles, pair, n_pairs, ku)) >= 0; ++ku) {
       const DLayer& L = P.L[d_layer_of(P, u)];
       const int lt = u - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -679,8 +680,18 @@ gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps
     P.n_tiles = (int32_t)tiles;
     P.err = err;
     P.inject_ns = b0 == 0 ? take_injected_wait(GS_ALGO_PREFILL_DENSE) : 0;
+    const int owners = (int)std::min<int64_t>(tiles, max_pairs);
+    if (tiles <= kTileListMax) {
+      // a unit's time follows its item count (one launch holds one chunk width)
+      std::vector<int32_t> cost((size_t)tiles);
+      for (int k = 0; k < nb; ++k) {
+        const int64_t nu = (int64_t)P.L[k].n_m * ((ps[order[b0 + k]]->out + kDW - 1) / kDW);
+        for (int64_t t = 0; t < nu; ++t) cost[(size_t)(P.L[k].tile_begin + t)] = P.L[k].G;
+      }
+      plan_tiles(cost, owners, P.tl);
+    }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(2 * std::min<int64_t>(tiles, max_pairs)));
+    cfg.gridDim = dim3((unsigned)(2 * owners));
     cfg.blockDim = dim3(kDThreads);
     cfg.dynamicSmemBytes = kDSmem;
     cfg.stream = s;
