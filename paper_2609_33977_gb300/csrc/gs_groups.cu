@@ -101,6 +101,7 @@ struct SqParams {
   int32_t n_layers, T, n_tiles;
   int32_t x_rows;            // rows of each x box: min(T, 128) (token rows past it hold stale data, never stored)
   int* err;
+  TileList tl;               // which owner takes which tiles
 };
 
 __device__ __forceinline__ int sq_layer_of(const SqParams& P, int t) {
@@ -207,7 +208,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
     uint32_t stage = 0, phase = 0;
     uint32_t armed = 0u, armed_par = 0u;
     bool ok = true;
-    for (int t = owner; t < n_tiles && ok; t += n_owners) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, owner, n_owners, kt)) >= 0; ++kt) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -280,7 +281,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
     bool ok = true;
     constexpr uint32_t idesc = idesc_bf16_f32(kPair ? 2 * kSqM : kSqM, G);
     constexpr int kTileRows = kPair ? G / 2 : G;   // rows of each tile this CTA holds
-    for (int t = owner; t < n_tiles && ok; t += n_owners) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, owner, n_owners, kt)) >= 0; ++kt) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int w = (t - L.tile_begin) / L.n_m;
       if (lane == 0) {
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(kSqThreads, 1) k_sq(const __grid_constant__ Sq
     int buf = 0;
     uint32_t af_ph = 0u;
     bool ok = true;
-    for (int t = owner; t < n_tiles && ok; t += n_owners) {
+    for (int kt = 0, t; ok && (t = owner_tile(P.tl, n_tiles, owner, n_owners, kt)) >= 0; ++kt) {
       const SqLayer& L = P.L[sq_layer_of(P, t)];
       const int lt = t - L.tile_begin;
       const int m = lt % L.n_m, w = lt / L.n_m;
@@ -560,11 +561,21 @@ gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int
   P.n_tiles = (int32_t)tiles;
   P.x_rows = (int32_t)xr;
   P.err = err;
+  const int owners = (int)std::min<int64_t>(tiles, kPair ? sq_sm_count() / 2 : sq_sm_count());
+  if (tiles <= kTileListMax) {
+    // a tile's time follows the kept tiles of its window: the layer's mean
+    std::vector<int32_t> cost((size_t)tiles);
+    for (int k = 0; k < nb; ++k) {
+      const gs_packed* p = ps[idx[k]];
+      const int32_t c = (int32_t)((p->kept + p->nwin - 1) / std::max<int64_t>(p->nwin, 1));
+      for (int64_t t = 0; t < (int64_t)P.L[k].n_m * P.L[k].nwin; ++t) cost[(size_t)(P.L[k].tile_begin + t)] = c;
+    }
+    plan_tiles(cost, owners, P.tl);
+  }
   cudaError_t e;
   if constexpr (kPair) {
-    const int64_t pairs = std::min<int64_t>(tiles, sq_sm_count() / 2);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(2 * pairs));
+    cfg.gridDim = dim3((unsigned)(2 * owners));
     cfg.blockDim = dim3(kSqThreads);
     cfg.dynamicSmemBytes = C::kSmem;
     cfg.stream = s;
@@ -577,8 +588,7 @@ gs_status sq_launch(const void* const* xs, const gs_packed* const* ps, const int
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, k_sq<G, true>, P);
   } else {
-    const int grid = (int)std::min<int64_t>(tiles, sq_sm_count());
-    k_sq<G, false><<<grid, kSqThreads, C::kSmem, s>>>(P);
+    k_sq<G, false><<<owners, kSqThreads, C::kSmem, s>>>(P);
     e = cudaGetLastError();
   }
   note_launch();
