@@ -53,9 +53,8 @@ typedef enum gs_algo {
   GS_ALGO_PREFILL = 2,  /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
   GS_ALGO_PREFILL_DENSE = 3  /* tcgen05 kernel over zero-filled 256-row windows: tensor
                                 work of the dense layer, no gather; 1 x 128 and 1 x 256
-                                groups; GS_ALGO_AUTO picks it for T > 128 (1 x 128;
-                                1 x 256: from T = 768, or when the layer holds enough
-                                256 x 256 units to fill the GPU)                       */
+                                groups; GS_ALGO_AUTO picks it from T = 33 (1 x 128)
+                                and from T = 129 (1 x 256)                             */
 } gs_algo;
 
 typedef struct gs_packed gs_packed;   /* opaque, library-owned */

@@ -604,28 +604,26 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 
 }  // namespace
 
-// Measured on GB300 at d = 0.5 (LLaMA-2 7B / 13B projection shapes, time
-// relative to the gathering kernel): 1 x 128 groups 0.47-0.95x at every T from
-// 256 to 2048; 1 x 256 groups 0.66-0.92x from T = 768 up, while at T <= 512
-// only the 13824 x 5120 layer gains (0.73-0.85x) and the smaller ones lose
-// (1.12-1.24x: too few 256 x 256 units for the CTA pairs).  Both kernels' times
-// hardly depend on the density.
-// Below T = 768 a 1 x 256 layer gains once its own 256 x 256 units fill the
-// CTA pairs (13824 x 5120 at T = 512: 108 units, 0.85x; 11008 x 4096: 86
-// units, 1.20x).  The choice depends on the layer and T only, so a batched call
-// gives each layer the result gs_linear gives it, bit for bit (a choice by the
-// launch's total units would have sped the LLaMA-2-13B stack at T = 512 from
-// 12.33 to 10.76 ms per pass, at the price of that guarantee).
-// 1 x 128 layers take it from 33 tokens on: over the five LLaMA-2 7B / 13B
-// projection shapes at T = 64 and 128 it takes 0.91-0.96x the gathering
-// kernel's time in nine of the ten cases (13824 x 5120 at T = 128: 1.02x),
-// while 1 x 256 layers there stay on the gathering kernel (1.15-1.24x).
+// Which 1 x KW layers take this kernel rather than the gathering one, by the
+// layer's own group shape and T (so that a batched call gives each layer what
+// gs_linear gives it, bit for bit).  Measured on GB300 at d = 0.5 with the
+// balanced tile lists, one batched call per block (7 projections):
+//  - 1 x 256 from 129 tokens: LLaMA-2-13B block 0.142 / 0.144 / 0.236 / 0.330
+//    ms at T = 160 / 256 / 512 / 640 against 0.172 / 0.173 / 0.294 / 0.426 with
+//    the gathering kernel for the 5120-row layers (7B block 0.101-0.220 against
+//    0.117-0.299; Qwen2.5-7B 0.180-0.249 against 0.217-0.304 from T = 384, 4 %
+//    behind at 160 and 256).  Alone, a 5120 x 5120 layer at T = 512 still runs
+//    faster gathering (0.040 vs 0.048 ms: 40 units for 76 CTA pairs), but layers
+//    are mostly called a block at a time;
+//  - 1 x 128 from 33 tokens: over the five 7B / 13B projection shapes at T = 64
+//    and 128 it takes 0.91-0.96x the gathering kernel's time in nine of the ten
+//    cases (13824 x 5120 at T = 128: 1.02x), while 1 x 256 layers up to 128
+//    tokens stay on the gathering kernel (1.15-1.24x).
+// Both kernels' times hardly depend on the density.
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
   if (p->kept == 0 || p->g_out != 1) return false;
   if (p->g_in == 128) return true;
-  if (p->g_in != 256 || T <= 128) return false;
-  const int64_t units = ((T + 255) / 256) * ((p->out + 255) / 256);
-  return T >= 768 || units * 10 >= 13 * (d_sm_count() / 2);
+  return p->g_in == 256 && T > 128;
 }
 
 gs_status launch_prefill_dense(const void* const* xs, const gs_packed* const* ps, int n, int64_t T, void* const* ys,
