@@ -149,6 +149,20 @@ def test_prefill_dense_large_ragged_layers(gs, go, gi):
     assert gs.device_status() == gs.GS_OK
 
 
+def test_prefill_more_tiles_than_the_tile_list(gs):
+    """Launches with more tiles than the balanced tile list holds (2048) fall back to the fixed
+    stride: a 41120-row layer on the gathering kernel (8 x 257 tiles) and a 65792-row layer on the
+    zero-filled kernel (8 x 257 units) at T = 2048, sampled tokens against the oracle."""
+    T = 2048
+    for out, algo, seed in ((41120, gs.ALGO_PREFILL, 65), (65792, gs.ALGO_PREFILL_DENSE, 66)):
+        Wb, B = layer(out, 256, 0.5, seed)
+        p = packed(gs, Wb, B)
+        xb = wl.random_activation_bits(T, 256, seed=seed + 7)
+        y = to_bits(gs.linear(to_dev(xb), p, algo=algo))
+        assert_within_bound(y, xb, Wb, B, tokens=sample_tokens(T, seed=seed), what=f"{out} rows algo {algo}")
+    assert gs.device_status() == gs.GS_OK
+
+
 def test_auto_dispatch_and_empty_batch(gs):
     import torch
     Wb, B = layer(1024, 1024, 0.5, 4)
