@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(kQdThreads) k_sq_decode(const __grid_constant_
 
   for (int v0 = va; v0 < vb; v0 += kQdListMax) {
     const int v1 = min(v0 + kQdListMax, vb);
-    // kept column blocks of this round, in ascending order (the block row's
+    // kept column blocks of this batch (v0 .. v1 - 1), in ascending order (the block row's
     // tile indices are contiguous: all loads go out before the first use)
     constexpr int kLd = kQdListMax / 32;
     int tv[kLd];
