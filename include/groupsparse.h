@@ -53,7 +53,7 @@ typedef enum gs_algo {
   GS_ALGO_PREFILL = 2,  /* tcgen05/TMEM/TMA tensor-core kernel (compute-bound)        */
   GS_ALGO_PREFILL_DENSE = 3  /* tcgen05 kernel over zero-filled 256-row windows: tensor
                                 work of the dense layer, no gather; 1 x 128 and 1 x 256
-                                groups; GS_ALGO_AUTO picks it from T = 33 (1 x 128)
+                                groups; GS_ALGO_AUTO picks it from T = 17 (1 x 128)
                                 and from T = 129 (1 x 256)                             */
 } gs_algo;
 
@@ -151,7 +151,7 @@ gs_status gs_linear_ex(const void* x_dev, const gs_packed* p, int64_t T, void* y
  * gs_linear_batched - n independent layers, ys[i] = xs[i] W_hat_i^T for the
  * i-th handle, all with the same token count T.  In the decode regime all n
  * layers share one launch per 16 tokens (one grid streams every layer's kept
- * groups); in the prefill regime (T >= 33) up to 8 layers share one launch
+ * groups); in the prefill regime (T >= 17) up to 8 layers share one launch
  * (one list of output tiles).  Results are those of gs_linear for each layer
  * (prefill: bit for bit).  Same per-layer semantics and errors as gs_linear.
  * 1 <= n <= 32 (n == 0 is a no-op); the handles must be distinct.

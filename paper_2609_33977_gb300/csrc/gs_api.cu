@@ -23,8 +23,12 @@ std::atomic<uint64_t> g_timeout_epoch{0};
 std::atomic<int64_t> g_fail_alloc_in{0};
 std::atomic<uint64_t> g_inject_ns[4] = {{0}, {0}, {0}, {0}};
 
-// Token count at and above which gs_linear uses the tensor-core kernel.
-constexpr int64_t kPrefillMinTokens = 33;
+// Token count at and above which gs_linear uses the tensor-core kernels: one
+// decode launch covers up to 16 tokens, while the tensor-core kernels' time is
+// flat up to 128.  At T = 17 / 24 / 32 a batched LLaMA-2-13B block takes
+// 0.098 ms there against 0.144-0.156 ms as two decode launches (7B 0.073 vs
+// 0.097-0.107; Qwen2.5-7B even), and one call per layer 0.30 against 0.38-0.49.
+constexpr int64_t kPrefillMinTokens = 17;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

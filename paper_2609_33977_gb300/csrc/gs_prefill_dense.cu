@@ -615,10 +615,10 @@ cudaError_t d_launch(const cudaLaunchConfig_t& cfg, const DParams& P) {
 //    behind at 160 and 256).  Alone, a 5120 x 5120 layer at T = 512 still runs
 //    faster gathering (0.040 vs 0.048 ms: 40 units for 76 CTA pairs), but layers
 //    are mostly called a block at a time;
-//  - 1 x 128 from 33 tokens: over the five 7B / 13B projection shapes at T = 64
-//    and 128 it takes 0.91-0.96x the gathering kernel's time in nine of the ten
-//    cases (13824 x 5120 at T = 128: 1.02x), while 1 x 256 layers up to 128
-//    tokens stay on the gathering kernel (1.15-1.24x).
+//  - 1 x 128 in the whole prefill regime: over the five 7B / 13B projection
+//    shapes at T = 64 and 128 it takes 0.91-0.96x the gathering kernel's time in
+//    nine of the ten cases (13824 x 5120 at T = 128: 1.02x), while 1 x 256
+//    layers up to 128 tokens stay on the gathering kernel (1.15-1.24x).
 // Both kernels' times hardly depend on the density.
 bool prefill_prefers_dense(const gs_packed* p, int64_t T) {
   if (p->kept == 0 || p->g_out != 1) return false;

@@ -167,7 +167,7 @@ def test_auto_dispatch_and_empty_batch(gs):
     import torch
     Wb, B = layer(1024, 1024, 0.5, 4)
     p = packed(gs, Wb, B)
-    for T in (1, 16, 32, 33, 200):
+    for T in (1, 16, 17, 24, 32, 33, 200):   # decode up to 16 tokens, tensor-core kernels from 17
         xb = wl.random_activation_bits(T, 1024, seed=T)
         assert_within_bound(to_bits(gs.linear(to_dev(xb), p)), xb, Wb, B, what=f"auto T={T}")
     x0 = torch.empty((0, 1024), dtype=torch.bfloat16, device="cuda")
