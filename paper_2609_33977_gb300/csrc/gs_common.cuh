@@ -8,6 +8,7 @@
 #include <cstddef>
 
 #include "groupsparse.h"
+#include "gs_plan.cuh"
 
 namespace gs {
 
@@ -108,19 +109,7 @@ gs_status lib_malloc(void** ptr, size_t bytes);
 // Reading it disarms it.
 uint64_t take_injected_wait(int family);
 
-// Tile assignment of the persistent tensor-core kernels.  A launch's tiles
-// differ in cost (a layer's tile walks all of its chunks, and wide-input layers
-// have 2-3x more), so a fixed stride over the tile list can leave a few owners
-// (CTAs or CTA pairs) with twice the mean.  Owner b takes
-// order[off[b]] .. order[off[b + 1] - 1]; on == 0: tiles b, b + owners, ...
-constexpr int kTileListMax = 2048;
-constexpr int kTileOwnersMax = 160;
-struct TileList {
-  uint16_t order[kTileListMax];
-  uint16_t off[kTileOwnersMax + 1];
-  int32_t on;
-};
-// The k-th tile of owner b, or -1 when it has no more.
+// The k-th tile of owner b, or -1 when it has no more (TileList: gs_plan.cuh).
 __device__ __forceinline__ int owner_tile(const TileList& L, int n_tiles, int b, int n_owners, int k) {
   if (L.on) {
     const int i = (int)L.off[b] + k;
@@ -129,10 +118,6 @@ __device__ __forceinline__ int owner_tile(const TileList& L, int n_tiles, int b,
   const int t = b + k * n_owners;
   return t < n_tiles ? t : -1;
 }
-// Longest tile first to the least-loaded owner (ties: the lowest owner);
-// cost[t] of each tile in list order.  Leaves on == 0 when the launch has more
-// tiles or owners than the list holds.
-void plan_tiles(const std::vector<int32_t>& cost, int n_owners, TileList& L);
 
 // pack.cu
 gs_status launch_pack_count_scan(const uint8_t* mask, gs_packed* p, cudaStream_t s, int32_t* cnt_tmp);
